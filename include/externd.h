@@ -1,0 +1,125 @@
+/*
+ * externd.h — C ABI of the GB300 ExTernD factorization library (libexternd.so).
+ *
+ * ExTernD (Expanded-Rank Ternary Decomposition, arxiv 2607.13511) approximates a real matrix A (m x n) as
+ *     A ~ B diag(D) C,   B in {-1,0,+1}^{m x k},  C in {-1,0,+1}^{k x n},  D in R^k          (§2.1, Eq. 1)
+ * with an inner rank k = mu * min(m, n) expanded past full rank, fitted greedily: components one at a time
+ * (§2.3) or in blocks of b components with decorrelated targets (§2.4, Eq. 3) and jointly solved scales
+ * (Eq. 4), optionally under per-column importance weights with the plain-residual V-step (§2.5).
+ *
+ * Conventions shared by every entry point
+ *   - Matrices are C-contiguous, row-major. All array pointers are CUDA device pointers (memory that the
+ *     current device can address: cudaMalloc'd, managed, or mapped pinned), owned by the caller, except where
+ *     a function says "host". The library never frees caller memory.
+ *   - B and the block factor U are int8 {-1,0,+1}; C and the block factor Cb are int8 {-1,0,+1}; real arrays
+ *     are float32; energies are double.
+ *   - Work is enqueued on the stream set with externd_set_stream (default: the legacy NULL stream). Functions
+ *     that return a double through a host pointer synchronize that stream before returning; the others only
+ *     enqueue work.
+ *   - Return value: EXTERND_OK (0) on success, a negative EXTERND_E* code on failure; on failure the output
+ *     arrays hold unspecified values. externd_strerror turns a code into a message.
+ *   - The library allocates its own device workspace (kept between calls, per device); EXTERND_ENOMEM reports
+ *     a failed allocation. Calls from several host threads are serialised inside the library.
+ *   - Importance weights ("weights", length n) are h~ of §2.5 (the caller forms h/max(h) + lambda); every
+ *     weight must be finite and > 0. NULL means unweighted (h~ = 1).
+ */
+#ifndef EXTERND_H
+#define EXTERND_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define EXTERND_OK 0
+#define EXTERND_EINVAL (-1)   /* bad size, parameter or NULL pointer                                  */
+#define EXTERND_EPTR (-2)     /* a pointer that must be device memory is not accessible from the device */
+#define EXTERND_ENOMEM (-3)   /* device workspace allocation failed                                   */
+#define EXTERND_ECUDA (-4)    /* a CUDA call or kernel launch failed (message: externd_last_cuda_error) */
+#define EXTERND_ENODEV (-5)   /* no usable CUDA device / unsupported architecture                       */
+
+/* Message for a status code (static string, never NULL). */
+const char *externd_strerror(int status);
+
+/* Text of the last CUDA error seen by the library in this process (static buffer, never NULL). */
+const char *externd_last_cuda_error(void);
+
+/* Library version string. */
+const char *externd_version(void);
+
+/* Stream used by every later call (a cudaStream_t; NULL = legacy default stream). */
+int externd_set_stream(void *cuda_stream);
+
+/* §2.1: inner rank k = floor(mu * min(m, n) + 0.5) for m, n >= 1 and mu > 0 (host only). */
+int externd_rank(int64_t m, int64_t n, double mu, int64_t *k);
+
+/* §2.4: block width b = min(block, floor(min(m, n) / 8)), at least 1 (host only). */
+int externd_block_width(int64_t m, int64_t n, int block, int *b);
+
+/*
+ * The whole method (§2.3 when the block width is 1, §2.4 otherwise; §2.5 when weights != NULL).
+ *   A        m x n float32, read only.
+ *   mu > 0   rank multiplier; k = externd_rank(m, n, mu).   tau >= 0: Eq. 2 threshold scale.
+ *   block >= 1 requested block width (clamped as externd_block_width; the last block is k mod b wide when
+ *            that is non-zero).   iters >= 1: ALS iterations per component/block (one V-step + one U-step).
+ *   weights  n float32 or NULL.
+ *   B        m x k int8 out;  D  k float32 out;  C  k x n int8 out.
+ *   energy   host double out: E = 1 - ||R||^2 / ||A||^2 (weighted by h~ when weights != NULL, §2.5) from the
+ *            final residual R = A - B diag(D) C kept in float32 on the device.
+ *   trace    host double[nblocks] out or NULL: the energy after each block (nblocks = ceil(k / b)).
+ */
+int externd_decompose(const float *A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
+                      const float *weights, int8_t *B, float *D, int8_t *C, double *energy, double *trace);
+
+/* Same as externd_decompose with every array in HOST memory (pageable or pinned): the library copies A and
+ * weights to the device, runs the method, and copies B, D, C back before returning. */
+int externd_decompose_host(const float *A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
+                           const float *weights, int8_t *B, float *D, int8_t *C, double *energy, double *trace);
+
+/* Eq. 1 (weighted form of §2.5): energy = 1 - sum_ij h_j (A - B diag(D) C)_ij^2 / sum_ij h_j A_ij^2, with B
+ * m x k, D k, C k x n on the device; energy is a host double. */
+int externd_energy(const float *A, int64_t m, int64_t n, const int8_t *B, const float *D, const int8_t *C,
+                   int64_t k, const float *weights, double *energy);
+
+/* ---------------------------------------------------------------------------------------------------------
+ * Single steps of the method, exposed for checking each kernel on its own. U is m x w int8 (a block of B's
+ * columns, row-major m x w), Cb is w x n int8 (a block of C's rows). 1 <= w <= 1024.
+ * ------------------------------------------------------------------------------------------------------- */
+
+/* Eq. 2 on every vector of X (rows x cols float32): axis = 1 ternarizes each row (length cols), axis = 0 each
+ * column (length rows). T (rows x cols int8) receives T_tau: sign(x_i) * [|x_i| > tau * mean_j |x_j|], and the
+ * single largest-magnitude entry (first index; +1 when it is 0) when nothing passes. */
+int externd_ternarize(const float *X, int64_t rows, int64_t cols, int axis, double tau, int8_t *T);
+
+/* §2.3 step 1 / §2.4: the V-step residual product PV = U^T R (w x n float32). Plain R even when weighted. */
+int externd_vstep_product(const float *R, int64_t m, int64_t n, const int8_t *U, int64_t w, float *PV);
+
+/* §2.3 step 1 / §2.5: the U-step residual product PU = R diag(h~) Cb^T (m x w float32). */
+int externd_ustep_product(const float *R, int64_t m, int64_t n, const int8_t *Cb, int64_t w, const float *weights,
+                          float *PU);
+
+/* Eq. 3 (left): X = (U^T U + eps I)^-1 U^T R (w x n float32), eps = 1e-4 * trace(U^T U) / w. Row a of X is
+ * the V target of component a (for w = 1 the product itself: T_tau is invariant to positive scaling). */
+int externd_vstep_target(const float *R, int64_t m, int64_t n, const int8_t *U, int64_t w, float *X);
+
+/* Eq. 3 (right) with §2.5: Y = R H V (V^T H V + eps I)^-1 (m x w float32), V = Cb^T, H = diag(h~),
+ * eps = 1e-4 * trace(V^T H V) / w (for w = 1 the product itself). */
+int externd_ustep_target(const float *R, int64_t m, int64_t n, const int8_t *Cb, int64_t w, const float *weights,
+                         float *Y);
+
+/* Eq. 4 with §2.5: d (w float32) solves [(U^T U) .* (V^T H V) + eps I] d = diag(U^T R H V); eps = 0 for w = 1
+ * (Prop. 1's scale u^T R H v / (||u||^2 v^T H v)) and 1e-4 * trace / w otherwise. */
+int externd_block_scales(const float *R, int64_t m, int64_t n, const int8_t *U, const int8_t *Cb, int64_t w,
+                         const float *weights, float *d);
+
+/* §2.3 step 3 / §2.4: R <- R - U diag(d) Cb in place (R m x n float32). If norm2 != NULL it receives (host)
+ * sum_ij h_j R_ij^2 of the updated residual. */
+int externd_deflate(float *R, int64_t m, int64_t n, const int8_t *U, const float *d, const int8_t *Cb, int64_t w,
+                    const float *weights, double *norm2);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EXTERND_H */

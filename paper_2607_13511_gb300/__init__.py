@@ -1,0 +1,274 @@
+"""GB300-native ExTernD: ternary expanded-rank factorization A ~ B diag(D) C on one GPU.
+
+Thin Python binding of libexternd.so (the C ABI in include/externd.h). Every function here only marshals
+arguments: it allocates result tensors with PyTorch on the current CUDA device, passes raw pointers and the current
+stream to the library, and raises ``ExterndError`` on a non-zero status. All arithmetic runs in the library's CUDA
+kernels; there is no CPU fallback. If the library has not been built, the first call raises ``ExterndError``
+(build it with ``python -m paper_2607_13511_gb300.build`` or ``__graft_entry__.build()``).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+__all__ = [
+    "ExterndError", "Decomposition", "library_path", "load", "rank", "block_width", "decompose", "decompose_host",
+    "energy", "ternarize", "vstep_product", "ustep_product", "vstep_target", "ustep_target", "block_scales",
+    "deflate",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB: Optional[ctypes.CDLL] = None
+
+_c_i64, _c_int, _c_double, _c_void = ctypes.c_int64, ctypes.c_int, ctypes.c_double, ctypes.c_void_p
+_c_dptr = ctypes.POINTER(ctypes.c_double)
+
+# name -> (restype, argtypes); mirrors include/externd.h
+_SIGNATURES = {
+    "externd_strerror": (ctypes.c_char_p, [_c_int]),
+    "externd_last_cuda_error": (ctypes.c_char_p, []),
+    "externd_version": (ctypes.c_char_p, []),
+    "externd_set_stream": (_c_int, [_c_void]),
+    "externd_rank": (_c_int, [_c_i64, _c_i64, _c_double, ctypes.POINTER(_c_i64)]),
+    "externd_block_width": (_c_int, [_c_i64, _c_i64, _c_int, ctypes.POINTER(_c_int)]),
+    "externd_decompose": (_c_int, [_c_void, _c_i64, _c_i64, _c_double, _c_double, _c_int, _c_int, _c_void,
+                                   _c_void, _c_void, _c_void, _c_dptr, _c_dptr]),
+    "externd_decompose_host": (_c_int, [_c_void, _c_i64, _c_i64, _c_double, _c_double, _c_int, _c_int, _c_void,
+                                        _c_void, _c_void, _c_void, _c_dptr, _c_dptr]),
+    "externd_energy": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_void, _c_i64, _c_void, _c_dptr]),
+    "externd_ternarize": (_c_int, [_c_void, _c_i64, _c_i64, _c_int, _c_double, _c_void]),
+    "externd_vstep_product": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_i64, _c_void]),
+    "externd_ustep_product": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_i64, _c_void, _c_void]),
+    "externd_vstep_target": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_i64, _c_void]),
+    "externd_ustep_target": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_i64, _c_void, _c_void]),
+    "externd_block_scales": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_i64, _c_void, _c_void]),
+    "externd_deflate": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_void, _c_i64, _c_void, _c_dptr]),
+}
+
+
+class ExterndError(RuntimeError):
+    """A non-zero status from libexternd, or the library missing."""
+
+
+def library_path() -> str:
+    return os.path.join(_HERE, "_build", "libexternd.so")
+
+
+def load() -> ctypes.CDLL:
+    """Loads libexternd.so (once) and declares the C signatures."""
+    global _LIB
+    if _LIB is None:
+        path = library_path()
+        if not os.path.exists(path):
+            raise ExterndError(f"libexternd.so is not built ({path}); run python -m paper_2607_13511_gb300.build")
+        lib = ctypes.CDLL(path)
+        for name, (res, args) in _SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.restype, fn.argtypes = res, args
+        _LIB = lib
+    return _LIB
+
+
+def _check(status: int) -> None:
+    if status != 0:
+        lib = load()
+        msg = lib.externd_strerror(status).decode()
+        if status == -4:
+            msg += ": " + lib.externd_last_cuda_error().decode()
+        raise ExterndError(f"libexternd status {status}: {msg}")
+
+
+def _torch():
+    import torch
+    return torch
+
+
+def _ptr(t) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _prep(t, dtype, name):
+    torch = _torch()
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ExterndError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ExterndError(f"{name} must be {dtype}, got {t.dtype}")
+    return t.contiguous()
+
+
+def _stream(lib, device) -> None:
+    torch = _torch()
+    lib.externd_set_stream(ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream))
+
+
+def rank(m: int, n: int, mu: float) -> int:
+    """§2.1 inner rank k = floor(mu * min(m, n) + 0.5)."""
+    k = _c_i64()
+    _check(load().externd_rank(m, n, mu, ctypes.byref(k)))
+    return k.value
+
+
+def block_width(m: int, n: int, block: int) -> int:
+    """§2.4 block width min(block, floor(min(m, n)/8)), at least 1."""
+    b = _c_int()
+    _check(load().externd_block_width(m, n, block, ctypes.byref(b)))
+    return b.value
+
+
+@dataclass
+class Decomposition:
+    B: "object"          # m x k int8 {-1, 0, 1}
+    D: "object"          # k float32
+    C: "object"          # k x n int8 {-1, 0, 1}
+    energy: float        # 1 - ||A - B diag(D) C||_H^2 / ||A||_H^2 (tracked residual)
+    trace: list          # energy after each block
+
+
+def decompose(A, mu: float, tau: float, block: int, iters: int, weights=None, out=None) -> Decomposition:
+    """ExTernD of a CUDA float32 matrix A (m x n): §2.3 (block 1) / §2.4 block ALS, §2.5 when weights is given.
+
+    ``out`` may pass preallocated (B, D, C) tensors to reuse."""
+    torch = _torch()
+    lib = load()
+    A = _prep(A, torch.float32, "A")
+    m, n = A.shape
+    k = rank(m, n, mu)
+    nblocks = -(-k // block_width(m, n, block))
+    h = None if weights is None else _prep(weights, torch.float32, "weights")
+    if out is None:
+        B = torch.empty((m, k), dtype=torch.int8, device=A.device)
+        D = torch.empty((k,), dtype=torch.float32, device=A.device)
+        C = torch.empty((k, n), dtype=torch.int8, device=A.device)
+    else:
+        B, D, C = out
+    e = _c_double()
+    tr = (_c_double * nblocks)()
+    with torch.cuda.device(A.device):
+        _stream(lib, A.device)
+        _check(lib.externd_decompose(_ptr(A), m, n, mu, tau, block, iters, _ptr(h), _ptr(B), _ptr(D), _ptr(C),
+                                     ctypes.byref(e), tr))
+    return Decomposition(B, D, C, e.value, list(tr))
+
+
+def decompose_host(A, mu: float, tau: float, block: int, iters: int, weights=None, out=None) -> Decomposition:
+    """Same as ``decompose`` for a host (CPU) float32 tensor: copies in and out happen inside the library call."""
+    torch = _torch()
+    lib = load()
+    if A.is_cuda or A.dtype != torch.float32:
+        raise ExterndError("A must be a CPU float32 tensor")
+    A = A.contiguous()
+    m, n = A.shape
+    k = rank(m, n, mu)
+    nblocks = -(-k // block_width(m, n, block))
+    h = None if weights is None else weights.contiguous()
+    if out is None:
+        pin = torch.cuda.is_available()
+        B = torch.empty((m, k), dtype=torch.int8, pin_memory=pin)
+        D = torch.empty((k,), dtype=torch.float32, pin_memory=pin)
+        C = torch.empty((k, n), dtype=torch.int8, pin_memory=pin)
+    else:
+        B, D, C = out
+    e = _c_double()
+    tr = (_c_double * nblocks)()
+    _stream(lib, torch.cuda.current_device())
+    _check(lib.externd_decompose_host(_ptr(A), m, n, mu, tau, block, iters, _ptr(h), _ptr(B), _ptr(D), _ptr(C),
+                                      ctypes.byref(e), tr))
+    return Decomposition(B, D, C, e.value, list(tr))
+
+
+def energy(A, B, D, C, weights=None) -> float:
+    """Eq. 1 (weighted per §2.5): 1 - ||A - B diag(D) C||_H^2 / ||A||_H^2 computed from the factors."""
+    torch = _torch()
+    lib = load()
+    A = _prep(A, torch.float32, "A")
+    B, D, C = _prep(B, torch.int8, "B"), _prep(D, torch.float32, "D"), _prep(C, torch.int8, "C")
+    h = None if weights is None else _prep(weights, torch.float32, "weights")
+    m, n = A.shape
+    e = _c_double()
+    with torch.cuda.device(A.device):
+        _stream(lib, A.device)
+        _check(lib.externd_energy(_ptr(A), m, n, _ptr(B), _ptr(D), _ptr(C), D.numel(), _ptr(h), ctypes.byref(e)))
+    return e.value
+
+
+def ternarize(X, tau: float, axis: int = 1):
+    """Eq. 2 on each row (axis=1) or column (axis=0) of a CUDA float32 matrix; returns int8."""
+    torch = _torch()
+    lib = load()
+    X = _prep(X, torch.float32, "X")
+    T = torch.empty(X.shape, dtype=torch.int8, device=X.device)
+    with torch.cuda.device(X.device):
+        _stream(lib, X.device)
+        _check(lib.externd_ternarize(_ptr(X), X.shape[0], X.shape[1], axis, tau, _ptr(T)))
+    return T
+
+
+def _step(fn_name, R, F, w_from, out_shape, weights=None, extra=()):
+    torch = _torch()
+    lib = load()
+    R = _prep(R, torch.float32, "R")
+    F = _prep(F, torch.int8, "factor")
+    m, n = R.shape
+    out = torch.empty(out_shape(m, n, w_from(F)), dtype=torch.float32, device=R.device)
+    with torch.cuda.device(R.device):
+        _stream(lib, R.device)
+        args = [_ptr(R), m, n, _ptr(F), w_from(F)]
+        if weights is not False:
+            args.append(_ptr(None if weights is None else _prep(weights, torch.float32, "weights")))
+        _check(getattr(lib, fn_name)(*args, _ptr(out)))
+    return out
+
+
+def vstep_product(R, U):
+    """U^T R (w x n) for U m x w int8 (§2.3 step 1, §2.4)."""
+    return _step("externd_vstep_product", R, U, lambda F: F.shape[1], lambda m, n, w: (w, n), weights=False)
+
+
+def ustep_product(R, Cb, weights=None):
+    """R diag(h) Cb^T (m x w) for Cb w x n int8 (§2.3 step 1, §2.5)."""
+    return _step("externd_ustep_product", R, Cb, lambda F: F.shape[0], lambda m, n, w: (m, w), weights=weights)
+
+
+def vstep_target(R, U):
+    """Eq. 3 left: (U^T U + eps I)^-1 U^T R (w x n)."""
+    return _step("externd_vstep_target", R, U, lambda F: F.shape[1], lambda m, n, w: (w, n), weights=False)
+
+
+def ustep_target(R, Cb, weights=None):
+    """Eq. 3 right with §2.5: R H V (V^T H V + eps I)^-1 (m x w), V = Cb^T."""
+    return _step("externd_ustep_target", R, Cb, lambda F: F.shape[0], lambda m, n, w: (m, w), weights=weights)
+
+
+def block_scales(R, U, Cb, weights=None):
+    """Eq. 4 (§2.5 weighted): the joint scales d of the block (U, Cb) against residual R."""
+    torch = _torch()
+    lib = load()
+    R = _prep(R, torch.float32, "R")
+    U, Cb = _prep(U, torch.int8, "U"), _prep(Cb, torch.int8, "Cb")
+    h = None if weights is None else _prep(weights, torch.float32, "weights")
+    m, n = R.shape
+    w = U.shape[1]
+    d = torch.empty((w,), dtype=torch.float32, device=R.device)
+    with torch.cuda.device(R.device):
+        _stream(lib, R.device)
+        _check(lib.externd_block_scales(_ptr(R), m, n, _ptr(U), _ptr(Cb), w, _ptr(h), _ptr(d)))
+    return d
+
+
+def deflate(R, U, d, Cb, weights=None) -> float:
+    """In place R <- R - U diag(d) Cb (§2.3 step 3, §2.4); returns sum_ij h_j R_ij^2 afterwards."""
+    torch = _torch()
+    lib = load()
+    if not (R.is_cuda and R.dtype == torch.float32 and R.is_contiguous()):
+        raise ExterndError("R must be a contiguous CUDA float32 tensor (updated in place)")
+    U, Cb, d = _prep(U, torch.int8, "U"), _prep(Cb, torch.int8, "Cb"), _prep(d, torch.float32, "d")
+    h = None if weights is None else _prep(weights, torch.float32, "weights")
+    m, n = R.shape
+    out = _c_double()
+    with torch.cuda.device(R.device):
+        _stream(lib, R.device)
+        _check(lib.externd_deflate(_ptr(R), m, n, _ptr(U), _ptr(d), _ptr(Cb), U.shape[1], _ptr(h),
+                                   ctypes.byref(out)))
+    return out.value

@@ -1,0 +1,682 @@
+// Host side of libexternd: argument checks, device workspace, the per-block schedule of the method, CUDA-graph
+// replay, and the extern "C" entry points declared in include/externd.h.
+//
+// Schedule of one block of w components (§2.4; w = 1 is the sequential algorithm of §2.3):
+//   select    the w residual columns of largest weighted energy (start of the block; the paper leaves it open)
+//   gather    Y = R[:, J], Eq. 2 statistics                 apply   U = T_tau(Y) column-wise
+//   iters x { gram(U) -> (U^T U + eps I)^-1;  V-step product U^T R;  decorrelate (Eq. 3 left);  apply -> V
+//             gram(V, h) -> (V^T H V + eps I)^-1;  U-step product R H V;  decorrelate (Eq. 3 right);  apply -> U }
+//   gram(U), r = diag(U^T R H V), Eq. 4 solve -> d;  deflate R -= U diag(d) V^T (+ ||R||_H^2, column energies)
+//   write B[:, j0:j0+w], C[j0:j0+w, :], D[j0:j0+w].
+// The whole decomposition is captured once into a CUDA graph per (shape, parameters, buffers) and replayed.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "../../include/externd.h"
+#include "kernels.h"
+
+using namespace externd;
+
+namespace {
+
+std::mutex g_mutex;
+cudaStream_t g_stream = nullptr;
+char g_cuda_error[512] = "no CUDA error";
+
+int cuda_fail(cudaError_t e, const char* where) {
+  std::snprintf(g_cuda_error, sizeof(g_cuda_error), "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
+  return EXTERND_ECUDA;
+}
+
+#define CK(call)                                              \
+  do {                                                        \
+    cudaError_t e_ = (call);                                  \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call);       \
+  } while (0)
+
+// Grow-only device buffers, one set per device.
+struct Buffer {
+  void* p = nullptr;
+  size_t cap = 0;
+};
+
+struct Workspace {
+  std::map<std::string, Buffer> bufs;
+  void* host = nullptr;        // pinned staging for results read on the host
+  size_t host_cap = 0;
+  cudaStream_t cap_stream = nullptr;
+  unsigned generation = 0;     // bumped whenever a buffer moves (invalidates captured graphs)
+};
+
+std::map<int, Workspace> g_ws;
+
+template <typename T>
+int need(Workspace& ws, const char* name, size_t count, T** out, bool zero = false) {
+  Buffer& b = ws.bufs[name];
+  size_t bytes = count * sizeof(T);
+  if (bytes == 0) bytes = 16;
+  if (b.cap < bytes) {
+    if (b.p) cudaFree(b.p);
+    b.p = nullptr;
+    b.cap = 0;
+    size_t alloc = bytes + bytes / 4;
+    if (cudaMalloc(&b.p, alloc) != cudaSuccess) {
+      cudaGetLastError();
+      return EXTERND_ENOMEM;
+    }
+    b.cap = alloc;
+    ++ws.generation;
+    if (zero) CK(cudaMemset(b.p, 0, alloc));
+  }
+  *out = static_cast<T*>(b.p);
+  return EXTERND_OK;
+}
+
+int need_host(Workspace& ws, size_t bytes, void** out) {
+  if (ws.host_cap < bytes) {
+    if (ws.host) cudaFreeHost(ws.host);
+    ws.host = nullptr;
+    ws.host_cap = 0;
+    if (cudaMallocHost(&ws.host, bytes) != cudaSuccess) {
+      cudaGetLastError();
+      return EXTERND_ENOMEM;
+    }
+    ws.host_cap = bytes;
+  }
+  *out = ws.host;
+  return EXTERND_OK;
+}
+
+int current_ws(Workspace** out) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    cuda_fail(e, "cudaGetDevice");
+    return EXTERND_ENODEV;
+  }
+  Workspace& ws = g_ws[dev];
+  if (ws.cap_stream == nullptr) CK(cudaStreamCreateWithFlags(&ws.cap_stream, cudaStreamNonBlocking));
+  *out = &ws;
+  return EXTERND_OK;
+}
+
+#define TRY(x)                        \
+  do {                                \
+    int rc_ = (x);                    \
+    if (rc_ != EXTERND_OK) return rc_; \
+  } while (0)
+
+bool is_device_ptr(const void* p) {
+  if (p == nullptr) return false;
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged ||
+         (at.type == cudaMemoryTypeHost && at.devicePointer != nullptr);
+}
+
+long long ld16(long long x) { return round_up(x, 16); }
+
+// A device float holding 1: the "inverse Gram" of a one-component block, where Eq. 3's positive scalar factor
+// does not change T_tau and the sequential algorithm of §2.3 ternarizes the product itself.
+int get_one(Workspace& ws, float** out) {
+  Buffer& one = ws.bufs["one"];
+  if (one.p == nullptr) {
+    if (cudaMalloc(&one.p, 256) != cudaSuccess) {
+      cudaGetLastError();
+      return EXTERND_ENOMEM;
+    }
+    one.cap = 256;
+    const float v = 1.f;
+    CK(cudaMemcpy(one.p, &v, sizeof(float), cudaMemcpyHostToDevice));
+  }
+  *out = static_cast<float*>(one.p);
+  return EXTERND_OK;
+}
+
+int block_width_of(long long m, long long n, int block) {
+  long long cap = std::min(m, n) / 8;
+  long long b = std::min<long long>(block, cap);
+  return (int)std::max<long long>(1, b);
+}
+
+// ------------------------------------------------------------------------------------------------------------
+// Decomposition
+// ------------------------------------------------------------------------------------------------------------
+struct Plan {
+  int m, n, b, iters, nblocks;
+  long long k;
+  double tau;
+  int sv, su, gm, gn;          // split counts: V-step, U-step, Gram over m, Gram over n
+  int nchunk_m, nchunk_n;
+  long long ldm, ldn;
+};
+
+struct Bufs {
+  float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE;
+  int8_t *Ut, *Vt;
+  double *spart, *r, *normpart, *norm_a, *norm_r, *trace;
+  u64* kpart;
+  int* J;
+};
+
+int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
+  const long long L = std::max(p.m, p.n);
+  const long long w = p.b;
+  TRY(need(ws, "R", (size_t)p.m * p.n, &B->R));
+  TRY(need(ws, "Ut", (size_t)w * p.ldm, &B->Ut, true));
+  TRY(need(ws, "Vt", (size_t)w * p.ldn, &B->Vt, true));
+  TRY(need(ws, "part", (size_t)std::max((long long)p.sv * w * p.n, (long long)p.su * w * p.m), &B->part));
+  TRY(need(ws, "X", (size_t)w * L, &B->X));
+  TRY(need(ws, "spart", (size_t)w * std::max(p.nchunk_m, p.nchunk_n), &B->spart));
+  TRY(need(ws, "kpart", (size_t)w * std::max(p.nchunk_m, p.nchunk_n), &B->kpart));
+  TRY(need(ws, "Gpart", (size_t)std::max(p.gm, p.gn) * w * w, &B->Gpart));
+  TRY(need(ws, "GrawU", (size_t)w * w, &B->GrawU));
+  TRY(need(ws, "GrawV", (size_t)w * w, &B->GrawV));
+  TRY(need(ws, "Ginv", (size_t)w * w, &B->Ginv));
+  TRY(need(ws, "d", (size_t)w, &B->d));
+  TRY(need(ws, "r", (size_t)w, &B->r));
+  TRY(need(ws, "J", (size_t)w, &B->J, true));
+  TRY(need(ws, "colpart", (size_t)deflate_row_tiles(p.m) * p.n, &B->colpart));
+  TRY(need(ws, "colE", (size_t)p.n, &B->colE));
+  TRY(need(ws, "normpart", (size_t)deflate_tiles(p.m, p.n), &B->normpart));
+  TRY(need(ws, "scalars", 4, &B->norm_a));
+  B->norm_r = B->norm_a + 1;
+  TRY(need(ws, "trace", (size_t)p.nblocks, &B->trace));
+  return get_one(ws, &B->one);
+}
+
+Plan make_plan(long long m, long long n, long long k, int block, int iters, double tau) {
+  Plan p;
+  p.m = (int)m;
+  p.n = (int)n;
+  p.k = k;
+  p.b = block_width_of(m, n, block);
+  p.iters = iters;
+  p.tau = tau;
+  p.nblocks = (int)cdiv(k, p.b);
+  p.sv = product_splits(p.b, p.n, p.m);
+  p.su = product_splits(p.b, p.m, p.n);
+  p.gm = gram_splits(p.b, p.m);
+  p.gn = gram_splits(p.b, p.n);
+  p.nchunk_m = (int)cdiv(p.m, kStatChunk);
+  p.nchunk_n = (int)cdiv(p.n, kStatChunk);
+  p.ldm = ld16(m);
+  p.ldn = ld16(n);
+  return p;
+}
+
+#define LK(call)                                        \
+  do {                                                  \
+    cudaError_t e_ = (call);                            \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call); \
+  } while (0)
+
+// Enqueues the whole decomposition on stream s.
+int enqueue_decompose(const Plan& p, const Bufs& B, const float* A, const float* h, int8_t* Bout, float* Dout,
+                      int8_t* Cout, cudaStream_t s) {
+  const int m = p.m, n = p.n;
+  const Stats st_m{B.spart, B.kpart, p.nchunk_m};
+  const Stats st_n{B.spart, B.kpart, p.nchunk_n};
+  const int nrt = deflate_row_tiles(m), ntiles = deflate_tiles(m, n);
+  // R = A, column energies, ||A||_H^2
+  LK(launch_deflate(A, B.R, m, n, nullptr, 0, false, nullptr, nullptr, 0, 0, h, B.colpart, B.normpart, s));
+  LK(launch_norm(B.normpart, ntiles, B.norm_a, nullptr, nullptr, s));
+  for (int blk = 0; blk < p.nblocks; ++blk) {
+    const long long j0 = (long long)blk * p.b;
+    const int w = (int)std::min<long long>(p.b, p.k - j0);
+    LK(launch_select_with(B.colpart, nrt, n, h, w, B.J, B.colE, s));
+    LK(launch_gather(B.R, m, n, B.J, w, B.X, m, st_m, s));
+    LK(launch_apply(B.X, w, m, m, st_m, p.tau, B.Ut, (int)p.ldm, s));
+    for (int it = 0; it < p.iters; ++it) {
+      // V-step: V <- T([(U^T U + eps I)^-1 U^T R]^T)   (plain R even when weighted, §2.5)
+      if (w > 1) {
+        LK(launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
+        LK(launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, s));
+      }
+      LK(launch_product_v(B.R, m, n, B.Ut, (int)p.ldm, w, B.part, p.sv, s));
+      LK(launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, p.sv, n, B.X, n, st_n, s));
+      LK(launch_apply(B.X, w, n, n, st_n, p.tau, B.Vt, (int)p.ldn, s));
+      // U-step: U <- T(R H V (V^T H V + eps I)^-1)
+      LK(launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, s));
+      LK(launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, s));
+      LK(launch_product_u(B.R, m, n, B.Vt, (int)p.ldn, w, h, B.part, p.su, s));
+      LK(launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, p.su, m, B.X, m, st_m, s));
+      LK(launch_apply(B.X, w, m, m, st_m, p.tau, B.Ut, (int)p.ldm, s));
+    }
+    // Eq. 4: [(U^T U) .* (V^T H V)] d = diag(U^T R H V), with R H V the last U-step product
+    LK(launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
+    LK(launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, p.su, B.r, s));
+    LK(launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s));
+    // R <- R - U diag(d) V^T
+    LK(launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart, B.normpart, s));
+    LK(launch_norm(B.normpart, ntiles, B.norm_r, B.norm_a, B.trace + blk, s));
+    LK(launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, s));
+    LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
+                         cudaMemcpyDeviceToDevice, s));
+    LK(cudaMemcpyAsync(Dout + j0, B.d, sizeof(float) * w, cudaMemcpyDeviceToDevice, s));
+  }
+  return EXTERND_OK;
+}
+
+struct GraphKey {
+  const void *A, *h, *B, *D, *C;
+  long long m, n, k;
+  int b, iters;
+  double tau;
+  unsigned gen;
+  bool operator<(const GraphKey& o) const {
+    return std::tie(A, h, B, D, C, m, n, k, b, iters, tau, gen) <
+           std::tie(o.A, o.h, o.B, o.D, o.C, o.m, o.n, o.k, o.b, o.iters, o.tau, o.gen);
+  }
+};
+
+std::map<int, std::map<GraphKey, cudaGraphExec_t>> g_graphs;
+
+bool graphs_enabled() {
+  const char* e = std::getenv("EXTERND_GRAPHS");
+  return !(e && std::strcmp(e, "0") == 0);
+}
+
+int run_decompose(const float* A, long long m, long long n, double mu, double tau, int block, int iters,
+                  const float* h, int8_t* Bout, float* Dout, int8_t* Cout, double* energy, double* trace) {
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  int64_t k;
+  TRY(externd_rank(m, n, mu, &k));
+  Plan p = make_plan(m, n, k, block, iters, tau);
+  Bufs B;
+  TRY(plan_buffers(*ws, p, &B));
+  int dev;
+  CK(cudaGetDevice(&dev));
+  cudaStream_t s = g_stream;
+  if (graphs_enabled()) {
+    GraphKey key{A, h, Bout, Dout, Cout, m, n, k, p.b, iters, tau, ws->generation};
+    auto& cache = g_graphs[dev];
+    auto it = cache.find(key);
+    if (it == cache.end()) {
+      if (cache.size() >= 16) {
+        for (auto& kv : cache) cudaGraphExecDestroy(kv.second);
+        cache.clear();
+      }
+      cudaGraph_t graph;
+      CK(cudaStreamBeginCapture(ws->cap_stream, cudaStreamCaptureModeThreadLocal));
+      int rc = enqueue_decompose(p, B, A, h, Bout, Dout, Cout, ws->cap_stream);
+      cudaError_t ec = cudaStreamEndCapture(ws->cap_stream, &graph);
+      if (rc != EXTERND_OK) return rc;
+      if (ec != cudaSuccess) return cuda_fail(ec, "cudaStreamEndCapture");
+      cudaGraphExec_t exec;
+      cudaError_t ei = cudaGraphInstantiate(&exec, graph, 0);
+      cudaGraphDestroy(graph);
+      if (ei != cudaSuccess) return cuda_fail(ei, "cudaGraphInstantiate");
+      it = cache.emplace(key, exec).first;
+    }
+    CK(cudaGraphLaunch(it->second, s));
+  } else {
+    TRY(enqueue_decompose(p, B, A, h, Bout, Dout, Cout, s));
+  }
+  if (energy != nullptr || trace != nullptr) {
+    void* hbuf;
+    TRY(need_host(*ws, sizeof(double) * (size_t)p.nblocks, &hbuf));
+    CK(cudaMemcpyAsync(hbuf, B.trace, sizeof(double) * p.nblocks, cudaMemcpyDeviceToHost, s));
+    CK(cudaStreamSynchronize(s));
+    const double* tr = static_cast<const double*>(hbuf);
+    if (energy) *energy = tr[p.nblocks - 1];
+    if (trace) std::memcpy(trace, tr, sizeof(double) * p.nblocks);
+  }
+  CK(cudaGetLastError());
+  return EXTERND_OK;
+}
+
+// Sizes the kernels' grids cover: rows of R tile by 64 in gridDim.y (<= 65535 tiles), columns by 128 in gridDim.x.
+constexpr long long kMaxRows = 65535LL * 64;
+constexpr long long kMaxCols = 1LL << 30;
+
+int check_common(long long m, long long n) {
+  if (m < 1 || n < 1 || m > kMaxRows || n > kMaxCols || m * n > (1LL << 40)) return EXTERND_EINVAL;
+  return EXTERND_OK;
+}
+
+int check_params(double mu, double tau, int block, int iters) {
+  if (!(mu > 0) || !std::isfinite(mu) || !(tau >= 0) || !std::isfinite(tau)) return EXTERND_EINVAL;
+  if (block < 1 || block > kMaxBlock || iters < 1) return EXTERND_EINVAL;
+  return EXTERND_OK;
+}
+
+int check_dev(const void* p) { return is_device_ptr(p) ? EXTERND_OK : (p ? EXTERND_EPTR : EXTERND_EINVAL); }
+
+// Per-step helpers: bring a caller's m x w U into the internal Ut layout, and a w x n Cb into Vt.
+int stage_u(Workspace& ws, const int8_t* U, long long m, int w, int8_t** Ut) {
+  TRY(need(ws, "Ut", (size_t)w * ld16(m), Ut, true));
+  LK(launch_transpose_i8(U, w, (int)m, w, *Ut, ld16(m), g_stream));
+  return EXTERND_OK;
+}
+
+int stage_v(Workspace& ws, const int8_t* Cb, long long n, int w, int8_t** Vt) {
+  TRY(need(ws, "Vt", (size_t)w * ld16(n), Vt, true));
+  LK(cudaMemcpy2DAsync(*Vt, (size_t)ld16(n), Cb, (size_t)n, (size_t)n, (size_t)w, cudaMemcpyDeviceToDevice, g_stream));
+  return EXTERND_OK;
+}
+
+int read_double(Workspace& ws, const double* dptr, double* out) {
+  void* hb;
+  TRY(need_host(ws, sizeof(double), &hb));
+  CK(cudaMemcpyAsync(hb, dptr, sizeof(double), cudaMemcpyDeviceToHost, g_stream));
+  CK(cudaStreamSynchronize(g_stream));
+  *out = *static_cast<double*>(hb);
+  return EXTERND_OK;
+}
+
+}  // namespace
+
+// ==============================================================================================================
+extern "C" {
+
+const char* externd_strerror(int status) {
+  switch (status) {
+    case EXTERND_OK: return "ok";
+    case EXTERND_EINVAL: return "invalid argument (size, parameter or NULL pointer)";
+    case EXTERND_EPTR: return "pointer is not accessible from the CUDA device";
+    case EXTERND_ENOMEM: return "device workspace allocation failed";
+    case EXTERND_ECUDA: return "CUDA error (see externd_last_cuda_error)";
+    case EXTERND_ENODEV: return "no usable CUDA device";
+    default: return "unknown status";
+  }
+}
+
+const char* externd_last_cuda_error(void) { return g_cuda_error; }
+
+const char* externd_version(void) { return "externd-gb300 0.1 (sm_103a)"; }
+
+int externd_set_stream(void* cuda_stream) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  g_stream = static_cast<cudaStream_t>(cuda_stream);
+  return EXTERND_OK;
+}
+
+int externd_rank(int64_t m, int64_t n, double mu, int64_t* k) {
+  if (k == nullptr || m < 1 || n < 1 || !(mu > 0) || !std::isfinite(mu)) return EXTERND_EINVAL;
+  const double v = std::floor(mu * (double)std::min(m, n) + 0.5);
+  if (v < 1 || v > 1e12) return EXTERND_EINVAL;
+  *k = (int64_t)v;
+  return EXTERND_OK;
+}
+
+int externd_block_width(int64_t m, int64_t n, int block, int* b) {
+  if (b == nullptr || m < 1 || n < 1 || block < 1 || block > kMaxBlock) return EXTERND_EINVAL;
+  *b = block_width_of(m, n, block);
+  return EXTERND_OK;
+}
+
+int externd_decompose(const float* A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
+                      const float* weights, int8_t* B, float* D, int8_t* C, double* energy, double* trace) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  TRY(check_common(m, n));
+  TRY(check_params(mu, tau, block, iters));
+  if (energy == nullptr && trace == nullptr) {
+    // results still land in B, D, C; nothing to report on the host
+  }
+  TRY(check_dev(A));
+  TRY(check_dev(B));
+  TRY(check_dev(D));
+  TRY(check_dev(C));
+  if (weights != nullptr) TRY(check_dev(weights));
+  return run_decompose(A, m, n, mu, tau, block, iters, weights, B, D, C, energy, trace);
+}
+
+int externd_decompose_host(const float* A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
+                           const float* weights, int8_t* B, float* D, int8_t* C, double* energy, double* trace) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  TRY(check_common(m, n));
+  TRY(check_params(mu, tau, block, iters));
+  if (A == nullptr || B == nullptr || D == nullptr || C == nullptr) return EXTERND_EINVAL;
+  int64_t k;
+  TRY(externd_rank(m, n, mu, &k));
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  float *dA, *dh = nullptr, *dD;
+  int8_t *dB, *dC;
+  TRY(need(*ws, "host.A", (size_t)m * n, &dA));
+  TRY(need(*ws, "host.B", (size_t)m * k, &dB));
+  TRY(need(*ws, "host.C", (size_t)k * n, &dC));
+  TRY(need(*ws, "host.D", (size_t)k, &dD));
+  if (weights) TRY(need(*ws, "host.h", (size_t)n, &dh));
+  cudaStream_t s = g_stream;
+  CK(cudaMemcpyAsync(dA, A, sizeof(float) * m * n, cudaMemcpyHostToDevice, s));
+  if (weights) CK(cudaMemcpyAsync(dh, weights, sizeof(float) * n, cudaMemcpyHostToDevice, s));
+  TRY(run_decompose(dA, m, n, mu, tau, block, iters, dh, dB, dD, dC, energy, trace));
+  CK(cudaMemcpyAsync(B, dB, (size_t)m * k, cudaMemcpyDeviceToHost, s));
+  CK(cudaMemcpyAsync(C, dC, (size_t)k * n, cudaMemcpyDeviceToHost, s));
+  CK(cudaMemcpyAsync(D, dD, sizeof(float) * k, cudaMemcpyDeviceToHost, s));
+  CK(cudaStreamSynchronize(s));
+  return EXTERND_OK;
+}
+
+int externd_energy(const float* A, int64_t m, int64_t n, const int8_t* B, const float* D, const int8_t* C, int64_t k,
+                   const float* weights, double* energy) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  TRY(check_common(m, n));
+  if (k < 1 || k > (1LL << 31) || energy == nullptr) return EXTERND_EINVAL;
+  TRY(check_dev(A));
+  TRY(check_dev(B));
+  TRY(check_dev(D));
+  TRY(check_dev(C));
+  if (weights != nullptr) TRY(check_dev(weights));
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  double* part;
+  double* sc;
+  TRY(need(*ws, "energy.part", (size_t)deflate_tiles((int)m, (int)n), &part));
+  TRY(need(*ws, "energy.sc", 4, &sc));
+  const int tiles = deflate_tiles((int)m, (int)n);
+  LK(launch_deflate(A, nullptr, (int)m, (int)n, nullptr, 0, false, nullptr, nullptr, 0, 0, weights, nullptr, part,
+                    g_stream));
+  LK(launch_norm(part, tiles, sc, nullptr, nullptr, g_stream));
+  LK(launch_deflate(A, nullptr, (int)m, (int)n, B, k, true, D, C, n, (int)k, weights, nullptr, part, g_stream));
+  LK(launch_norm(part, tiles, sc + 1, sc, sc + 2, g_stream));
+  return read_double(*ws, sc + 2, energy);
+}
+
+int externd_ternarize(const float* X, int64_t rows, int64_t cols, int axis, double tau, int8_t* T) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  TRY(check_common(rows, cols));
+  if ((axis != 0 && axis != 1) || !(tau >= 0) || !std::isfinite(tau)) return EXTERND_EINVAL;
+  TRY(check_dev(X));
+  TRY(check_dev(T));
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  const long long nv = axis == 1 ? rows : cols, L = axis == 1 ? cols : rows;
+  if (nv > 65535) return EXTERND_EINVAL;   // one grid row per vector
+  const int nchunk = (int)cdiv(L, kStatChunk);
+  double* sp;
+  u64* kp;
+  TRY(need(*ws, "tern.spart", (size_t)nv * nchunk, &sp));
+  TRY(need(*ws, "tern.kpart", (size_t)nv * nchunk, &kp));
+  Stats st{sp, kp, nchunk};
+  if (axis == 1) {
+    LK(launch_stats(X, (int)nv, (int)L, (int)L, st, g_stream));
+    LK(launch_apply(X, (int)nv, (int)L, L, st, tau, T, (int)L, g_stream));
+  } else {
+    float* Xt;
+    int8_t* Tt;
+    TRY(need(*ws, "tern.X", (size_t)nv * L, &Xt));
+    TRY(need(*ws, "tern.T", (size_t)nv * L, &Tt));
+    LK(launch_transpose_f32(X, cols, (int)rows, (int)cols, Xt, L, g_stream));
+    LK(launch_stats(Xt, (int)nv, (int)L, (int)L, st, g_stream));
+    LK(launch_apply(Xt, (int)nv, (int)L, L, st, tau, Tt, (int)L, g_stream));
+    LK(launch_transpose_i8(Tt, L, (int)nv, (int)L, T, cols, g_stream));
+  }
+  CK(cudaGetLastError());
+  return EXTERND_OK;
+}
+
+#define STEP_CHECKS(R_, w_)                                  \
+  TRY(check_common(m, n));                                   \
+  if ((w_) < 1 || (w_) > kMaxBlock) return EXTERND_EINVAL;   \
+  TRY(check_dev(R_));
+
+int externd_vstep_product(const float* R, int64_t m, int64_t n, const int8_t* U, int64_t w, float* PV) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  STEP_CHECKS(R, w);
+  TRY(check_dev(U));
+  TRY(check_dev(PV));
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  int8_t* Ut;
+  float* part;
+  TRY(stage_u(*ws, U, m, (int)w, &Ut));
+  const int sv = product_splits((int)w, (int)n, (int)m);
+  TRY(need(*ws, "part", (size_t)sv * w * n, &part));
+  LK(launch_product_v(R, (int)m, (int)n, Ut, (int)ld16(m), (int)w, part, sv, g_stream));
+  LK(launch_sum_splits(part, sv, (int)w, (int)n, PV, n, g_stream));
+  return EXTERND_OK;
+}
+
+int externd_ustep_product(const float* R, int64_t m, int64_t n, const int8_t* Cb, int64_t w, const float* weights,
+                          float* PU) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  STEP_CHECKS(R, w);
+  TRY(check_dev(Cb));
+  TRY(check_dev(PU));
+  if (weights) TRY(check_dev(weights));
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  int8_t* Vt;
+  float *part, *X;
+  TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
+  const int su = product_splits((int)w, (int)m, (int)n);
+  TRY(need(*ws, "part", (size_t)su * w * m, &part));
+  TRY(need(*ws, "X", (size_t)w * m, &X));
+  LK(launch_product_u(R, (int)m, (int)n, Vt, (int)ld16(n), (int)w, weights, part, su, g_stream));
+  LK(launch_sum_splits(part, su, (int)w, (int)m, X, m, g_stream));
+  LK(launch_transpose_f32(X, m, (int)w, (int)m, PU, w, g_stream));
+  return EXTERND_OK;
+}
+
+namespace {
+int step_target(bool vstep, const float* R, long long m, long long n, const int8_t* F, int w, const float* h,
+                float* out) {
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  const long long L = vstep ? n : m;
+  const int nchunk = (int)cdiv(L, kStatChunk);
+  int8_t* T;
+  float *part, *X, *Gpart, *Graw, *Ginv, *one;
+  double* sp;
+  u64* kp;
+  if (vstep) TRY(stage_u(*ws, F, m, w, &T));
+  else TRY(stage_v(*ws, F, n, w, &T));
+  const long long ldt = vstep ? ld16(m) : ld16(n);
+  const long long Lred = vstep ? m : n;
+  const int splits = product_splits(w, (int)L, (int)Lred);
+  const int gs = gram_splits(w, (int)Lred);
+  TRY(need(*ws, "part", (size_t)splits * w * L, &part));
+  TRY(need(*ws, "X", (size_t)w * L, &X));
+  TRY(need(*ws, "Gpart", (size_t)gs * w * w, &Gpart));
+  TRY(need(*ws, "GrawV", (size_t)w * w, &Graw));
+  TRY(need(*ws, "Ginv", (size_t)w * w, &Ginv));
+  TRY(need(*ws, "spart", (size_t)w * nchunk, &sp));
+  TRY(need(*ws, "kpart", (size_t)w * nchunk, &kp));
+  TRY(get_one(*ws, &one));
+  if (vstep) LK(launch_product_v(R, (int)m, (int)n, T, (int)ldt, w, part, splits, g_stream));
+  else LK(launch_product_u(R, (int)m, (int)n, T, (int)ldt, w, h, part, splits, g_stream));
+  if (w > 1) {
+    LK(launch_gram(T, (int)ldt, w, (int)Lred, vstep ? nullptr : h, Gpart, gs, g_stream));
+    LK(launch_inverse(Gpart, gs, w, Graw, Ginv, g_stream));
+  }
+  Stats st{sp, kp, nchunk};
+  if (vstep) {
+    LK(launch_decorrelate(w > 1 ? Ginv : one, w, part, splits, (int)L, out, (int)L, st, g_stream));
+  } else {
+    LK(launch_decorrelate(w > 1 ? Ginv : one, w, part, splits, (int)L, X, (int)L, st, g_stream));
+    LK(launch_transpose_f32(X, L, w, (int)L, out, w, g_stream));
+  }
+  return EXTERND_OK;
+}
+}  // namespace
+
+int externd_vstep_target(const float* R, int64_t m, int64_t n, const int8_t* U, int64_t w, float* X) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  STEP_CHECKS(R, w);
+  TRY(check_dev(U));
+  TRY(check_dev(X));
+  return step_target(true, R, m, n, U, (int)w, nullptr, X);
+}
+
+int externd_ustep_target(const float* R, int64_t m, int64_t n, const int8_t* Cb, int64_t w, const float* weights,
+                         float* Y) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  STEP_CHECKS(R, w);
+  TRY(check_dev(Cb));
+  TRY(check_dev(Y));
+  if (weights) TRY(check_dev(weights));
+  return step_target(false, R, m, n, Cb, (int)w, weights, Y);
+}
+
+int externd_block_scales(const float* R, int64_t m, int64_t n, const int8_t* U, const int8_t* Cb, int64_t w,
+                         const float* weights, float* d) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  STEP_CHECKS(R, w);
+  TRY(check_dev(U));
+  TRY(check_dev(Cb));
+  TRY(check_dev(d));
+  if (weights) TRY(check_dev(weights));
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  int8_t *Ut, *Vt;
+  float *part, *Gpart, *GrawV, *Ginv;
+  double* r;
+  TRY(stage_u(*ws, U, m, (int)w, &Ut));
+  TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
+  const int su = product_splits((int)w, (int)m, (int)n);
+  const int gm = gram_splits((int)w, (int)m), gn = gram_splits((int)w, (int)n);
+  TRY(need(*ws, "part", (size_t)su * w * m, &part));
+  TRY(need(*ws, "Gpart", (size_t)std::max(gm, gn) * w * w, &Gpart));
+  TRY(need(*ws, "GrawV", (size_t)w * w, &GrawV));
+  TRY(need(*ws, "Ginv", (size_t)w * w, &Ginv));
+  TRY(need(*ws, "r", (size_t)w, &r));
+  LK(launch_product_u(R, (int)m, (int)n, Vt, (int)ld16(n), (int)w, weights, part, su, g_stream));
+  LK(launch_gram(Vt, (int)ld16(n), (int)w, (int)n, weights, Gpart, gn, g_stream));
+  LK(launch_inverse(Gpart, gn, (int)w, GrawV, Ginv, g_stream));
+  LK(launch_gram(Ut, (int)ld16(m), (int)w, (int)m, nullptr, Gpart, gm, g_stream));
+  LK(launch_rvec(Ut, (int)ld16(m), (int)w, (int)m, part, su, r, g_stream));
+  LK(launch_scales(Gpart, gm, GrawV, r, (int)w, d, g_stream));
+  return EXTERND_OK;
+}
+
+int externd_deflate(float* R, int64_t m, int64_t n, const int8_t* U, const float* d, const int8_t* Cb, int64_t w,
+                    const float* weights, double* norm2) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  STEP_CHECKS(R, w);
+  TRY(check_dev(U));
+  TRY(check_dev(d));
+  TRY(check_dev(Cb));
+  if (weights) TRY(check_dev(weights));
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  int8_t *Ut, *Vt;
+  double *part, *sc;
+  TRY(stage_u(*ws, U, m, (int)w, &Ut));
+  TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
+  const int tiles = deflate_tiles((int)m, (int)n);
+  TRY(need(*ws, "energy.part", (size_t)tiles, &part));
+  TRY(need(*ws, "energy.sc", 4, &sc));
+  LK(launch_deflate(R, R, (int)m, (int)n, Ut, ld16(m), false, d, Vt, ld16(n), (int)w, weights, nullptr, part,
+                    g_stream));
+  LK(launch_norm(part, tiles, sc, nullptr, nullptr, g_stream));
+  if (norm2 != nullptr) return read_double(*ws, sc, norm2);
+  return EXTERND_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,381 @@
+// Residual products, decorrelation and deflation on the CUDA cores (float32 FMA, register-tiled).
+//
+//   V-step product   part[s][a][c] = sum_{r in split s} U[r][a] R[r][c]            (§2.3 step 1, §2.4)
+//   U-step product   part[s][a][r] = sum_{c in split s} R[r][c] h[c] V[c][a]        (§2.3 step 1, §2.5)
+//   decorrelation    X[a][x] = sum_b Ginv[a][b] sum_s part[s][b][x]               (Eq. 3)
+//   deflation        R[r][c] -= sum_a U[r][a] d[a] V[c][a], fused ||R||_H^2 and column energies (§2.3, §2.4)
+//
+// Every kernel computes a 64 x 128 output tile with 256 threads (4 x 8 outputs per thread) from 16-deep slices
+// staged in shared memory. Split-K partials are written, never atomically added, so results are reproducible.
+#include "kernels.h"
+
+namespace externd {
+
+namespace {
+
+constexpr int TM = 64;   // rows of the output tile (components, or residual rows for the deflation)
+constexpr int TN = 128;  // columns of the output tile
+constexpr int TK = 16;   // depth of one shared-memory slice
+
+// One 16-deep step of the 64 x 128 tile: acc[i][j] += As[k][ty*4+i] * Bs[k][(j<4 ? 0 : 64) + tx*4 + j%4].
+__device__ __forceinline__ void tile_fma(const float (*As)[TM + 4], const float (*Bs)[TN], int tx, int ty,
+                                         float acc[4][8]) {
+#pragma unroll
+  for (int k = 0; k < TK; ++k) {
+    const float4 a = *reinterpret_cast<const float4*>(&As[k][ty * 4]);
+    const float4 b0 = *reinterpret_cast<const float4*>(&Bs[k][tx * 4]);
+    const float4 b1 = *reinterpret_cast<const float4*>(&Bs[k][64 + tx * 4]);
+    const float av[4] = {a.x, a.y, a.z, a.w};
+    const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+  }
+}
+
+__device__ __forceinline__ int col_of(int tx, int j) { return (j < 4 ? 0 : 64) + tx * 4 + (j & 3); }
+
+// Ternary slice: Ts[ky][a] = T[a0 + a][y0 + ky] for ky < 16, a < 64 (zero outside w / [y0, yend)).
+__device__ __forceinline__ void load_ternary_slice(float (*Ts)[TM + 4], const int8_t* __restrict__ T, int ldt, int w,
+                                                   int a0, int y0, int yend, int tid) {
+  const int a = tid >> 2;
+  const int ky = (tid & 3) * 4;
+  const int ag = a0 + a;
+  int packed = 0;
+  if (ag < w) packed = __ldg(reinterpret_cast<const int*>(T + (long long)ag * ldt + y0 + ky));
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int y = y0 + ky + j;
+    const int8_t t = (int8_t)((packed >> (8 * j)) & 0xff);
+    Ts[ky + j][a] = (y < yend) ? (float)t : 0.f;
+  }
+}
+
+template <bool USTEP>
+__global__ void __launch_bounds__(256) product_kernel(const float* __restrict__ R, int m, int n,
+                                                      const int8_t* __restrict__ T, int ldt, int w,
+                                                      const float* __restrict__ h, float* __restrict__ part,
+                                                      int ychunk) {
+  __shared__ __align__(16) float Rs[TK][TN];
+  __shared__ __align__(16) float Ts[TK][TM + 4];
+  const int Lx = USTEP ? m : n;
+  const int Ly = USTEP ? n : m;
+  const int x0 = blockIdx.x * TN;
+  const int a0 = blockIdx.y * TM;
+  const int ybeg = blockIdx.z * ychunk;
+  const int yend = min(Ly, ybeg + ychunk);
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const bool vec = (n & 3) == 0;
+  float acc[4][8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+
+  for (int y0 = ybeg; y0 < yend; y0 += TK) {
+    if (!USTEP) {
+      // Rs[ky][kx] = R[y0 + ky][x0 + kx]
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const int idx = tid + 256 * q;
+        const int ky = idx >> 5, kx = (idx & 31) * 4;
+        const int y = y0 + ky;
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (y < yend) v = load4(R + (long long)y * n, x0 + kx, n, vec);
+        *reinterpret_cast<float4*>(&Rs[ky][kx]) = v;
+      }
+    } else {
+      // Rs[ky][kx] = R[x0 + kx][y0 + ky] * h[y0 + ky]
+      const int kx = tid & 127, half = tid >> 7;
+      const int x = x0 + kx;
+      const int yb = y0 + 8 * half;
+      float4 v0 = make_float4(0.f, 0.f, 0.f, 0.f), v1 = v0;
+      if (x < m) {
+        v0 = load4(R + (long long)x * n, yb, yend, vec);
+        v1 = load4(R + (long long)x * n, yb + 4, yend, vec);
+      }
+      float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int y = yb + j;
+        const float hy = (h != nullptr && y < yend) ? __ldg(h + y) : 1.f;
+        Rs[8 * half + j][kx] = v[j] * hy;
+      }
+    }
+    load_ternary_slice(Ts, T, ldt, w, a0, y0, yend, tid);
+    __syncthreads();
+    tile_fma(Ts, Rs, tx, ty, acc);
+    __syncthreads();
+  }
+
+  float* out = part + (long long)blockIdx.z * w * Lx;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int a = a0 + ty * 4 + i;
+    if (a >= w) continue;
+#pragma unroll
+    for (int g = 0; g < 2; ++g) {
+      const int x = x0 + g * 64 + tx * 4;
+      float* o = out + (long long)a * Lx + x;
+      if ((Lx & 3) == 0 && x + 3 < Lx) {
+        *reinterpret_cast<float4*>(o) = make_float4(acc[i][4 * g], acc[i][4 * g + 1], acc[i][4 * g + 2], acc[i][4 * g + 3]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (x + j < Lx) o[j] = acc[i][4 * g + j];
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restrict__ Ginv, int w,
+                                                          const float* __restrict__ part, int splits, int L,
+                                                          float* __restrict__ X, int ldx, Stats st) {
+  __shared__ __align__(16) float Ps[TK][TN];
+  __shared__ __align__(16) float Gs[TK][TM + 4];
+  const int x0 = blockIdx.x * TN;
+  const int a0 = blockIdx.y * TM;
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const bool vec = (L & 3) == 0;
+  float acc[4][8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+
+  for (int b0 = 0; b0 < w; b0 += TK) {
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int idx = tid + 256 * q;
+      const int kb = idx >> 5, kx = (idx & 31) * 4;
+      const int b = b0 + kb;
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (b < w) {
+        for (int s = 0; s < splits; ++s) {
+          const float4 p = load4(part + ((long long)s * w + b) * L, x0 + kx, L, vec);
+          v.x += p.x; v.y += p.y; v.z += p.z; v.w += p.w;
+        }
+      }
+      *reinterpret_cast<float4*>(&Ps[kb][kx]) = v;
+    }
+    {
+      const int kb = tid >> 4, a4 = (tid & 15) * 4;
+      const int b = b0 + kb;
+      float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (b < w) g = load4(Ginv + (long long)b * w, a0 + a4, w, (w & 3) == 0);
+      *reinterpret_cast<float4*>(&Gs[kb][a4]) = g;
+    }
+    __syncthreads();
+    tile_fma(Gs, Ps, tx, ty, acc);
+    __syncthreads();
+  }
+
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int a = a0 + ty * 4 + i;
+    AbsSum sum;
+    u64 key = 0;
+    if (a < w) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int x = x0 + col_of(tx, j);
+        if (x < L) {
+          X[(long long)a * ldx + x] = acc[i][j];
+          sum.add(acc[i][j]);
+          const u64 kk = mag_key(acc[i][j], (uint32_t)x);
+          key = kk > key ? kk : key;
+        }
+      }
+    }
+    double s = sum.value();
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) {
+      s += __shfl_xor_sync(0xffffffffu, s, o);
+      const u64 t = __shfl_xor_sync(0xffffffffu, key, o);
+      key = t > key ? t : key;
+    }
+    if (tx == 0 && a < w) {
+      st.spart[(long long)a * st.nchunk + blockIdx.x] = s;
+      st.kpart[(long long)a * st.nchunk + blockIdx.x] = key;
+    }
+  }
+}
+
+template <bool UROW>
+__global__ void __launch_bounds__(256) deflate_kernel(const float* Rin, float* Rout, int m, int n,
+                                                      const int8_t* __restrict__ U, long long ldu,
+                                                      const float* __restrict__ d, const int8_t* __restrict__ V,
+                                                      long long ldv, int w, const float* __restrict__ h,
+                                                      float* __restrict__ colpart, double* __restrict__ normpart) {
+  __shared__ __align__(16) float As[TK][TM + 4];
+  __shared__ __align__(16) float Bs[TK][TN];
+  __shared__ float red[16][TN];
+  __shared__ double wred[8];
+  const int c0 = blockIdx.x * TN;
+  const int r0 = blockIdx.y * TM;
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  float acc[4][8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+
+  for (int a0 = 0; a0 < w; a0 += TK) {
+    if (!UROW) {
+      const int ka = tid >> 4, r4 = (tid & 15) * 4;
+      const int a = a0 + ka;
+      const float da = (a < w) ? __ldg(d + a) : 0.f;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int r = r0 + r4 + j;
+        const float u = (a < w && r < m) ? (float)__ldg(U + a * ldu + r) : 0.f;
+        As[ka][r4 + j] = u * da;
+      }
+    } else {
+      const int r = tid >> 2, a4 = (tid & 3) * 4;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int a = a0 + a4 + j;
+        const float u = (a < w && r0 + r < m) ? (float)__ldg(U + (long long)(r0 + r) * ldu + a) : 0.f;
+        As[a4 + j][r] = (a < w) ? u * __ldg(d + a) : 0.f;
+      }
+    }
+    {
+      const int ka = tid >> 4, c8 = (tid & 15) * 8;
+      const int a = a0 + ka;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int c = c0 + c8 + j;
+        Bs[ka][c8 + j] = (a < w && c < n) ? (float)__ldg(V + a * ldv + c) : 0.f;
+      }
+    }
+    __syncthreads();
+    tile_fma(As, Bs, tx, ty, acc);
+    __syncthreads();
+  }
+
+  const bool vec = (n & 3) == 0;
+  float csum[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) csum[j] = 0.f;
+  float nrm = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = r0 + ty * 4 + i;
+    if (r >= m) continue;
+#pragma unroll
+    for (int g = 0; g < 2; ++g) {
+      const int c = c0 + g * 64 + tx * 4;
+      const float* src = Rin + (long long)r * n;
+      float4 v4;
+      if (vec && c + 3 < n) {
+        v4 = *reinterpret_cast<const float4*>(src + c);
+      } else {
+        v4.x = (c + 0 < n) ? src[c + 0] : 0.f;
+        v4.y = (c + 1 < n) ? src[c + 1] : 0.f;
+        v4.z = (c + 2 < n) ? src[c + 2] : 0.f;
+        v4.w = (c + 3 < n) ? src[c + 3] : 0.f;
+      }
+      float v[4] = {v4.x - acc[i][4 * g], v4.y - acc[i][4 * g + 1], v4.z - acc[i][4 * g + 2], v4.w - acc[i][4 * g + 3]};
+      if (Rout != nullptr) {
+        float* dst = Rout + (long long)r * n;
+        if (vec && c + 3 < n) {
+          *reinterpret_cast<float4*>(dst + c) = make_float4(v[0], v[1], v[2], v[3]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (c + j < n) dst[c + j] = v[j];
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (c + j < n) {
+          const float sq = v[j] * v[j];
+          csum[4 * g + j] += sq;
+          nrm = fmaf(h != nullptr ? __ldg(h + c + j) : 1.f, sq, nrm);
+        }
+      }
+    }
+  }
+  if (colpart != nullptr) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) red[ty][col_of(tx, j)] = csum[j];
+    __syncthreads();
+    if (tid < TN && c0 + tid < n) {
+      float s = 0.f;
+#pragma unroll
+      for (int t = 0; t < 16; ++t) s += red[t][tid];
+      colpart[(long long)blockIdx.y * n + c0 + tid] = s;
+    }
+  }
+  double dn = warp_sum((double)nrm);
+  if ((tid & 31) == 0) wred[tid >> 5] = dn;
+  __syncthreads();
+  if (tid == 0) {
+    double s = 0.0;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) s += wred[q];
+    normpart[(long long)blockIdx.y * gridDim.x + blockIdx.x] = s;
+  }
+}
+
+// Split-K factor: enough CTAs to cover the GPU twice, each split at least 64 deep and a multiple of TK.
+void choose_split(int tiles, int Ly, int* splits, int* chunk) {
+  int sms = 152;
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int s = (int)cdiv(2 * sms, tiles);
+  s = max(1, min(s, (int)cdiv(Ly, 64)));
+  int c = (int)round_up(cdiv(Ly, s), TK);
+  *chunk = c;
+  *splits = (int)cdiv(Ly, c);
+}
+
+}  // namespace
+
+int product_splits(int w, int Lx, int Ly) {
+  int s, c;
+  choose_split((int)(cdiv(Lx, TN) * cdiv(w, TM)), Ly, &s, &c);
+  return s;
+}
+
+cudaError_t launch_product_v(const float* R, int m, int n, const int8_t* Ut, int ldu, int w, float* part, int splits,
+                             cudaStream_t s) {
+  // every one of the `splits` partial slices is written (an empty split writes zeros)
+  const int chunk = (int)round_up(cdiv(m, splits), TK);
+  dim3 grid((unsigned)cdiv(n, TN), (unsigned)cdiv(w, TM), (unsigned)splits);
+  product_kernel<false><<<grid, 256, 0, s>>>(R, m, n, Ut, ldu, w, nullptr, part, chunk);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int ldv, int w, const float* h,
+                             float* part, int splits, cudaStream_t s) {
+  const int chunk = (int)round_up(cdiv(n, splits), TK);
+  dim3 grid((unsigned)cdiv(m, TN), (unsigned)cdiv(w, TM), (unsigned)splits);
+  product_kernel<true><<<grid, 256, 0, s>>>(R, m, n, Vt, ldv, w, h, part, chunk);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
+                               Stats st, cudaStream_t s) {
+  dim3 grid((unsigned)cdiv(L, TN), (unsigned)cdiv(w, TM));
+  decorrelate_kernel<<<grid, 256, 0, s>>>(Ginv, w, part, splits, L, X, ldx, st);
+  return cudaGetLastError();
+}
+
+int deflate_row_tiles(int m) { return (int)cdiv(m, TM); }
+int deflate_tiles(int m, int n) { return (int)(cdiv(m, TM) * cdiv(n, TN)); }
+
+cudaError_t launch_deflate(const float* Rin, float* Rout, int m, int n, const int8_t* U, long long ldu, bool u_rowmajor,
+                           const float* d, const int8_t* Vt, long long ldv, int w, const float* h, float* colpart,
+                           double* normpart, cudaStream_t s) {
+  dim3 grid((unsigned)cdiv(n, TN), (unsigned)cdiv(m, TM));
+  if (u_rowmajor)
+    deflate_kernel<true><<<grid, 256, 0, s>>>(Rin, Rout, m, n, U, ldu, d, Vt, ldv, w, h, colpart, normpart);
+  else
+    deflate_kernel<false><<<grid, 256, 0, s>>>(Rin, Rout, m, n, U, ldu, d, Vt, ldv, w, h, colpart, normpart);
+  return cudaGetLastError();
+}
+
+}  // namespace externd

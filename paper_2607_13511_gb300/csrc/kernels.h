@@ -1,0 +1,80 @@
+// Internal launch interface of the ExTernD kernels (host side). Not part of the public C ABI.
+//
+// Internal layouts (all row-major):
+//   R      m x n float32 residual (ld n).
+//   Ut     w x ldu int8: row a is component a's u (length m; ldu = round_up(m, 16), zero padded).
+//   Vt     w x ldv int8: row a is component a's v (length n; ldv = round_up(n, 16), zero padded) = a block of C.
+//   part   splits x w x L float32: split-K partial products; L = n for the V-step, m for the U-step.
+//   X      w x ldx float32: decorrelated targets, one vector per row (the Eq. 2 input).
+//   Stats  per-vector partials of the Eq. 2 statistics: spart[a * nchunk + c] = sum |x| over chunk c,
+//          kpart[a * nchunk + c] = max magnitude key over chunk c (chunks of kStatChunk positions).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "common.cuh"
+
+namespace externd {
+
+struct Stats {
+  double* spart;
+  u64* kpart;
+  int nchunk;
+};
+
+// ---- products (gemm.cu)
+// Split-K factor of a product with Lx output positions per component and reduction length Ly.
+int product_splits(int w, int Lx, int Ly);
+cudaError_t launch_product_v(const float* R, int m, int n, const int8_t* Ut, int ldu, int w, float* part, int splits,
+                             cudaStream_t s);
+cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int ldv, int w, const float* h,
+                             float* part, int splits, cudaStream_t s);
+cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
+                               Stats st, cudaStream_t s);
+// Rout = Rin - U diag(d) V (Rout may alias Rin or be NULL); U is Ut (component-major, ldu) or, when
+// u_rowmajor, an m x ldu row-major block of B. colpart: [cdiv(m,64)][n] per-tile column sums of Rout^2 (or NULL);
+// normpart: [cdiv(m,64) * cdiv(n,128)] per-tile sums of h_j Rout_ij^2.
+cudaError_t launch_deflate(const float* Rin, float* Rout, int m, int n, const int8_t* U, long long ldu, bool u_rowmajor,
+                           const float* d, const int8_t* Vt, long long ldv, int w, const float* h, float* colpart,
+                           double* normpart, cudaStream_t s);
+int deflate_row_tiles(int m);
+int deflate_tiles(int m, int n);
+
+// ---- ternarization and bookkeeping (tern.cu)
+cudaError_t launch_stats(const float* X, int nv, int L, int ldx, Stats st, cudaStream_t s);
+cudaError_t launch_apply(const float* X, int nv, int L, int ldx, Stats st, double tau, int8_t* T, int ldt,
+                         cudaStream_t s);
+cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, float* Y, int ldy, Stats st,
+                          cudaStream_t s);
+// J = the w columns of largest h_c * sum_t colpart[t][c] (ties to the lower c), ascending; e (n floats) is scratch.
+cudaError_t launch_select_with(const float* colpart, int nrt, int n, const float* h, int w, int* J, float* e,
+                               cudaStream_t s);
+// out[0] = sum of count partials (fixed order); if trace != NULL, trace[0] = 1 - out[0] / norm_a[0].
+cudaError_t launch_norm(const double* normpart, int count, double* out, const double* norm_a, double* trace,
+                        cudaStream_t s);
+cudaError_t launch_write_b(const int8_t* Ut, int ldu, int w, int m, int8_t* B, long long k, long long j0,
+                           cudaStream_t s);
+// dst[c][r] = src[r][c] for an rows x cols int8 / float32 matrix (leading dims given).
+cudaError_t launch_transpose_i8(const int8_t* src, long long lds, int rows, int cols, int8_t* dst, long long ldd,
+                                cudaStream_t s);
+cudaError_t launch_transpose_f32(const float* src, long long lds, int rows, int cols, float* dst, long long ldd,
+                                 cudaStream_t s);
+// out[a][x] = sum_s part[s][a][x]
+cudaError_t launch_sum_splits(const float* part, int splits, int w, int L, float* out, long long ldo, cudaStream_t s);
+
+// ---- small dense algebra (solve.cu)
+int gram_splits(int w, int L);
+// Gpart[s][a][b] = sum_{y in split s} T[a][y] T[b][y] (* h[y] if h)
+cudaError_t launch_gram(const int8_t* T, int ldt, int w, int L, const float* h, float* Gpart, int splits,
+                        cudaStream_t s);
+// Graw = sum_s Gpart[s]; Ginv = (Graw + eps I)^-1 with eps = kEpsRel * trace / w.
+cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s);
+// r[a] = sum_y Ut[a][y] * sum_s part[s][a][y]
+cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, double* r,
+                        cudaStream_t s);
+// d solves [(sum_s GUpart[s]) .* GVraw + eps I] d = r (eps = 0 when w == 1).
+cudaError_t launch_scales(const float* GUpart, int splits, const float* GVraw, const double* r, int w, float* d,
+                          cudaStream_t s);
+
+}  // namespace externd

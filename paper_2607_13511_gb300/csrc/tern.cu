@@ -1,0 +1,345 @@
+// Eq. 2 ternarization (statistics + apply), the start of each block (top-w residual columns), and the small
+// data-movement kernels around them.
+//
+// Eq. 2: T_tau(x)_i = sign(x_i) [|x_i| > tau * (1/L) sum_j |x_j|]; if nothing passes, the single largest |x_i|
+// (first index) is kept. The sum is gathered as per-chunk partials (compensated float, combined in double) by
+// whichever kernel produces x, then summed in a fixed order by the apply kernel: theta = tau * (S / L) in double,
+// compared in float against RD_float(theta), which decides exactly like a double comparison for float x.
+#include "kernels.h"
+
+namespace externd {
+
+namespace {
+
+// Per-chunk statistics of vector a over positions [x0, x0 + 128): optionally gathering x = R[r][J[a]].
+template <bool GATHER>
+__global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X, int L, long long ldx, int ncols,
+                                                    const int* __restrict__ J, float* __restrict__ Y, long long ldy,
+                                                    Stats st) {
+  __shared__ double ssum[4];
+  __shared__ u64 skey[4];
+  const int a = blockIdx.y;
+  const int x = blockIdx.x * kStatChunk + threadIdx.x;
+  float v = 0.f;
+  bool valid = x < L;
+  if (valid) {
+    if (GATHER) {
+      const int j = min(max(__ldg(J + a), 0), ncols - 1);   // J comes from select_kernel; never read outside R
+      v = __ldg(X + (long long)x * ncols + j);
+      Y[(long long)a * ldy + x] = v;
+    } else {
+      v = __ldg(X + (long long)a * ldx + x);
+    }
+  }
+  double s = valid ? (double)fabsf(v) : 0.0;
+  u64 key = valid ? mag_key(v, (uint32_t)x) : 0ull;
+  s = warp_sum(s);
+  key = warp_max(key);
+  const int warp = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) {
+    ssum[warp] = s;
+    skey[warp] = key;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    u64 k = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      t += ssum[q];
+      k = skey[q] > k ? skey[q] : k;
+    }
+    st.spart[(long long)a * st.nchunk + blockIdx.x] = t;
+    st.kpart[(long long)a * st.nchunk + blockIdx.x] = k;
+  }
+}
+
+// Threshold of vector a from its chunk partials (warp 0, fixed order): RD_float(tau * S / L), fallback flag and
+// the fallback index.
+__device__ __forceinline__ void vector_threshold(const Stats& st, int a, int L, double tau, float* theta_dn,
+                                                 int* fallback, uint32_t* argidx) {
+  const int lane = threadIdx.x & 31;
+  double s = 0.0;
+  u64 key = 0;
+  for (int c = lane; c < st.nchunk; c += 32) {
+    s += st.spart[(long long)a * st.nchunk + c];
+    const u64 k = st.kpart[(long long)a * st.nchunk + c];
+    key = k > key ? k : key;
+  }
+  s = warp_sum(s);
+  key = warp_max(key);
+  const double theta = tau * (s / (double)L);
+  const float th = __double2float_rd(theta);
+  *theta_dn = th;
+  *fallback = !(key_mag(key) > th);
+  *argidx = key_index(key);
+}
+
+__global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X, int L, long long ldx, Stats st,
+                                                    double tau, int8_t* __restrict__ T, long long ldt) {
+  __shared__ float s_theta;
+  __shared__ int s_fallback;
+  __shared__ uint32_t s_arg;
+  const int a = blockIdx.y;
+  if (threadIdx.x < 32) {
+    float th;
+    int fb;
+    uint32_t ai;
+    vector_threshold(st, a, L, tau, &th, &fb, &ai);
+    if (threadIdx.x == 0) {
+      s_theta = th;
+      s_fallback = fb;
+      s_arg = ai;
+    }
+  }
+  __syncthreads();
+  const float th = s_theta;
+  const int fb = s_fallback;
+  const uint32_t ai = s_arg;
+  const int x0 = (blockIdx.x * 256 + threadIdx.x) * 4;
+  if (x0 >= L) return;
+  const float* src = X + (long long)a * ldx;
+  int8_t t[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int x = x0 + j;
+    t[j] = 0;
+    if (x < L) {
+      const float v = src[x];
+      t[j] = ternary_of(v, th);
+      if (fb && (uint32_t)x == ai) t[j] = v < 0.f ? (int8_t)-1 : (int8_t)1;
+    }
+  }
+  int8_t* dst = T + (long long)a * ldt + x0;
+  if ((ldt & 3) == 0 && x0 + 3 < L) {
+    *reinterpret_cast<int*>(dst) = (int)(uint8_t)t[0] | ((int)(uint8_t)t[1] << 8) | ((int)(uint8_t)t[2] << 16) |
+                                   ((int)(uint8_t)t[3] << 24);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (x0 + j < L) dst[j] = t[j];
+  }
+}
+
+// Column energies e_c = h_c * sum_t colpart[t][c].
+__global__ void colsum_kernel(const float* __restrict__ colpart, int nrt, int n, const float* __restrict__ h,
+                              float* __restrict__ e) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= n) return;
+  float s = 0.f;
+  for (int t = 0; t < nrt; ++t) s += colpart[(long long)t * n + c];
+  e[c] = (h != nullptr) ? s * __ldg(h + c) : s;
+}
+
+// Inclusive scan of one int per thread over a 1024-thread block.
+__device__ int block_scan_incl(int v, int* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += t;
+  }
+  if (lane == 31) sh[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    int t = sh[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int u = __shfl_up_sync(0xffffffffu, t, o);
+      if (lane >= o) t += u;
+    }
+    sh[lane] = t;
+  }
+  __syncthreads();
+  const int r = v + (warp > 0 ? sh[warp - 1] : 0);
+  __syncthreads();
+  return r;
+}
+
+// The w columns with the largest energy (ties to the lower index), in ascending column order. One CTA:
+// radix select of the w-th largest key (energies are non-negative floats, so their bits order like the values),
+// then an ordered compaction.
+__global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ e, int n, int w, int* __restrict__ J) {
+  __shared__ unsigned hist[256];
+  __shared__ unsigned s_bin, s_rem;
+  __shared__ int scan_sh[32];
+  const int tid = threadIdx.x;
+  const int per = (int)cdiv(n, 1024);
+  const int cb = min(n, tid * per), ce = min(n, cb + per);
+  unsigned prefix = 0, mask = 0, remaining = (unsigned)w;
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int i = tid; i < 256; i += 1024) hist[i] = 0;
+    __syncthreads();
+    for (int c = cb; c < ce; ++c) {
+      const unsigned key = __float_as_uint(e[c]);
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (tid < 32) {
+      // lane l holds bins 255-8l ... 248-8l (descending)
+      unsigned cnt[8], tot = 0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        cnt[q] = hist[255 - 8 * tid - q];
+        tot += cnt[q];
+      }
+      unsigned incl = tot;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (tid >= o) incl += t;
+      }
+      const unsigned excl = incl - tot;
+      const bool here = excl < remaining && remaining <= incl;
+      if (here) {
+        unsigned cum = excl;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          if (cum + cnt[q] >= remaining) {
+            s_bin = 255 - 8 * tid - q;
+            s_rem = remaining - cum;
+            break;
+          }
+          cum += cnt[q];
+        }
+      }
+    }
+    __syncthreads();
+    prefix |= s_bin << shift;
+    mask |= 255u << shift;
+    remaining = s_rem;
+    __syncthreads();
+  }
+  // prefix = key of the w-th largest; take every key above it and the first `remaining` keys equal to it.
+  int eq = 0;
+  for (int c = cb; c < ce; ++c) eq += (__float_as_uint(e[c]) == prefix);
+  int eq_before = block_scan_incl(eq, scan_sh) - eq;
+  int sel = 0;
+  {
+    int e_seen = eq_before;
+    for (int c = cb; c < ce; ++c) {
+      const unsigned key = __float_as_uint(e[c]);
+      if (key > prefix) ++sel;
+      else if (key == prefix) sel += (unsigned)(e_seen++) < remaining;
+    }
+  }
+  int pos = block_scan_incl(sel, scan_sh) - sel;
+  int e_seen = eq_before;
+  for (int c = cb; c < ce; ++c) {
+    const unsigned key = __float_as_uint(e[c]);
+    bool take = key > prefix;
+    if (key == prefix) take = (unsigned)(e_seen++) < remaining;
+    if (take) J[pos++] = c;
+  }
+}
+
+__global__ void norm_kernel(const double* __restrict__ part, int count, double* out, const double* norm_a,
+                            double* trace) {
+  double s = 0.0;
+  for (int i = threadIdx.x; i < count; i += 32) s += part[i];
+  s = warp_sum(s);
+  if (threadIdx.x == 0) {
+    out[0] = s;
+    if (trace != nullptr) trace[0] = 1.0 - s / norm_a[0];
+  }
+}
+
+__global__ void write_b_kernel(const int8_t* __restrict__ Ut, int ldu, int w, int m, int8_t* __restrict__ B,
+                               long long k, long long j0) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= m) return;
+  int8_t* dst = B + (long long)r * k + j0;
+  for (int a = 0; a < w; ++a) dst[a] = Ut[(long long)a * ldu + r];
+}
+
+template <typename T>
+__global__ void transpose_kernel(const T* __restrict__ src, long long lds, int rows, int cols, T* __restrict__ dst,
+                                 long long ldd) {
+  __shared__ T tile[32][33];
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = r0 + i, c = c0 + threadIdx.x;
+    if (r < rows && c < cols) tile[i][threadIdx.x] = src[(long long)r * lds + c];
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int c = c0 + i, r = r0 + threadIdx.x;
+    if (r < rows && c < cols) dst[(long long)c * ldd + r] = tile[threadIdx.x][i];
+  }
+}
+
+__global__ void sum_splits_kernel(const float* __restrict__ part, int splits, int w, int L, float* __restrict__ out,
+                                  long long ldo) {
+  const int a = blockIdx.y;
+  const int x = blockIdx.x * blockDim.x + threadIdx.x;
+  if (x >= L) return;
+  float s = 0.f;
+  for (int q = 0; q < splits; ++q) s += part[((long long)q * w + a) * L + x];
+  out[(long long)a * ldo + x] = s;
+}
+
+}  // namespace
+
+cudaError_t launch_stats(const float* X, int nv, int L, int ldx, Stats st, cudaStream_t s) {
+  dim3 grid((unsigned)cdiv(L, kStatChunk), (unsigned)nv);
+  stats_kernel<false><<<grid, kStatChunk, 0, s>>>(X, L, ldx, 0, nullptr, nullptr, 0, st);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, float* Y, int ldy, Stats st,
+                          cudaStream_t s) {
+  dim3 grid((unsigned)cdiv(m, kStatChunk), (unsigned)w);
+  stats_kernel<true><<<grid, kStatChunk, 0, s>>>(R, m, 0, n, J, Y, ldy, st);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_apply(const float* X, int nv, int L, int ldx, Stats st, double tau, int8_t* T, int ldt,
+                         cudaStream_t s) {
+  dim3 grid((unsigned)cdiv(L, 1024), (unsigned)nv);
+  apply_kernel<<<grid, 256, 0, s>>>(X, L, ldx, st, tau, T, ldt);
+  return cudaGetLastError();
+}
+
+// e (n floats) is scratch for the column energies.
+cudaError_t launch_select_with(const float* colpart, int nrt, int n, const float* h, int w, int* J, float* e,
+                               cudaStream_t s) {
+  colsum_kernel<<<(unsigned)cdiv(n, 256), 256, 0, s>>>(colpart, nrt, n, h, e);
+  cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  select_kernel<<<1, 1024, 0, s>>>(e, n, w, J);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_norm(const double* normpart, int count, double* out, const double* norm_a, double* trace,
+                        cudaStream_t s) {
+  norm_kernel<<<1, 32, 0, s>>>(normpart, count, out, norm_a, trace);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_write_b(const int8_t* Ut, int ldu, int w, int m, int8_t* B, long long k, long long j0,
+                           cudaStream_t s) {
+  write_b_kernel<<<(unsigned)cdiv(m, 256), 256, 0, s>>>(Ut, ldu, w, m, B, k, j0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_transpose_i8(const int8_t* src, long long lds, int rows, int cols, int8_t* dst, long long ldd,
+                                cudaStream_t s) {
+  dim3 grid((unsigned)cdiv(cols, 32), (unsigned)cdiv(rows, 32));
+  transpose_kernel<int8_t><<<grid, dim3(32, 8), 0, s>>>(src, lds, rows, cols, dst, ldd);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_transpose_f32(const float* src, long long lds, int rows, int cols, float* dst, long long ldd,
+                                 cudaStream_t s) {
+  dim3 grid((unsigned)cdiv(cols, 32), (unsigned)cdiv(rows, 32));
+  transpose_kernel<float><<<grid, dim3(32, 8), 0, s>>>(src, lds, rows, cols, dst, ldd);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sum_splits(const float* part, int splits, int w, int L, float* out, long long ldo, cudaStream_t s) {
+  dim3 grid((unsigned)cdiv(L, 256), (unsigned)w);
+  sum_splits_kernel<<<grid, 256, 0, s>>>(part, splits, w, L, out, ldo);
+  return cudaGetLastError();
+}
+
+}  // namespace externd

@@ -1,0 +1,83 @@
+"""The C-ABI library builds, loads and exports every entry point include/externd.h declares (no GPU needed).
+
+Only host-side functions (rank, block width, status strings) are called here: no compute call without a GPU.
+"""
+import ctypes
+import os
+import re
+import shutil
+
+import pytest
+
+from oracle import externd_oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "externd.h")
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(externd_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("nvcc not available")
+    from paper_2607_13511_gb300 import build
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def test_header_declares_the_boundary():
+    syms = declared_symbols()
+    for name in ("externd_decompose", "externd_energy", "externd_rank", "externd_set_stream", "externd_strerror",
+                 "externd_ternarize", "externd_vstep_product", "externd_ustep_product", "externd_block_scales",
+                 "externd_deflate"):
+        assert name in syms
+
+
+def test_library_exports_every_declared_symbol(lib):
+    missing = [s for s in declared_symbols() if not hasattr(lib, s)]
+    assert not missing, missing
+
+
+def test_binding_declares_every_symbol():
+    import paper_2607_13511_gb300 as X
+    assert sorted(X._SIGNATURES) == declared_symbols()
+
+
+def test_host_side_rank_and_block_width_match_the_oracle(lib):
+    rank = lib.externd_rank
+    rank.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_double, ctypes.POINTER(ctypes.c_int64)]
+    bw = lib.externd_block_width
+    bw.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.POINTER(ctypes.c_int)]
+    k = ctypes.c_int64()
+    b = ctypes.c_int()
+    for m, n, mu in [(256, 256, 2.0), (2048, 2048, 3.0), (2560, 9728, 3.0), (4096, 4096, 2.5), (10, 7, 0.5),
+                     (10, 7, 0.2), (3, 1000, 1.7), (1, 1, 1.0)]:
+        assert rank(m, n, mu, ctypes.byref(k)) == 0
+        assert k.value == O.inner_rank(m, n, mu)
+    for m, n, block in [(2048, 2048, 64), (2560, 1024, 256), (256, 256, 1), (12, 40, 64), (7, 7, 16), (9, 9, 200)]:
+        assert bw(m, n, block, ctypes.byref(b)) == 0
+        assert b.value == O.block_width(m, n, block)
+
+
+def test_host_side_argument_errors(lib):
+    rank = lib.externd_rank
+    rank.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_double, ctypes.POINTER(ctypes.c_int64)]
+    k = ctypes.c_int64()
+    assert rank(0, 5, 1.0, ctypes.byref(k)) == -1
+    assert rank(5, 5, 0.0, ctypes.byref(k)) == -1
+    assert rank(5, 5, float("nan"), ctypes.byref(k)) == -1
+    assert rank(5, 5, 1.0, None) == -1
+    bw = lib.externd_block_width
+    bw.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.POINTER(ctypes.c_int)]
+    b = ctypes.c_int()
+    assert bw(5, 5, 0, ctypes.byref(b)) == -1
+    assert bw(5000, 5000, 257, ctypes.byref(b)) == -1     # widest supported block is 256
+    se = lib.externd_strerror
+    se.restype = ctypes.c_char_p
+    for code in (0, -1, -2, -3, -4, -5, 7):
+        assert se(code)
