@@ -1,0 +1,364 @@
+#!/usr/bin/env python3
+"""Throughput of the GB300 ExTernD library: ternary components fitted per second.
+
+One step is one complete decomposition of one synthetic matrix (every block, every ALS iteration, the joint
+scales and the deflation), by default the 2048 x 2048 N(0, 0.02^2) matrix with 0.1 % outliers x20, mu = 3
+(k = 6144 components), tau = 0.7, block 64, 4 ALS iterations. The matrix is generated once, resident in HBM;
+its 16.8 MB residual fits in L2, so L2 is flushed (a 512 MB write) before every step, inside the timed region.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference] [--workload NAME]
+
+With N > 1 (torchrun, one rank per GPU) every rank decomposes its own matrix (independent problems, no
+collective on the data path): value = all ranks' components / the slowest rank's time ("scaling": "weak").
+``--impl reference`` times the CPU oracle (the plain fp64 restatement of the method) on a bounded sample of the
+same workload: the first blocks of the same matrix, which by the greedy prefix property are the same work.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2607_13511_gb300 import workloads as W  # noqa: E402
+
+METRIC = "ternary components fitted/sec per matrix"
+UNIT = "components/s"
+DEFAULT_WORKLOAD = W.OUTLIER_2048.name
+ROOFLINE_KIND = "vstep"   # the kernel class with the largest share of device time (profiles/launches_*.md)
+
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of the profiled kernel, from one ncu capture, valid
+# only while the kernel's source is unchanged (sha256 of the file that holds it).
+NCU_TRAFFIC: dict = {}
+
+
+def env_int(name, default):
+    try:
+        return int(os.environ.get(name, default))
+    except ValueError:
+        return default
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        p = json.load(open(path))
+        return p.get("hbm_gbs", 6800.0), "measured"
+    return 6800.0, "fallback"
+
+
+def golden_energy(name):
+    path = os.path.join(ROOT, "tests", "golden", "oracle_energies.json")
+    try:
+        return json.load(open(path))[name]["energy"]
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+def workload(name) -> W.Workload:
+    return W.WORKLOADS[name]
+
+
+def block_width(wl):
+    return max(1, min(wl.block, min(wl.m, wl.n) // 8))
+
+
+def inner_rank(wl, mu=None):
+    return int(math.floor((wl.mu if mu is None else mu) * min(wl.m, wl.n) + 0.5))
+
+
+# ----------------------------------------------------------------------------------------------- CPU oracle
+def oracle_sample(wl, budget_blocks):
+    """Times the CPU oracle on the first `budget_blocks` blocks of the workload (same matrix, same parameters)."""
+    from oracle import externd_oracle as O
+    A = wl.matrix()
+    h = wl.weights()
+    b = block_width(wl)
+    k_sample = min(inner_rank(wl), budget_blocks * b)
+    mu_sample = k_sample / min(wl.m, wl.n)
+    t0 = time.perf_counter()
+    res = O.decompose(A, mu_sample, wl.tau, wl.block, wl.iters, h)
+    dt = time.perf_counter() - t0
+    assert res.D.size == k_sample
+    return k_sample, dt
+
+
+def cpu_cores():
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(var, "").isdigit():
+            return int(os.environ[var])
+    return os.cpu_count()
+
+
+def run_reference(args):
+    rank = env_int("RANK", 0)
+    if rank != 0:
+        return
+    wl = workload(args.workload)
+    blocks = args.reference_blocks
+    for _ in range(args.warmup):
+        oracle_sample(wl, blocks)
+    comps, secs = 0, 0.0
+    for _ in range(args.steps):
+        k, dt = oracle_sample(wl, blocks)
+        comps += k
+        secs += dt
+    value = comps / secs
+    sample = f"first {blocks} blocks ({comps // args.steps} of {inner_rank(wl)} components) of {wl.name} per step"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_of(wl),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_of(wl):
+    return {"workload": wl.name, "m": wl.m, "n": wl.n, "mu": wl.mu, "k": inner_rank(wl), "tau": wl.tau,
+            "block": block_width(wl), "iters": wl.iters, "weighted": wl.weighted, "matrix": wl.kind,
+            "seed": wl.seed, "l2": "flushed before every step (512 MB write, inside the timed region)"}
+
+
+# ----------------------------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{env_int('RANK', 0)}.csv")
+        self.idx = device_index
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, ValueError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return None
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------------------------- GPU arm
+def algorithmic_bytes(kind, wl):
+    """Bytes one launch of the kernel class must move at minimum (R dominates; ternary factors are int8)."""
+    m, n, b = wl.m, wl.n, block_width(wl)
+    hbytes = 4 * n if wl.weighted else 0
+    if kind == "vstep":      # read R and U, write U^T R
+        return 4 * m * n + m * b + 4 * b * n
+    if kind == "ustep":      # read R, V (and h), write R H V
+        return 4 * m * n + n * b + hbytes + 4 * m * b
+    if kind == "deflate":    # read and write R, read U, V, d
+        return 8 * m * n + (m + n) * b + 4 * b + hbytes
+    raise ValueError(kind)
+
+
+def source_sha(path):
+    return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2607_13511_gb300 as X
+
+    rank, world, local = env_int("RANK", 0), env_int("WORLD_SIZE", 1), env_int("LOCAL_RANK", 0)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    X.load()
+
+    wl = workload(args.workload)
+    A_host = torch.from_numpy(wl.matrix())
+    h_np = wl.weights()
+    A = A_host.to(dev)
+    h = None if h_np is None else torch.from_numpy(h_np).to(dev)
+    k = X.rank(wl.m, wl.n, wl.mu)
+    out = (torch.empty((wl.m, k), dtype=torch.int8, device=dev), torch.empty((k,), dtype=torch.float32, device=dev),
+           torch.empty((k, wl.n), dtype=torch.int8, device=dev))
+    flush = torch.empty(128 * 1024 * 1024, dtype=torch.float32, device=dev)   # 512 MB > L2
+
+    def step():
+        return X.decompose(A, wl.mu, wl.tau, wl.block, wl.iters, h, out=out)
+
+    for _ in range(args.warmup):
+        flush.fill_(0.0)
+        res = step()
+    launches_per_step = X.kernel_launches()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    # ---- timed region: K decompositions, device-timed with CUDA events on the current stream
+    stream = torch.cuda.current_stream(dev)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        barrier()
+        ev0.record(stream)
+        for i in range(args.steps):
+            flush.fill_(float(i))
+            res = step()
+        ev1.record(stream)
+        barrier()
+    ms = ev0.elapsed_time(ev1)
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+    value = world * k * args.steps / (ms_max / 1e3)
+    energy = res.energy
+
+    # ---- end to end through the host entry point: H2D of A (and h), decomposition, D2H of B, D, C, energies
+    A_pin = A_host.pin_memory()
+    h_pin = None if h_np is None else torch.from_numpy(h_np).pin_memory()
+    hout = (torch.empty((wl.m, k), dtype=torch.int8, pin_memory=True),
+            torch.empty((k,), dtype=torch.float32, pin_memory=True),
+            torch.empty((k, wl.n), dtype=torch.int8, pin_memory=True))
+    for _ in range(max(1, min(args.warmup, 2))):
+        X.decompose_host(A_pin, wl.mu, wl.tau, wl.block, wl.iters, h_pin, out=hout)
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(args.steps):
+        flush.fill_(float(i))
+        X.decompose_host(A_pin, wl.mu, wl.tau, wl.block, wl.iters, h_pin, out=hout)
+    e1.record(stream)
+    barrier()
+    t = torch.tensor([e0.elapsed_time(e1)], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    e2e_value = world * k * args.steps / (float(t.item()) / 1e3)
+    nblocks = -(-k // block_width(wl))
+    h2d = 4 * wl.m * wl.n + (4 * wl.n if wl.weighted else 0)
+    d2h = wl.m * k + k * wl.n + 4 * k + 8 * nblocks
+
+    # ---- live roofline of the dominant kernel: event pairs inside the graph, over a second timed pass
+    kind = args.roofline_kind
+    X.profile(kind)
+    for _ in range(2):
+        flush.fill_(0.0)
+        step()
+    X.profile_read()
+    prof_ms, prof_n = 0.0, 0
+    for i in range(args.steps):
+        flush.fill_(float(i))
+        step()
+        a, b = X.profile_read()
+        prof_ms += a
+        prof_n += b
+    X.profile("off")
+    per_launch_s = prof_ms / 1e3 / max(prof_n, 1)
+    bytes_per_launch = algorithmic_bytes(kind, wl)
+    achieved = bytes_per_launch / per_launch_s / 1e9
+    peak, peak_src = peaks()
+    src = os.path.join(ROOT, "paper_2607_13511_gb300", "csrc", NCU_TRAFFIC.get("file", "gemm.cu"))
+    traffic = None
+    if NCU_TRAFFIC.get("kind") == kind and NCU_TRAFFIC.get("sha") == source_sha(src) \
+            and NCU_TRAFFIC.get("workload") == wl.name:
+        traffic = NCU_TRAFFIC["bytes_per_launch"]
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded numpy PCG64; see workloads.py)",
+        "config": {**config_of(wl), "parallelism": f"replicas x{world}"},
+        "energy": energy,
+    }
+    g = golden_energy(wl.name)
+    line["delta_E_vs_oracle"] = None if g is None else energy - g
+    line["e2e"] = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                   "path": "externd_decompose_host (pinned host buffers)"}
+    line["gpu_launches"] = launches_per_step * args.steps
+    line["roofline"] = {"bound": "hbm", "kernel": kind, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                        "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
+                        "bytes_per_launch": bytes_per_launch, "launches": prof_n,
+                        "us_per_launch": per_launch_s * 1e6}
+    cs = clocks.summary()
+    if cs is not None:
+        line["clocks"] = cs
+    if world == 1 and not args.no_cpu_baseline:
+        kk, dt = oracle_sample(wl, args.cpu_blocks)
+        line["cpu_baseline"] = {"value": kk / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                                "sample": f"first {args.cpu_blocks} blocks ({kk} of {k} components) of {wl.name}, "
+                                          f"{dt:.1f} s"}
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(W.WORKLOADS))
+    ap.add_argument("--roofline-kind", default=ROOFLINE_KIND, choices=["vstep", "ustep", "deflate"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-blocks", type=int, default=48, help="blocks of the workload the CPU baseline times")
+    ap.add_argument("--reference-blocks", type=int, default=2, help="blocks per step of the reference arm")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

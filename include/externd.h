@@ -83,6 +83,21 @@ int externd_energy(const float *A, int64_t m, int64_t n, const int8_t *B, const 
                    int64_t k, const float *weights, double *energy);
 
 /* ---------------------------------------------------------------------------------------------------------
+ * Measurement. Not part of the method: lets a caller time one kernel class inside externd_decompose with CUDA
+ * events (recorded as nodes of the captured graph, on the stream the kernels run on).
+ *   kind: 0 off, 1 V-step product, 2 U-step product, 3 deflation, 4 decorrelation (Eq. 3), 5 Eq. 2 apply,
+ *         6 Gram matrices, 7 small solves (inverse + Eq. 4), 8 block start (select + gather).
+ * ------------------------------------------------------------------------------------------------------- */
+int externd_profile(int kind);
+
+/* Device time (ms) summed over the instrumented launches of the last externd_decompose call, and their count.
+ * Waits for that call's work to finish. */
+int externd_profile_read(double *ms, int64_t *launches);
+
+/* Number of kernels the last externd_decompose call launched (the kernel nodes of its graph). */
+int externd_kernel_launches(int64_t *count);
+
+/* ---------------------------------------------------------------------------------------------------------
  * Single steps of the method, exposed for checking each kernel on its own. U is m x w int8 (a block of B's
  * columns, row-major m x w), Cb is w x n int8 (a block of C's rows). 1 <= w <= 1024.
  * ------------------------------------------------------------------------------------------------------- */

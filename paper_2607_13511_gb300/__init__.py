@@ -16,7 +16,7 @@ from typing import Optional
 __all__ = [
     "ExterndError", "Decomposition", "library_path", "load", "rank", "block_width", "decompose", "decompose_host",
     "energy", "ternarize", "vstep_product", "ustep_product", "vstep_target", "ustep_target", "block_scales",
-    "deflate",
+    "deflate", "profile", "profile_read", "kernel_launches", "PROFILE_KINDS",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -38,6 +38,9 @@ _SIGNATURES = {
     "externd_decompose_host": (_c_int, [_c_void, _c_i64, _c_i64, _c_double, _c_double, _c_int, _c_int, _c_void,
                                         _c_void, _c_void, _c_void, _c_dptr, _c_dptr]),
     "externd_energy": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_void, _c_i64, _c_void, _c_dptr]),
+    "externd_profile": (_c_int, [_c_int]),
+    "externd_profile_read": (_c_int, [_c_dptr, ctypes.POINTER(_c_i64)]),
+    "externd_kernel_launches": (_c_int, [ctypes.POINTER(_c_i64)]),
     "externd_ternarize": (_c_int, [_c_void, _c_i64, _c_i64, _c_int, _c_double, _c_void]),
     "externd_vstep_product": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_i64, _c_void]),
     "externd_ustep_product": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_i64, _c_void, _c_void]),
@@ -101,6 +104,29 @@ def _prep(t, dtype, name):
 def _stream(lib, device) -> None:
     torch = _torch()
     lib.externd_set_stream(ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream))
+
+
+PROFILE_KINDS = {"off": 0, "vstep": 1, "ustep": 2, "deflate": 3, "decorrelate": 4, "apply": 5, "gram": 6,
+                 "solve": 7, "start": 8}
+
+
+def profile(kind: str) -> None:
+    """Times one kernel class inside later decompose calls with CUDA events (see profile_read)."""
+    _check(load().externd_profile(PROFILE_KINDS[kind]))
+
+
+def profile_read() -> tuple[float, int]:
+    """(device ms, launches) of the profiled kernel class during the last decompose call."""
+    ms, n = _c_double(), _c_i64()
+    _check(load().externd_profile_read(ctypes.byref(ms), ctypes.byref(n)))
+    return ms.value, n.value
+
+
+def kernel_launches() -> int:
+    """Kernels launched by the last decompose call."""
+    n = _c_i64()
+    _check(load().externd_kernel_launches(ctypes.byref(n)))
+    return n.value
 
 
 def rank(m: int, n: int, mu: float) -> int:

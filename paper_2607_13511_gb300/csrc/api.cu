@@ -59,6 +59,27 @@ struct Workspace {
 
 std::map<int, Workspace> g_ws;
 
+// Event-pair instrumentation of one kernel class (externd_profile) and the kernel count of the last decompose.
+struct Profile {
+  int kind = 0;
+  std::vector<cudaEvent_t> events;   // shared by every graph; a graph records events [0, used)
+  size_t used = 0;                   // events recorded by the enqueue in progress
+  size_t last_used = 0;              // events recorded by the last decompose
+  long long launches = 0;            // kernels enqueued by the enqueue in progress
+  long long last_launches = 0;
+};
+Profile g_prof;
+
+cudaError_t prof_mark(cudaStream_t s) {
+  if (g_prof.used == g_prof.events.size()) {
+    cudaEvent_t e;
+    cudaError_t err = cudaEventCreate(&e);
+    if (err != cudaSuccess) return err;
+    g_prof.events.push_back(e);
+  }
+  return cudaEventRecordWithFlags(g_prof.events[g_prof.used++], s, cudaEventRecordExternal);
+}
+
 template <typename T>
 int need(Workspace& ws, const char* name, size_t count, T** out, bool zero = false) {
   Buffer& b = ws.bufs[name];
@@ -223,6 +244,18 @@ Plan make_plan(long long m, long long n, long long k, int block, int iters, doub
     if (e_ != cudaSuccess) return cuda_fail(e_, #call); \
   } while (0)
 
+// A kernel launch of class `kind` that launches `nk` kernels: counted, and bracketed by events when profiled.
+#define KL(kind_, nk, call)                                 \
+  do {                                                      \
+    const bool prof_ = g_prof.kind == (kind_);              \
+    if (prof_) LK(prof_mark(s));                            \
+    LK(call);                                               \
+    if (prof_) LK(prof_mark(s));                            \
+    g_prof.launches += (nk);                                \
+  } while (0)
+
+enum Kind { kVstep = 1, kUstep = 2, kDeflate = 3, kDecor = 4, kApply = 5, kGram = 6, kSolve = 7, kStart = 8 };
+
 // Enqueues the whole decomposition on stream s.
 int enqueue_decompose(const Plan& p, const Bufs& B, const float* A, const float* h, int8_t* Bout, float* Dout,
                       int8_t* Cout, cudaStream_t s) {
@@ -230,39 +263,41 @@ int enqueue_decompose(const Plan& p, const Bufs& B, const float* A, const float*
   const Stats st_m{B.spart, B.kpart, p.nchunk_m};
   const Stats st_n{B.spart, B.kpart, p.nchunk_n};
   const int nrt = deflate_row_tiles(m), ntiles = deflate_tiles(m, n);
+  g_prof.used = 0;
+  g_prof.launches = 0;
   // R = A, column energies, ||A||_H^2
-  LK(launch_deflate(A, B.R, m, n, nullptr, 0, false, nullptr, nullptr, 0, 0, h, B.colpart, B.normpart, s));
-  LK(launch_norm(B.normpart, ntiles, B.norm_a, nullptr, nullptr, s));
+  KL(kDeflate, 1, launch_deflate(A, B.R, m, n, nullptr, 0, false, nullptr, nullptr, 0, 0, h, B.colpart, B.normpart, s));
+  KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_a, nullptr, nullptr, s));
   for (int blk = 0; blk < p.nblocks; ++blk) {
     const long long j0 = (long long)blk * p.b;
     const int w = (int)std::min<long long>(p.b, p.k - j0);
-    LK(launch_select_with(B.colpart, nrt, n, h, w, B.J, B.colE, s));
-    LK(launch_gather(B.R, m, n, B.J, w, B.X, m, st_m, s));
-    LK(launch_apply(B.X, w, m, m, st_m, p.tau, B.Ut, (int)p.ldm, s));
+    KL(kStart, 2, launch_select_with(B.colpart, nrt, n, h, w, B.J, B.colE, s));
+    KL(kStart, 1, launch_gather(B.R, m, n, B.J, w, B.X, m, st_m, s));
+    KL(kApply, 1, launch_apply(B.X, w, m, m, st_m, p.tau, B.Ut, (int)p.ldm, s));
     for (int it = 0; it < p.iters; ++it) {
       // V-step: V <- T([(U^T U + eps I)^-1 U^T R]^T)   (plain R even when weighted, §2.5)
       if (w > 1) {
-        LK(launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
-        LK(launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, s));
+        KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
+        KL(kSolve, 1, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, s));
       }
-      LK(launch_product_v(B.R, m, n, B.Ut, (int)p.ldm, w, B.part, p.sv, s));
-      LK(launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, p.sv, n, B.X, n, st_n, s));
-      LK(launch_apply(B.X, w, n, n, st_n, p.tau, B.Vt, (int)p.ldn, s));
+      KL(kVstep, 1, launch_product_v(B.R, m, n, B.Ut, (int)p.ldm, w, B.part, p.sv, s));
+      KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, p.sv, n, B.X, n, st_n, s));
+      KL(kApply, 1, launch_apply(B.X, w, n, n, st_n, p.tau, B.Vt, (int)p.ldn, s));
       // U-step: U <- T(R H V (V^T H V + eps I)^-1)
-      LK(launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, s));
-      LK(launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, s));
-      LK(launch_product_u(B.R, m, n, B.Vt, (int)p.ldn, w, h, B.part, p.su, s));
-      LK(launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, p.su, m, B.X, m, st_m, s));
-      LK(launch_apply(B.X, w, m, m, st_m, p.tau, B.Ut, (int)p.ldm, s));
+      KL(kGram, 1, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, s));
+      KL(kSolve, 1, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, s));
+      KL(kUstep, 1, launch_product_u(B.R, m, n, B.Vt, (int)p.ldn, w, h, B.part, p.su, s));
+      KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, p.su, m, B.X, m, st_m, s));
+      KL(kApply, 1, launch_apply(B.X, w, m, m, st_m, p.tau, B.Ut, (int)p.ldm, s));
     }
     // Eq. 4: [(U^T U) .* (V^T H V)] d = diag(U^T R H V), with R H V the last U-step product
-    LK(launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
-    LK(launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, p.su, B.r, s));
-    LK(launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s));
+    KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
+    KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, p.su, B.r, s));
+    KL(kSolve, 1, launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s));
     // R <- R - U diag(d) V^T
-    LK(launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart, B.normpart, s));
-    LK(launch_norm(B.normpart, ntiles, B.norm_r, B.norm_a, B.trace + blk, s));
-    LK(launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, s));
+    KL(kDeflate, 1, launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart, B.normpart, s));
+    KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_r, B.norm_a, B.trace + blk, s));
+    KL(0, 1, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, s));
     LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
                          cudaMemcpyDeviceToDevice, s));
     LK(cudaMemcpyAsync(Dout + j0, B.d, sizeof(float) * w, cudaMemcpyDeviceToDevice, s));
@@ -276,13 +311,20 @@ struct GraphKey {
   int b, iters;
   double tau;
   unsigned gen;
+  int prof;
   bool operator<(const GraphKey& o) const {
-    return std::tie(A, h, B, D, C, m, n, k, b, iters, tau, gen) <
-           std::tie(o.A, o.h, o.B, o.D, o.C, o.m, o.n, o.k, o.b, o.iters, o.tau, o.gen);
+    return std::tie(A, h, B, D, C, m, n, k, b, iters, tau, gen, prof) <
+           std::tie(o.A, o.h, o.B, o.D, o.C, o.m, o.n, o.k, o.b, o.iters, o.tau, o.gen, o.prof);
   }
 };
 
-std::map<int, std::map<GraphKey, cudaGraphExec_t>> g_graphs;
+struct CachedGraph {
+  cudaGraphExec_t exec;
+  size_t events;        // profiling events the graph records
+  long long launches;   // kernel nodes
+};
+
+std::map<int, std::map<GraphKey, CachedGraph>> g_graphs;
 
 bool graphs_enabled() {
   const char* e = std::getenv("EXTERND_GRAPHS");
@@ -302,12 +344,12 @@ int run_decompose(const float* A, long long m, long long n, double mu, double ta
   CK(cudaGetDevice(&dev));
   cudaStream_t s = g_stream;
   if (graphs_enabled()) {
-    GraphKey key{A, h, Bout, Dout, Cout, m, n, k, p.b, iters, tau, ws->generation};
+    GraphKey key{A, h, Bout, Dout, Cout, m, n, k, p.b, iters, tau, ws->generation, g_prof.kind};
     auto& cache = g_graphs[dev];
     auto it = cache.find(key);
     if (it == cache.end()) {
       if (cache.size() >= 16) {
-        for (auto& kv : cache) cudaGraphExecDestroy(kv.second);
+        for (auto& kv : cache) cudaGraphExecDestroy(kv.second.exec);
         cache.clear();
       }
       cudaGraph_t graph;
@@ -320,11 +362,15 @@ int run_decompose(const float* A, long long m, long long n, double mu, double ta
       cudaError_t ei = cudaGraphInstantiate(&exec, graph, 0);
       cudaGraphDestroy(graph);
       if (ei != cudaSuccess) return cuda_fail(ei, "cudaGraphInstantiate");
-      it = cache.emplace(key, exec).first;
+      it = cache.emplace(key, CachedGraph{exec, g_prof.used, g_prof.launches}).first;
     }
-    CK(cudaGraphLaunch(it->second, s));
+    CK(cudaGraphLaunch(it->second.exec, s));
+    g_prof.last_used = it->second.events;
+    g_prof.last_launches = it->second.launches;
   } else {
     TRY(enqueue_decompose(p, B, A, h, Bout, Dout, Cout, s));
+    g_prof.last_used = g_prof.used;
+    g_prof.last_launches = g_prof.launches;
   }
   if (energy != nullptr || trace != nullptr) {
     void* hbuf;
@@ -402,6 +448,36 @@ const char* externd_version(void) { return "externd-gb300 0.1 (sm_103a)"; }
 int externd_set_stream(void* cuda_stream) {
   std::lock_guard<std::mutex> lock(g_mutex);
   g_stream = static_cast<cudaStream_t>(cuda_stream);
+  return EXTERND_OK;
+}
+
+int externd_profile(int kind) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (kind < 0 || kind > 8) return EXTERND_EINVAL;
+  g_prof.kind = kind;
+  return EXTERND_OK;
+}
+
+int externd_profile_read(double* ms, int64_t* launches) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (ms == nullptr || launches == nullptr) return EXTERND_EINVAL;
+  double total = 0.0;
+  const size_t n = g_prof.last_used;
+  if (n >= 2) CK(cudaEventSynchronize(g_prof.events[n - 1]));
+  for (size_t i = 0; i + 1 < n; i += 2) {
+    float t = 0.f;
+    CK(cudaEventElapsedTime(&t, g_prof.events[i], g_prof.events[i + 1]));
+    total += t;
+  }
+  *ms = total;
+  *launches = (int64_t)(n / 2);
+  return EXTERND_OK;
+}
+
+int externd_kernel_launches(int64_t* count) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (count == nullptr) return EXTERND_EINVAL;
+  *count = g_prof.last_launches;
   return EXTERND_OK;
 }
 
