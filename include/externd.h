@@ -82,6 +82,20 @@ int externd_decompose_host(const float *A, int64_t m, int64_t n, double mu, doub
 int externd_energy(const float *A, int64_t m, int64_t n, const int8_t *B, const float *D, const int8_t *C,
                    int64_t k, const float *weights, double *energy);
 
+/* The paper has no counterpart to this entry point. It is externd_energy for callers that cannot allocate
+ * device memory: a process whose framework has taken the whole GPU for its own caching allocator and forbids
+ * raw cudaMalloc, a latency-critical path that cannot afford the implicit device synchronisation of
+ * cudaMalloc/cudaFree, or a plugin that is only handed buffers. It calls no allocating routine: its scratch is
+ * a static device array of EXTERND_ENERGY_NOALLOC_SCRATCH doubles (256 KiB) that every GPU loading the library
+ * holds until the process exits. Arguments and result are those of externd_energy. Sizes whose
+ * ceil(m/64) * ceil(n/128) + 3 exceeds EXTERND_ENERGY_NOALLOC_SCRATCH return EXTERND_EINVAL (e.g. 16384 x 16000
+ * fits, 16384 x 16384 does not). The first call on each device, with that device current, looks up the
+ * array's device address; make that first call before any stream capture. All calls share the array, so calls
+ * whose work overlaps on the GPU (other threads, other streams) race on it. */
+#define EXTERND_ENERGY_NOALLOC_SCRATCH 32768
+int externd_energy_noalloc(const float *A, int64_t m, int64_t n, const int8_t *B, const float *D, const int8_t *C,
+                           int64_t k, const float *weights, double *energy);
+
 /* ---------------------------------------------------------------------------------------------------------
  * Measurement. Not part of the method: lets a caller time one kernel class inside externd_decompose with CUDA
  * events (recorded as nodes of the captured graph, on the stream the kernels run on).

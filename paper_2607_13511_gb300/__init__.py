@@ -38,6 +38,8 @@ _SIGNATURES = {
     "externd_decompose_host": (_c_int, [_c_void, _c_i64, _c_i64, _c_double, _c_double, _c_int, _c_int, _c_void,
                                         _c_void, _c_void, _c_void, _c_dptr, _c_dptr]),
     "externd_energy": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_void, _c_i64, _c_void, _c_dptr]),
+    "externd_energy_noalloc": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_void, _c_i64, _c_void,
+                                        _c_dptr]),
     "externd_profile": (_c_int, [_c_int]),
     "externd_profile_read": (_c_int, [_c_dptr, ctypes.POINTER(_c_i64)]),
     "externd_kernel_launches": (_c_int, [ctypes.POINTER(_c_i64)]),

@@ -756,3 +756,10 @@ int externd_deflate(float* R, int64_t m, int64_t n, const int8_t* U, const float
 }
 
 }  // extern "C"
+
+// Accessors for other translation units of the library (the stream, lock and error text above).
+namespace externd {
+cudaStream_t library_stream() { return g_stream; }
+std::mutex& library_mutex() { return g_mutex; }
+int record_cuda_error(cudaError_t e, const char* where) { return cuda_fail(e, where); }
+}  // namespace externd
