@@ -38,6 +38,7 @@ extern "C" {
 #define EXTERND_ENOMEM (-3)   /* device workspace allocation failed                                   */
 #define EXTERND_ECUDA (-4)    /* a CUDA call or kernel launch failed (message: externd_last_cuda_error) */
 #define EXTERND_ENODEV (-5)   /* no usable CUDA device / unsupported architecture                       */
+#define EXTERND_ETIMEOUT (-6) /* a kernel's bounded wait expired; it gave up and returned (results invalid) */
 
 /* Message for a status code (static string, never NULL). */
 const char *externd_strerror(int status);

@@ -54,6 +54,8 @@ struct Workspace {
   void* host = nullptr;        // pinned staging for results read on the host
   size_t host_cap = 0;
   cudaStream_t cap_stream = nullptr;
+  cudaStream_t side = nullptr;          // second branch of the graph: Gram + inverse beside each product
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   unsigned generation = 0;     // bumped whenever a buffer moves (invalidates captured graphs)
 };
 
@@ -126,6 +128,9 @@ int current_ws(Workspace** out) {
   }
   Workspace& ws = g_ws[dev];
   if (ws.cap_stream == nullptr) CK(cudaStreamCreateWithFlags(&ws.cap_stream, cudaStreamNonBlocking));
+  if (ws.side == nullptr) CK(cudaStreamCreateWithFlags(&ws.side, cudaStreamNonBlocking));
+  if (ws.ev_fork == nullptr) CK(cudaEventCreateWithFlags(&ws.ev_fork, cudaEventDisableTiming));
+  if (ws.ev_join == nullptr) CK(cudaEventCreateWithFlags(&ws.ev_join, cudaEventDisableTiming));
   *out = &ws;
   return EXTERND_OK;
 }
@@ -172,6 +177,32 @@ int block_width_of(long long m, long long n, int block) {
   return (int)std::max<long long>(1, b);
 }
 
+// Products run on the tensor cores for blocks of 16 or more components (the float32 FMA tiles otherwise);
+// EXTERND_TCGEN05=0 selects the FMA tiles everywhere, for comparisons.
+bool use_tc(int w) {
+  static const bool enabled = [] {
+    const char* e = std::getenv("EXTERND_TCGEN05");
+    return !(e && std::strcmp(e, "0") == 0);
+  }();
+  return enabled && w >= 16;
+}
+int splits_v(int w, int m, int n) { return use_tc(w) ? tc_product_splits(w, n, m) : product_splits(w, n, m); }
+int splits_u(int w, int m, int n) { return use_tc(w) ? tc_product_splits(w, m, n) : product_splits(w, m, n); }
+
+cudaError_t product_v(const float* R, int m, int n, const int8_t* Ut, int ldu, int w, float* part, int splits,
+                      const float* maxabs, unsigned* err, cudaStream_t s) {
+  if (use_tc(w)) return launch_product_v_tc(R, m, n, Ut, ldu, w, part, splits, maxabs, err, s);
+  return launch_product_v(R, m, n, Ut, ldu, w, part, splits, s);
+}
+cudaError_t product_u(const float* R, int m, int n, const int8_t* Vt, int ldv, int w, const float* h, float* part,
+                      int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
+  if (use_tc(w)) return launch_product_u_tc(R, m, n, Vt, ldv, w, h, part, splits, maxabs, err, s);
+  return launch_product_u(R, m, n, Vt, ldv, w, h, part, splits, s);
+}
+
+// Device error word of the bounded waits in the tensor-core kernels: nonzero -> EXTERND_ETIMEOUT (and reset).
+int check_device_error(Workspace& ws, unsigned* err, cudaStream_t s);
+
 // ------------------------------------------------------------------------------------------------------------
 // Decomposition
 // ------------------------------------------------------------------------------------------------------------
@@ -179,13 +210,14 @@ struct Plan {
   int m, n, b, iters, nblocks;
   long long k;
   double tau;
-  int sv, su, gm, gn;          // split counts: V-step, U-step, Gram over m, Gram over n
+  int gm, gn;                  // Gram split counts over m and n
   int nchunk_m, nchunk_n;
   long long ldm, ldn;
 };
 
 struct Bufs {
-  float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE;
+  float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE, *maxpart, *maxabs;
+  unsigned* err;
   int8_t *Ut, *Vt;
   double *spart, *r, *normpart, *norm_a, *norm_r, *trace;
   u64* kpart;
@@ -198,7 +230,17 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "R", (size_t)p.m * p.n, &B->R));
   TRY(need(ws, "Ut", (size_t)w * p.ldm, &B->Ut, true));
   TRY(need(ws, "Vt", (size_t)w * p.ldn, &B->Vt, true));
-  TRY(need(ws, "part", (size_t)std::max((long long)p.sv * w * p.n, (long long)p.su * w * p.m), &B->part));
+  // split-K partials for both block widths that occur (b and the tail k mod b)
+  size_t part = 0;
+  for (long long wi : {(long long)p.b, p.k % p.b}) {
+    if (wi < 1) continue;
+    part = std::max(part, (size_t)std::max((long long)splits_v((int)wi, p.m, p.n) * wi * p.n,
+                                           (long long)splits_u((int)wi, p.m, p.n) * wi * p.m));
+  }
+  TRY(need(ws, "part", part, &B->part));
+  TRY(need(ws, "maxpart", (size_t)deflate_tiles(p.m, p.n), &B->maxpart));
+  TRY(need(ws, "maxabs", 2, &B->maxabs));
+  TRY(need(ws, "err", 1, &B->err, true));
   TRY(need(ws, "X", (size_t)w * L, &B->X));
   TRY(need(ws, "spart", (size_t)w * std::max(p.nchunk_m, p.nchunk_n), &B->spart));
   TRY(need(ws, "kpart", (size_t)w * std::max(p.nchunk_m, p.nchunk_n), &B->kpart));
@@ -227,12 +269,10 @@ Plan make_plan(long long m, long long n, long long k, int block, int iters, doub
   p.iters = iters;
   p.tau = tau;
   p.nblocks = (int)cdiv(k, p.b);
-  p.sv = product_splits(p.b, p.n, p.m);
-  p.su = product_splits(p.b, p.m, p.n);
   p.gm = gram_splits(p.b, p.m);
   p.gn = gram_splits(p.b, p.n);
-  p.nchunk_m = (int)cdiv(p.m, kStatChunk);
-  p.nchunk_n = (int)cdiv(p.n, kStatChunk);
+  p.nchunk_m = std::max((int)cdiv(p.m, kStatChunk), decorrelate_chunks(p.m));
+  p.nchunk_n = std::max((int)cdiv(p.n, kStatChunk), decorrelate_chunks(p.n));
   p.ldm = ld16(m);
   p.ldn = ld16(n);
   return p;
@@ -245,58 +285,84 @@ Plan make_plan(long long m, long long n, long long k, int block, int iters, doub
   } while (0)
 
 // A kernel launch of class `kind` that launches `nk` kernels: counted, and bracketed by events when profiled.
-#define KL(kind_, nk, call)                                 \
+#define KLS(kind_, nk, st_, call)                           \
   do {                                                      \
     const bool prof_ = g_prof.kind == (kind_);              \
-    if (prof_) LK(prof_mark(s));                            \
+    if (prof_) LK(prof_mark(st_));                          \
     LK(call);                                               \
-    if (prof_) LK(prof_mark(s));                            \
+    if (prof_) LK(prof_mark(st_));                          \
     g_prof.launches += (nk);                                \
+  } while (0)
+#define KL(kind_, nk, call) KLS(kind_, nk, s, call)
+// Fork the side branch from stream s / join it back into s.
+#define FORK()                                              \
+  do {                                                      \
+    if (side == s) break;                                   \
+    LK(cudaEventRecord(ws.ev_fork, s));                     \
+    LK(cudaStreamWaitEvent(side, ws.ev_fork, 0));           \
+  } while (0)
+#define JOIN()                                              \
+  do {                                                      \
+    if (side == s) break;                                   \
+    LK(cudaEventRecord(ws.ev_join, side));                  \
+    LK(cudaStreamWaitEvent(s, ws.ev_join, 0));              \
   } while (0)
 
 enum Kind { kVstep = 1, kUstep = 2, kDeflate = 3, kDecor = 4, kApply = 5, kGram = 6, kSolve = 7, kStart = 8 };
 
 // Enqueues the whole decomposition on stream s.
-int enqueue_decompose(const Plan& p, const Bufs& B, const float* A, const float* h, int8_t* Bout, float* Dout,
-                      int8_t* Cout, cudaStream_t s) {
+int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* A, const float* h, int8_t* Bout,
+                      float* Dout, int8_t* Cout, cudaStream_t s) {
+  cudaStream_t side = ws.side;
   const int m = p.m, n = p.n;
-  const Stats st_m{B.spart, B.kpart, p.nchunk_m};
-  const Stats st_n{B.spart, B.kpart, p.nchunk_n};
+  // each producer of Eq. 2 statistics and its apply agree on the chunk count
+  const Stats st_g{B.spart, B.kpart, (int)cdiv(m, kStatChunk)};    // gather (block start)
+  const Stats st_m{B.spart, B.kpart, decorrelate_chunks(m)};       // U-step decorrelation
+  const Stats st_n{B.spart, B.kpart, decorrelate_chunks(n)};       // V-step decorrelation
   const int nrt = deflate_row_tiles(m), ntiles = deflate_tiles(m, n);
   g_prof.used = 0;
   g_prof.launches = 0;
   // R = A, column energies, ||A||_H^2
-  KL(kDeflate, 1, launch_deflate(A, B.R, m, n, nullptr, 0, false, nullptr, nullptr, 0, 0, h, B.colpart, B.normpart, s));
-  KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_a, nullptr, nullptr, s));
+  KL(kDeflate, 1, launch_deflate(A, B.R, m, n, nullptr, 0, false, nullptr, nullptr, 0, 0, h, B.colpart, B.normpart, s,
+                                 B.maxpart));
+  KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_a, nullptr, nullptr, s, B.maxpart, B.maxabs));
+  if (h != nullptr) KL(0, 1, launch_absmax(h, n, B.maxabs + 1, s));
   for (int blk = 0; blk < p.nblocks; ++blk) {
     const long long j0 = (long long)blk * p.b;
     const int w = (int)std::min<long long>(p.b, p.k - j0);
+    const int sv = splits_v(w, m, n), su = splits_u(w, m, n);
     KL(kStart, 2, launch_select_with(B.colpart, nrt, n, h, w, B.J, B.colE, s));
-    KL(kStart, 1, launch_gather(B.R, m, n, B.J, w, B.X, m, st_m, s));
-    KL(kApply, 1, launch_apply(B.X, w, m, m, st_m, p.tau, B.Ut, (int)p.ldm, s));
+    KL(kStart, 1, launch_gather(B.R, m, n, B.J, w, B.X, m, st_g, s));
+    KL(kApply, 1, launch_apply(B.X, w, m, m, st_g, p.tau, B.Ut, (int)p.ldm, s));
     for (int it = 0; it < p.iters; ++it) {
-      // V-step: V <- T([(U^T U + eps I)^-1 U^T R]^T)   (plain R even when weighted, §2.5)
+      // V-step: V <- T([(U^T U + eps I)^-1 U^T R]^T)   (plain R even when weighted, §2.5).
+      // The Gram inverse depends only on U: it runs on the side branch while the product streams R.
       if (w > 1) {
-        KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
-        KL(kSolve, 1, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, s));
+        FORK();
+        KLS(kGram, 1, side, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, side));
+        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side));
       }
-      KL(kVstep, 1, launch_product_v(B.R, m, n, B.Ut, (int)p.ldm, w, B.part, p.sv, s));
-      KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, p.sv, n, B.X, n, st_n, s));
+      KL(kVstep, 1, product_v(B.R, m, n, B.Ut, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
+      if (w > 1) JOIN();
+      KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, sv, n, B.X, n, st_n, s));
       KL(kApply, 1, launch_apply(B.X, w, n, n, st_n, p.tau, B.Vt, (int)p.ldn, s));
       // U-step: U <- T(R H V (V^T H V + eps I)^-1)
-      KL(kGram, 1, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, s));
-      KL(kSolve, 1, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, s));
-      KL(kUstep, 1, launch_product_u(B.R, m, n, B.Vt, (int)p.ldn, w, h, B.part, p.su, s));
-      KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, p.su, m, B.X, m, st_m, s));
+      FORK();
+      KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
+      KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side));
+      KL(kUstep, 1, product_u(B.R, m, n, B.Vt, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s));
+      JOIN();
+      KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, su, m, B.X, m, st_m, s));
       KL(kApply, 1, launch_apply(B.X, w, m, m, st_m, p.tau, B.Ut, (int)p.ldm, s));
     }
     // Eq. 4: [(U^T U) .* (V^T H V)] d = diag(U^T R H V), with R H V the last U-step product
     KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
-    KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, p.su, B.r, s));
+    KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, su, B.r, s));
     KL(kSolve, 1, launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s));
     // R <- R - U diag(d) V^T
-    KL(kDeflate, 1, launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart, B.normpart, s));
-    KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_r, B.norm_a, B.trace + blk, s));
+    KL(kDeflate, 1, launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart, B.normpart,
+                                   s, B.maxpart));
+    KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_r, B.norm_a, B.trace + blk, s, B.maxpart, B.maxabs));
     KL(0, 1, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, s));
     LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
                          cudaMemcpyDeviceToDevice, s));
@@ -354,7 +420,7 @@ int run_decompose(const float* A, long long m, long long n, double mu, double ta
       }
       cudaGraph_t graph;
       CK(cudaStreamBeginCapture(ws->cap_stream, cudaStreamCaptureModeThreadLocal));
-      int rc = enqueue_decompose(p, B, A, h, Bout, Dout, Cout, ws->cap_stream);
+      int rc = enqueue_decompose(*ws, p, B, A, h, Bout, Dout, Cout, ws->cap_stream);
       cudaError_t ec = cudaStreamEndCapture(ws->cap_stream, &graph);
       if (rc != EXTERND_OK) return rc;
       if (ec != cudaSuccess) return cuda_fail(ec, "cudaStreamEndCapture");
@@ -368,7 +434,7 @@ int run_decompose(const float* A, long long m, long long n, double mu, double ta
     g_prof.last_used = it->second.events;
     g_prof.last_launches = it->second.launches;
   } else {
-    TRY(enqueue_decompose(p, B, A, h, Bout, Dout, Cout, s));
+    TRY(enqueue_decompose(*ws, p, B, A, h, Bout, Dout, Cout, s));
     g_prof.last_used = g_prof.used;
     g_prof.last_launches = g_prof.launches;
   }
@@ -380,8 +446,22 @@ int run_decompose(const float* A, long long m, long long n, double mu, double ta
     const double* tr = static_cast<const double*>(hbuf);
     if (energy) *energy = tr[p.nblocks - 1];
     if (trace) std::memcpy(trace, tr, sizeof(double) * p.nblocks);
+    TRY(check_device_error(*ws, B.err, s));
   }
   CK(cudaGetLastError());
+  return EXTERND_OK;
+}
+
+int check_device_error(Workspace& ws, unsigned* err, cudaStream_t s) {
+  void* hb;
+  TRY(need_host(ws, sizeof(double), &hb));
+  CK(cudaMemcpyAsync(hb, err, sizeof(unsigned), cudaMemcpyDeviceToHost, s));
+  CK(cudaStreamSynchronize(s));
+  if (*static_cast<unsigned*>(hb) != 0u) {
+    CK(cudaMemsetAsync(err, 0, sizeof(unsigned), s));
+    CK(cudaStreamSynchronize(s));
+    return EXTERND_ETIMEOUT;
+  }
   return EXTERND_OK;
 }
 
@@ -401,6 +481,16 @@ int check_params(double mu, double tau, int block, int iters) {
 }
 
 int check_dev(const void* p) { return is_device_ptr(p) ? EXTERND_OK : (p ? EXTERND_EPTR : EXTERND_EINVAL); }
+
+// Per-step helpers: the fp16 scaling scalars {max |R|, max h} and the error word for a tensor-core product.
+int step_scalars(Workspace& ws, const float* R, long long count, const float* h, long long n, float** mx,
+                 unsigned** err) {
+  TRY(need(ws, "step.maxabs", 2, mx));
+  TRY(need(ws, "err", 1, err, true));
+  LK(launch_absmax(R, count, *mx, g_stream));
+  if (h != nullptr) LK(launch_absmax(h, n, *mx + 1, g_stream));
+  return EXTERND_OK;
+}
 
 // Per-step helpers: bring a caller's m x w U into the internal Ut layout, and a w x n Cb into Vt.
 int stage_u(Workspace& ws, const int8_t* U, long long m, int w, int8_t** Ut) {
@@ -437,6 +527,7 @@ const char* externd_strerror(int status) {
     case EXTERND_ENOMEM: return "device workspace allocation failed";
     case EXTERND_ECUDA: return "CUDA error (see externd_last_cuda_error)";
     case EXTERND_ENODEV: return "no usable CUDA device";
+    case EXTERND_ETIMEOUT: return "a bounded device wait expired (a kernel gave up and returned)";
     default: return "unknown status";
   }
 }
@@ -610,13 +701,15 @@ int externd_vstep_product(const float* R, int64_t m, int64_t n, const int8_t* U,
   Workspace* ws;
   TRY(current_ws(&ws));
   int8_t* Ut;
-  float* part;
+  float *part, *mx;
+  unsigned* err;
   TRY(stage_u(*ws, U, m, (int)w, &Ut));
-  const int sv = product_splits((int)w, (int)n, (int)m);
+  TRY(step_scalars(*ws, R, m * n, nullptr, 0, &mx, &err));
+  const int sv = splits_v((int)w, (int)m, (int)n);
   TRY(need(*ws, "part", (size_t)sv * w * n, &part));
-  LK(launch_product_v(R, (int)m, (int)n, Ut, (int)ld16(m), (int)w, part, sv, g_stream));
+  LK(product_v(R, (int)m, (int)n, Ut, (int)ld16(m), (int)w, part, sv, mx, err, g_stream));
   LK(launch_sum_splits(part, sv, (int)w, (int)n, PV, n, g_stream));
-  return EXTERND_OK;
+  return check_device_error(*ws, err, g_stream);
 }
 
 int externd_ustep_product(const float* R, int64_t m, int64_t n, const int8_t* Cb, int64_t w, const float* weights,
@@ -629,15 +722,17 @@ int externd_ustep_product(const float* R, int64_t m, int64_t n, const int8_t* Cb
   Workspace* ws;
   TRY(current_ws(&ws));
   int8_t* Vt;
-  float *part, *X;
+  float *part, *X, *mx;
+  unsigned* err;
   TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
-  const int su = product_splits((int)w, (int)m, (int)n);
+  TRY(step_scalars(*ws, R, m * n, weights, n, &mx, &err));
+  const int su = splits_u((int)w, (int)m, (int)n);
   TRY(need(*ws, "part", (size_t)su * w * m, &part));
   TRY(need(*ws, "X", (size_t)w * m, &X));
-  LK(launch_product_u(R, (int)m, (int)n, Vt, (int)ld16(n), (int)w, weights, part, su, g_stream));
+  LK(product_u(R, (int)m, (int)n, Vt, (int)ld16(n), (int)w, weights, part, su, mx, err, g_stream));
   LK(launch_sum_splits(part, su, (int)w, (int)m, X, m, g_stream));
   LK(launch_transpose_f32(X, m, (int)w, (int)m, PU, w, g_stream));
-  return EXTERND_OK;
+  return check_device_error(*ws, err, g_stream);
 }
 
 namespace {
@@ -646,7 +741,7 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   Workspace* ws;
   TRY(current_ws(&ws));
   const long long L = vstep ? n : m;
-  const int nchunk = (int)cdiv(L, kStatChunk);
+  const int nchunk = decorrelate_chunks((int)L);
   int8_t* T;
   float *part, *X, *Gpart, *Graw, *Ginv, *one;
   double* sp;
@@ -655,7 +750,10 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   else TRY(stage_v(*ws, F, n, w, &T));
   const long long ldt = vstep ? ld16(m) : ld16(n);
   const long long Lred = vstep ? m : n;
-  const int splits = product_splits(w, (int)L, (int)Lred);
+  float* mx;
+  unsigned* err;
+  TRY(step_scalars(*ws, R, m * n, vstep ? nullptr : h, n, &mx, &err));
+  const int splits = vstep ? splits_v(w, (int)m, (int)n) : splits_u(w, (int)m, (int)n);
   const int gs = gram_splits(w, (int)Lred);
   TRY(need(*ws, "part", (size_t)splits * w * L, &part));
   TRY(need(*ws, "X", (size_t)w * L, &X));
@@ -665,8 +763,8 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   TRY(need(*ws, "spart", (size_t)w * nchunk, &sp));
   TRY(need(*ws, "kpart", (size_t)w * nchunk, &kp));
   TRY(get_one(*ws, &one));
-  if (vstep) LK(launch_product_v(R, (int)m, (int)n, T, (int)ldt, w, part, splits, g_stream));
-  else LK(launch_product_u(R, (int)m, (int)n, T, (int)ldt, w, h, part, splits, g_stream));
+  if (vstep) LK(product_v(R, (int)m, (int)n, T, (int)ldt, w, part, splits, mx, err, g_stream));
+  else LK(product_u(R, (int)m, (int)n, T, (int)ldt, w, h, part, splits, mx, err, g_stream));
   if (w > 1) {
     LK(launch_gram(T, (int)ldt, w, (int)Lred, vstep ? nullptr : h, Gpart, gs, g_stream));
     LK(launch_inverse(Gpart, gs, w, Graw, Ginv, g_stream));
@@ -678,7 +776,7 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
     LK(launch_decorrelate(w > 1 ? Ginv : one, w, part, splits, (int)L, X, (int)L, st, g_stream));
     LK(launch_transpose_f32(X, L, w, (int)L, out, w, g_stream));
   }
-  return EXTERND_OK;
+  return check_device_error(*ws, err, g_stream);
 }
 }  // namespace
 
@@ -711,24 +809,26 @@ int externd_block_scales(const float* R, int64_t m, int64_t n, const int8_t* U, 
   Workspace* ws;
   TRY(current_ws(&ws));
   int8_t *Ut, *Vt;
-  float *part, *Gpart, *GrawV, *Ginv;
+  float *part, *Gpart, *GrawV, *Ginv, *mx;
+  unsigned* err;
   double* r;
   TRY(stage_u(*ws, U, m, (int)w, &Ut));
   TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
-  const int su = product_splits((int)w, (int)m, (int)n);
+  TRY(step_scalars(*ws, R, m * n, weights, n, &mx, &err));
+  const int su = splits_u((int)w, (int)m, (int)n);
   const int gm = gram_splits((int)w, (int)m), gn = gram_splits((int)w, (int)n);
   TRY(need(*ws, "part", (size_t)su * w * m, &part));
   TRY(need(*ws, "Gpart", (size_t)std::max(gm, gn) * w * w, &Gpart));
   TRY(need(*ws, "GrawV", (size_t)w * w, &GrawV));
   TRY(need(*ws, "Ginv", (size_t)w * w, &Ginv));
   TRY(need(*ws, "r", (size_t)w, &r));
-  LK(launch_product_u(R, (int)m, (int)n, Vt, (int)ld16(n), (int)w, weights, part, su, g_stream));
+  LK(product_u(R, (int)m, (int)n, Vt, (int)ld16(n), (int)w, weights, part, su, mx, err, g_stream));
   LK(launch_gram(Vt, (int)ld16(n), (int)w, (int)n, weights, Gpart, gn, g_stream));
   LK(launch_inverse(Gpart, gn, (int)w, GrawV, Ginv, g_stream));
   LK(launch_gram(Ut, (int)ld16(m), (int)w, (int)m, nullptr, Gpart, gm, g_stream));
   LK(launch_rvec(Ut, (int)ld16(m), (int)w, (int)m, part, su, r, g_stream));
   LK(launch_scales(Gpart, gm, GrawV, r, (int)w, d, g_stream));
-  return EXTERND_OK;
+  return check_device_error(*ws, err, g_stream);
 }
 
 int externd_deflate(float* R, int64_t m, int64_t n, const int8_t* U, const float* d, const int8_t* Cb, int64_t w,

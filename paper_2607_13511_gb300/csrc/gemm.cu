@@ -129,35 +129,47 @@ __global__ void __launch_bounds__(256) product_kernel(const float* __restrict__ 
   }
 }
 
+// X tile of 64 components x 32 positions: thread (ty, tx) owns components ty*4..+3 at positions tx*2, tx*2+1.
+// Narrow tiles give enough CTAs to read the split-K partials in parallel at small L.
+constexpr int DX = 32;
+
 __global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restrict__ Ginv, int w,
                                                           const float* __restrict__ part, int splits, int L,
                                                           float* __restrict__ X, int ldx, Stats st) {
-  __shared__ __align__(16) float Ps[TK][TN];
+  __shared__ __align__(16) float Ps[TK][DX];
   __shared__ __align__(16) float Gs[TK][TM + 4];
-  const int x0 = blockIdx.x * TN;
+  const int x0 = blockIdx.x * DX;
   const int a0 = blockIdx.y * TM;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
-  const bool vec = (L & 3) == 0;
-  float acc[4][8];
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+  float acc[4][2] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
 
   for (int b0 = 0; b0 < w; b0 += TK) {
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      const int idx = tid + 256 * q;
-      const int kb = idx >> 5, kx = (idx & 31) * 4;
-      const int b = b0 + kb;
-      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    {
+      // Ps[kb][kx..kx+1] = sum_s part[s][b0 + kb][x0 + kx..]: 16 x 32 floats, 2 per thread
+      const int kb = tid >> 4, kx = (tid & 15) * 2;
+      const int b = b0 + kb, x = x0 + kx;
+      float v0 = 0.f, v1 = 0.f;
       if (b < w) {
-        for (int s = 0; s < splits; ++s) {
-          const float4 p = load4(part + ((long long)s * w + b) * L, x0 + kx, L, vec);
-          v.x += p.x; v.y += p.y; v.z += p.z; v.w += p.w;
+        // independent loads first (8 splits at a time), then the sum in split order
+        const float* p = part + (long long)b * L + x;
+        const long long stride = (long long)w * L;
+        for (int q0 = 0; q0 < splits; q0 += 8) {
+          float a0[8], a1[8];
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const bool in = q0 + q < splits;
+            a0[q] = (in && x < L) ? p[(q0 + q) * stride] : 0.f;
+            a1[q] = (in && x + 1 < L) ? p[(q0 + q) * stride + 1] : 0.f;
+          }
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            v0 += a0[q];
+            v1 += a1[q];
+          }
         }
       }
-      *reinterpret_cast<float4*>(&Ps[kb][kx]) = v;
+      Ps[kb][kx] = v0;
+      Ps[kb][kx + 1] = v1;
     }
     {
       const int kb = tid >> 4, a4 = (tid & 15) * 4;
@@ -167,7 +179,15 @@ __global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restric
       *reinterpret_cast<float4*>(&Gs[kb][a4]) = g;
     }
     __syncthreads();
-    tile_fma(Gs, Ps, tx, ty, acc);
+#pragma unroll
+    for (int k = 0; k < TK; ++k) {
+      const float4 g = *reinterpret_cast<const float4*>(&Gs[k][ty * 4]);
+      const float2 p = *reinterpret_cast<const float2*>(&Ps[k][tx * 2]);
+      acc[0][0] = fmaf(g.x, p.x, acc[0][0]); acc[0][1] = fmaf(g.x, p.y, acc[0][1]);
+      acc[1][0] = fmaf(g.y, p.x, acc[1][0]); acc[1][1] = fmaf(g.y, p.y, acc[1][1]);
+      acc[2][0] = fmaf(g.z, p.x, acc[2][0]); acc[2][1] = fmaf(g.z, p.y, acc[2][1]);
+      acc[3][0] = fmaf(g.w, p.x, acc[3][0]); acc[3][1] = fmaf(g.w, p.y, acc[3][1]);
+    }
     __syncthreads();
   }
 
@@ -178,8 +198,8 @@ __global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restric
     u64 key = 0;
     if (a < w) {
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int x = x0 + col_of(tx, j);
+      for (int j = 0; j < 2; ++j) {
+        const int x = x0 + tx * 2 + j;
         if (x < L) {
           X[(long long)a * ldx + x] = acc[i][j];
           sum.add(acc[i][j]);
@@ -207,8 +227,10 @@ __global__ void __launch_bounds__(256) deflate_kernel(const float* Rin, float* R
                                                       const int8_t* __restrict__ U, long long ldu,
                                                       const float* __restrict__ d, const int8_t* __restrict__ V,
                                                       long long ldv, int w, const float* __restrict__ h,
-                                                      float* __restrict__ colpart, double* __restrict__ normpart) {
+                                                      float* __restrict__ colpart, double* __restrict__ normpart,
+                                                      float* __restrict__ maxpart) {
   __shared__ __align__(16) float As[TK][TM + 4];
+  __shared__ float wmax[8];
   __shared__ __align__(16) float Bs[TK][TN];
   __shared__ float red[16][TN];
   __shared__ double wred[8];
@@ -259,7 +281,7 @@ __global__ void __launch_bounds__(256) deflate_kernel(const float* Rin, float* R
   float csum[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) csum[j] = 0.f;
-  float nrm = 0.f;
+  float nrm = 0.f, vmax = 0.f;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int r = r0 + ty * 4 + i;
@@ -294,6 +316,7 @@ __global__ void __launch_bounds__(256) deflate_kernel(const float* Rin, float* R
           const float sq = v[j] * v[j];
           csum[4 * g + j] += sq;
           nrm = fmaf(h != nullptr ? __ldg(h + c + j) : 1.f, sq, nrm);
+          vmax = fmaxf(vmax, fabsf(v[j]));
         }
       }
     }
@@ -310,17 +333,29 @@ __global__ void __launch_bounds__(256) deflate_kernel(const float* Rin, float* R
     }
   }
   double dn = warp_sum((double)nrm);
-  if ((tid & 31) == 0) wred[tid >> 5] = dn;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
+  if ((tid & 31) == 0) {
+    wred[tid >> 5] = dn;
+    wmax[tid >> 5] = vmax;
+  }
   __syncthreads();
   if (tid == 0) {
     double s = 0.0;
+    float mx = 0.f;
 #pragma unroll
-    for (int q = 0; q < 8; ++q) s += wred[q];
-    normpart[(long long)blockIdx.y * gridDim.x + blockIdx.x] = s;
+    for (int q = 0; q < 8; ++q) {
+      s += wred[q];
+      mx = fmaxf(mx, wmax[q]);
+    }
+    const long long tile = (long long)blockIdx.y * gridDim.x + blockIdx.x;
+    normpart[tile] = s;
+    if (maxpart != nullptr) maxpart[tile] = mx;
   }
 }
 
-// Split-K factor: enough CTAs to cover the GPU twice, each split at least 64 deep and a multiple of TK.
+// Split-K factor: enough CTAs to cover the GPU twice (the float32 FMA tiles need the warps), each split at
+// least 64 deep and a multiple of TK.
 void choose_split(int tiles, int Ly, int* splits, int* chunk) {
   int sms = 152;
   int dev = 0;
@@ -357,9 +392,11 @@ cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int
   return cudaGetLastError();
 }
 
+int decorrelate_chunks(int L) { return (int)cdiv(L, DX); }
+
 cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
                                Stats st, cudaStream_t s) {
-  dim3 grid((unsigned)cdiv(L, TN), (unsigned)cdiv(w, TM));
+  dim3 grid((unsigned)cdiv(L, DX), (unsigned)cdiv(w, TM));
   decorrelate_kernel<<<grid, 256, 0, s>>>(Ginv, w, part, splits, L, X, ldx, st);
   return cudaGetLastError();
 }
@@ -369,12 +406,12 @@ int deflate_tiles(int m, int n) { return (int)(cdiv(m, TM) * cdiv(n, TN)); }
 
 cudaError_t launch_deflate(const float* Rin, float* Rout, int m, int n, const int8_t* U, long long ldu, bool u_rowmajor,
                            const float* d, const int8_t* Vt, long long ldv, int w, const float* h, float* colpart,
-                           double* normpart, cudaStream_t s) {
+                           double* normpart, cudaStream_t s, float* maxpart) {
   dim3 grid((unsigned)cdiv(n, TN), (unsigned)cdiv(m, TM));
   if (u_rowmajor)
-    deflate_kernel<true><<<grid, 256, 0, s>>>(Rin, Rout, m, n, U, ldu, d, Vt, ldv, w, h, colpart, normpart);
+    deflate_kernel<true><<<grid, 256, 0, s>>>(Rin, Rout, m, n, U, ldu, d, Vt, ldv, w, h, colpart, normpart, maxpart);
   else
-    deflate_kernel<false><<<grid, 256, 0, s>>>(Rin, Rout, m, n, U, ldu, d, Vt, ldv, w, h, colpart, normpart);
+    deflate_kernel<false><<<grid, 256, 0, s>>>(Rin, Rout, m, n, U, ldu, d, Vt, ldv, w, h, colpart, normpart, maxpart);
   return cudaGetLastError();
 }
 

@@ -30,16 +30,26 @@ cudaError_t launch_product_v(const float* R, int m, int n, const int8_t* Ut, int
                              cudaStream_t s);
 cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int ldv, int w, const float* h,
                              float* part, int splits, cudaStream_t s);
+// Statistics chunks the decorrelation writes per vector of length L.
+int decorrelate_chunks(int L);
 cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
                                Stats st, cudaStream_t s);
 // Rout = Rin - U diag(d) V (Rout may alias Rin or be NULL); U is Ut (component-major, ldu) or, when
 // u_rowmajor, an m x ldu row-major block of B. colpart: [cdiv(m,64)][n] per-tile column sums of Rout^2 (or NULL);
 // normpart: [cdiv(m,64) * cdiv(n,128)] per-tile sums of h_j Rout_ij^2.
+// maxpart (optional): per-tile max |Rout|.
 cudaError_t launch_deflate(const float* Rin, float* Rout, int m, int n, const int8_t* U, long long ldu, bool u_rowmajor,
                            const float* d, const int8_t* Vt, long long ldv, int w, const float* h, float* colpart,
-                           double* normpart, cudaStream_t s);
+                           double* normpart, cudaStream_t s, float* maxpart = nullptr);
 int deflate_row_tiles(int m);
 int deflate_tiles(int m, int n);
+
+// ---- tensor-core products (product_tc.cu): w >= 16; maxabs = {max |R|, max h}; err = device error word
+int tc_product_splits(int w, int Lx, int Ly);
+cudaError_t launch_product_v_tc(const float* R, int m, int n, const int8_t* Ut, int ldu, int w, float* part,
+                                int splits, const float* maxabs, unsigned* err, cudaStream_t s);
+cudaError_t launch_product_u_tc(const float* R, int m, int n, const int8_t* Vt, int ldv, int w, const float* h,
+                                float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s);
 
 // ---- ternarization and bookkeeping (tern.cu)
 cudaError_t launch_stats(const float* X, int nv, int L, int ldx, Stats st, cudaStream_t s);
@@ -50,9 +60,12 @@ cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, flo
 // J = the w columns of largest h_c * sum_t colpart[t][c] (ties to the lower c), ascending; e (n floats) is scratch.
 cudaError_t launch_select_with(const float* colpart, int nrt, int n, const float* h, int w, int* J, float* e,
                                cudaStream_t s);
-// out[0] = sum of count partials (fixed order); if trace != NULL, trace[0] = 1 - out[0] / norm_a[0].
+// out[0] = sum of count partials (fixed order); if trace != NULL, trace[0] = 1 - out[0] / norm_a[0];
+// if maxpart != NULL, maxout[0] = max of the count per-tile maxima.
 cudaError_t launch_norm(const double* normpart, int count, double* out, const double* norm_a, double* trace,
-                        cudaStream_t s);
+                        cudaStream_t s, const float* maxpart = nullptr, float* maxout = nullptr);
+// out[0] = max |x_i|
+cudaError_t launch_absmax(const float* x, long long n, float* out, cudaStream_t s);
 cudaError_t launch_write_b(const int8_t* Ut, int ldu, int w, int m, int8_t* B, long long k, long long j0,
                            cudaStream_t s);
 // dst[c][r] = src[r][c] for an rows x cols int8 / float32 matrix (leading dims given).

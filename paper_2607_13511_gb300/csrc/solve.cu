@@ -81,25 +81,33 @@ __global__ void __launch_bounds__(256) gram_kernel(const int8_t* __restrict__ T,
 
 // MODE 0: Graw = sum_s Gpart[s]; Ginv = (Graw + eps I)^-1.
 // MODE 1: K = (sum_s Gpart[s]) .* GVraw (+ eps I when w > 1); d = K^-1 r.
-template <int W_PAD, int MODE>
-__global__ void __launch_bounds__(1024) sweep_kernel(const float* __restrict__ Gpart, int splits, int w,
-                                                     const float* __restrict__ GVraw, const double* __restrict__ r,
-                                                     float* __restrict__ Graw, float* __restrict__ out) {
-  constexpr int TPR = 1024 / W_PAD;       // threads per row
-  constexpr int EPT = W_PAD / TPR;        // elements per thread
-  __shared__ float colk[2][W_PAD];
+//
+// Symmetric sweep: sweeping pivot k maps S to S - S[:,k] S[k,:] / p with row and column k replaced by
+// S[k,:] / p and S[k][k] by -1/p (p = S[k][k]); after all pivots S = -G^-1. Every intermediate S stays
+// symmetric, so the pivot column equals the pivot row: the threads that own row k publish it to shared memory
+// with vector stores, every thread applies the same branch-free rank-1 update to its EPT elements, and row k
+// and column k are fixed up with predicated selects. One barrier per pivot.
+template <int W_PAD, int NT, int MODE>
+__global__ void __launch_bounds__(NT) sweep_kernel(const float* __restrict__ Gpart, int splits, int w,
+                                                   const float* __restrict__ GVraw, const double* __restrict__ r,
+                                                   float* __restrict__ Graw, float* __restrict__ out) {
+  constexpr int TPR = NT / W_PAD;         // threads per row
+  constexpr int EPT = W_PAD / TPR;        // elements per thread (a multiple of 4)
+  static_assert(EPT % 4 == 0, "EPT must allow 16-byte row stores");
+  __shared__ __align__(16) float rowk[2][W_PAD];
   __shared__ double dsum[32];
   const int tid = threadIdx.x;
   const int i = tid / TPR, q = tid % TPR;
+  const int j0 = q * EPT;
   float S[EPT];
   double diag = 0.0;
 #pragma unroll
   for (int e = 0; e < EPT; ++e) {
-    const int j = q * EPT + e;
+    const int j = j0 + e;
     float v = (i == j) ? 1.f : 0.f;
     if (i < w && j < w) {
       float g = 0.f;
-      for (int s = 0; s < splits; ++s) g += Gpart[(long long)s * w * w + (long long)i * w + j];
+      for (int sp = 0; sp < splits; ++sp) g += Gpart[(long long)sp * w * w + (long long)i * w + j];
       if (MODE == 0) {
         Graw[(long long)i * w + j] = g;
       } else {
@@ -115,7 +123,7 @@ __global__ void __launch_bounds__(1024) sweep_kernel(const float* __restrict__ G
   if ((tid & 31) == 0) dsum[tid >> 5] = t;
   __syncthreads();
   if (tid < 32) {
-    double u = warp_sum(dsum[tid]);
+    double u = warp_sum(tid < NT / 32 ? dsum[tid] : 0.0);
     if (tid == 0) dsum[0] = u;
   }
   __syncthreads();
@@ -123,40 +131,40 @@ __global__ void __launch_bounds__(1024) sweep_kernel(const float* __restrict__ G
   const float eps = ridge ? (float)(kEpsRel * dsum[0] / (double)w) : 0.f;
 #pragma unroll
   for (int e = 0; e < EPT; ++e)
-    if (i < w && q * EPT + e == i) S[e] += eps;
+    if (i < w && j0 + e == i) S[e] += eps;
 
-  int buf = 0;
   for (int k = 0; k < w; ++k) {
-    if (q == k / EPT) {
-      float v = 0.f;
+    float* rk = rowk[k & 1];
+    if (i == k) {
 #pragma unroll
-      for (int e = 0; e < EPT; ++e)
-        if (e == k % EPT) v = S[e];
-      colk[buf][i] = v;
+      for (int e = 0; e < EPT; e += 4)
+        *reinterpret_cast<float4*>(&rk[j0 + e]) = make_float4(S[e], S[e + 1], S[e + 2], S[e + 3]);
     }
     __syncthreads();
-    const float ip = 1.f / colk[buf][k];
-    const float ci = colk[buf][i];
+    const float ip = __frcp_rn(rk[k]);
+    const float ci = rk[i];           // S[i][k] = S[k][i]
+    const float f = -ci * ip;
+    const bool own_row = (i == k);
 #pragma unroll
-    for (int e = 0; e < EPT; ++e) {
-      const int j = q * EPT + e;
-      const float cj = colk[buf][j];
-      if (i == k) {
-        S[e] = (j == k) ? -ip : cj * ip;
-      } else if (j == k) {
-        S[e] = ci * ip;
-      } else {
-        S[e] = fmaf(-ci * ip, cj, S[e]);
+    for (int e = 0; e < EPT; e += 4) {
+      const float4 c4 = *reinterpret_cast<const float4*>(&rk[j0 + e]);
+      const float cj[4] = {c4.x, c4.y, c4.z, c4.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int j = j0 + e + u;
+        float v = fmaf(f, cj[u], S[e + u]);
+        v = own_row ? cj[u] * ip : v;       // row k: S[k][j] / p
+        v = (j == k) ? (own_row ? -ip : ci * ip) : v;   // column k: S[i][k] / p; pivot: -1/p
+        S[e + u] = v;
       }
     }
-    buf ^= 1;
   }
 
   if (MODE == 0) {
     if (i < w) {
 #pragma unroll
       for (int e = 0; e < EPT; ++e) {
-        const int j = q * EPT + e;
+        const int j = j0 + e;
         if (j < w) out[(long long)i * w + j] = -S[e];
       }
     }
@@ -164,7 +172,7 @@ __global__ void __launch_bounds__(1024) sweep_kernel(const float* __restrict__ G
     double acc = 0.0;
 #pragma unroll
     for (int e = 0; e < EPT; ++e) {
-      const int j = q * EPT + e;
+      const int j = j0 + e;
       if (i < w && j < w) acc += -(double)S[e] * r[j];
     }
 #pragma unroll
@@ -210,10 +218,11 @@ int gram_chunk(int w, int L, int* splits) {
 template <int MODE>
 cudaError_t launch_sweep(const float* Gpart, int splits, int w, const float* GVraw, const double* r, float* Graw,
                          float* out, cudaStream_t s) {
-  if (w <= 32) sweep_kernel<32, MODE><<<1, 1024, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
-  else if (w <= 64) sweep_kernel<64, MODE><<<1, 1024, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
-  else if (w <= 128) sweep_kernel<128, MODE><<<1, 1024, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
-  else sweep_kernel<256, MODE><<<1, 1024, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
+  // 16 elements per thread up to w = 128 (one barrier per pivot; the update is a branch-free rank-1 FMA)
+  if (w <= 32) sweep_kernel<32, 128, MODE><<<1, 128, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
+  else if (w <= 64) sweep_kernel<64, 256, MODE><<<1, 256, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
+  else if (w <= 128) sweep_kernel<128, 1024, MODE><<<1, 1024, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
+  else sweep_kernel<256, 1024, MODE><<<1, 1024, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
   return cudaGetLastError();
 }
 

@@ -234,22 +234,67 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
 }
 
 __global__ void norm_kernel(const double* __restrict__ part, int count, double* out, const double* norm_a,
-                            double* trace) {
+                            double* trace, const float* __restrict__ maxpart, float* maxout) {
   double s = 0.0;
-  for (int i = threadIdx.x; i < count; i += 32) s += part[i];
+  float mx = 0.f;
+  for (int i = threadIdx.x; i < count; i += 32) {
+    s += part[i];
+    if (maxpart != nullptr) mx = fmaxf(mx, maxpart[i]);
+  }
   s = warp_sum(s);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
   if (threadIdx.x == 0) {
     out[0] = s;
     if (trace != nullptr) trace[0] = 1.0 - s / norm_a[0];
+    if (maxout != nullptr) maxout[0] = mx;
   }
 }
 
-__global__ void write_b_kernel(const int8_t* __restrict__ Ut, int ldu, int w, int m, int8_t* __restrict__ B,
-                               long long k, long long j0) {
-  const int r = blockIdx.x * blockDim.x + threadIdx.x;
-  if (r >= m) return;
-  int8_t* dst = B + (long long)r * k + j0;
-  for (int a = 0; a < w; ++a) dst[a] = Ut[(long long)a * ldu + r];
+// out[0] = max |x_i| over n floats (one CTA; the result feeds the fp16 scaling of the tensor-core products).
+__global__ void __launch_bounds__(1024) absmax_kernel(const float* __restrict__ x, long long n, float* out) {
+  __shared__ float red[32];
+  float mx = 0.f;
+  for (long long i = threadIdx.x; i < n; i += 1024) mx = fmaxf(mx, fabsf(x[i]));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    mx = red[threadIdx.x];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    if (threadIdx.x == 0) out[0] = mx;
+  }
+}
+
+// B[r][j0 + a] = Ut[a][r] for a 64-row slab: read Ut rows coalesced, transpose in shared memory, write each
+// row's w bytes as 4-byte words when aligned.
+__global__ void __launch_bounds__(256) write_b_kernel(const int8_t* __restrict__ Ut, int ldu, int w, int m,
+                                                      int8_t* __restrict__ B, long long k, long long j0) {
+  __shared__ int8_t tile[kMaxBlock][68];
+  const int r0 = blockIdx.x * 64;
+  for (int i = threadIdx.x; i < w * 64; i += 256) {
+    const int a = i >> 6, r = i & 63;
+    tile[a][r] = (r0 + r < m) ? Ut[(long long)a * ldu + r0 + r] : (int8_t)0;
+  }
+  __syncthreads();
+  const bool words = ((k & 3) == 0) && ((j0 & 3) == 0) && ((w & 3) == 0);
+  if (words) {
+    const int wq = w >> 2;
+    for (int i = threadIdx.x; i < 64 * wq; i += 256) {
+      const int r = i / wq, q = i % wq;
+      if (r0 + r >= m) continue;
+      const int v = (int)(uint8_t)tile[4 * q][r] | ((int)(uint8_t)tile[4 * q + 1][r] << 8) |
+                    ((int)(uint8_t)tile[4 * q + 2][r] << 16) | ((int)(uint8_t)tile[4 * q + 3][r] << 24);
+      *reinterpret_cast<int*>(B + (long long)(r0 + r) * k + j0 + 4 * q) = v;
+    }
+  } else {
+    for (int i = threadIdx.x; i < 64 * w; i += 256) {
+      const int r = i / w, a = i % w;
+      if (r0 + r < m) B[(long long)(r0 + r) * k + j0 + a] = tile[a][r];
+    }
+  }
 }
 
 template <typename T>
@@ -311,14 +356,19 @@ cudaError_t launch_select_with(const float* colpart, int nrt, int n, const float
 }
 
 cudaError_t launch_norm(const double* normpart, int count, double* out, const double* norm_a, double* trace,
-                        cudaStream_t s) {
-  norm_kernel<<<1, 32, 0, s>>>(normpart, count, out, norm_a, trace);
+                        cudaStream_t s, const float* maxpart, float* maxout) {
+  norm_kernel<<<1, 32, 0, s>>>(normpart, count, out, norm_a, trace, maxpart, maxout);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_absmax(const float* x, long long n, float* out, cudaStream_t s) {
+  absmax_kernel<<<1, 1024, 0, s>>>(x, n, out);
   return cudaGetLastError();
 }
 
 cudaError_t launch_write_b(const int8_t* Ut, int ldu, int w, int m, int8_t* B, long long k, long long j0,
                            cudaStream_t s) {
-  write_b_kernel<<<(unsigned)cdiv(m, 256), 256, 0, s>>>(Ut, ldu, w, m, B, k, j0);
+  write_b_kernel<<<(unsigned)cdiv(m, 64), 256, 0, s>>>(Ut, ldu, w, m, B, k, j0);
   return cudaGetLastError();
 }
 
