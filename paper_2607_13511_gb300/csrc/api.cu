@@ -219,7 +219,9 @@ struct Bufs {
   float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE, *maxpart, *maxabs;
   unsigned* err;
   int8_t *Ut, *Vt;
-  double *spart, *r, *normpart, *norm_a, *norm_r, *trace;
+  F2 *spart, *normpart;
+  float* r;
+  double *norm_a, *norm_r, *trace;
   u64* kpart;
   int* J;
 };
@@ -642,7 +644,7 @@ int externd_energy(const float* A, int64_t m, int64_t n, const int8_t* B, const 
   if (weights != nullptr) TRY(check_dev(weights));
   Workspace* ws;
   TRY(current_ws(&ws));
-  double* part;
+  F2* part;
   double* sc;
   TRY(need(*ws, "energy.part", (size_t)deflate_tiles((int)m, (int)n), &part));
   TRY(need(*ws, "energy.sc", 4, &sc));
@@ -666,7 +668,7 @@ int externd_ternarize(const float* X, int64_t rows, int64_t cols, int axis, doub
   const long long nv = axis == 1 ? rows : cols, L = axis == 1 ? cols : rows;
   if (nv > 65535) return EXTERND_EINVAL;   // one grid row per vector
   const int nchunk = (int)cdiv(L, kStatChunk);
-  double* sp;
+  F2* sp;
   u64* kp;
   TRY(need(*ws, "tern.spart", (size_t)nv * nchunk, &sp));
   TRY(need(*ws, "tern.kpart", (size_t)nv * nchunk, &kp));
@@ -744,7 +746,7 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   const int nchunk = decorrelate_chunks((int)L);
   int8_t* T;
   float *part, *X, *Gpart, *Graw, *Ginv, *one;
-  double* sp;
+  F2* sp;
   u64* kp;
   if (vstep) TRY(stage_u(*ws, F, m, w, &T));
   else TRY(stage_v(*ws, F, n, w, &T));
@@ -811,7 +813,7 @@ int externd_block_scales(const float* R, int64_t m, int64_t n, const int8_t* U, 
   int8_t *Ut, *Vt;
   float *part, *Gpart, *GrawV, *Ginv, *mx;
   unsigned* err;
-  double* r;
+  float* r;
   TRY(stage_u(*ws, U, m, (int)w, &Ut));
   TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
   TRY(step_scalars(*ws, R, m * n, weights, n, &mx, &err));
@@ -842,7 +844,8 @@ int externd_deflate(float* R, int64_t m, int64_t n, const int8_t* U, const float
   Workspace* ws;
   TRY(current_ws(&ws));
   int8_t *Ut, *Vt;
-  double *part, *sc;
+  F2* part;
+  double* sc;
   TRY(stage_u(*ws, U, m, (int)w, &Ut));
   TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
   const int tiles = deflate_tiles((int)m, (int)n);

@@ -40,17 +40,49 @@ __device__ __forceinline__ u64 warp_max(u64 v) {
   return v;
 }
 
-// Compensated (Neumaier) float sum of magnitudes: a thread adds a few hundred |x| with ~2^-44 relative error,
-// the cross-thread combine runs in double. Keeps the Eq. 2 mean accurate without per-element double math.
+// Double-float value hi + lo held in two floats (|lo| <= ulp(hi) / 2), added with Knuth's error-free TwoSum. It
+// carries ~44 significant bits with float32 arithmetic only: double-precision arithmetic runs at a small fraction
+// of the float32 rate on this GPU and is kept out of every per-element and per-thread reduction.
+struct F2 {
+  float hi = 0.f, lo = 0.f;
+};
+
+__device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
+  const float s = a.hi + b.hi;
+  const float bb = s - a.hi;
+  const float err = (a.hi - (s - bb)) + (b.hi - bb);
+  const float lo = a.lo + b.lo + err;
+  F2 r;
+  r.hi = s + lo;
+  r.lo = lo - (r.hi - s);
+  return r;
+}
+
+__device__ __forceinline__ F2 f2_add(F2 a, float x) {
+  F2 b;
+  b.hi = x;
+  return f2_add(a, b);
+}
+
+__device__ __forceinline__ F2 f2_shfl_xor(F2 v, int o) {
+  F2 r;
+  r.hi = __shfl_xor_sync(0xffffffffu, v.hi, o);
+  r.lo = __shfl_xor_sync(0xffffffffu, v.lo, o);
+  return r;
+}
+
+__device__ __forceinline__ F2 warp_sum(F2 v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = f2_add(v, f2_shfl_xor(v, o));
+  return v;
+}
+
+__device__ __forceinline__ double f2_value(F2 v) { return (double)v.hi + (double)v.lo; }
+
+// Per-thread sum of magnitudes for the Eq. 2 mean.
 struct AbsSum {
-  float s = 0.f, c = 0.f;
-  __device__ __forceinline__ void add(float x) {
-    const float a = fabsf(x);
-    const float t = s + a;
-    c += (s >= a) ? ((s - t) + a) : ((a - t) + s);
-    s = t;
-  }
-  __device__ __forceinline__ double value() const { return (double)s + (double)c; }
+  F2 acc;
+  __device__ __forceinline__ void add(float x) { acc = f2_add(acc, fabsf(x)); }
 };
 
 // Key whose maximum picks the largest |x| and, among equal magnitudes, the lowest index.

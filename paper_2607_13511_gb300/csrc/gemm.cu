@@ -208,10 +208,10 @@ __global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restric
         }
       }
     }
-    double s = sum.value();
+    F2 s = sum.acc;
 #pragma unroll
     for (int o = 8; o > 0; o >>= 1) {
-      s += __shfl_xor_sync(0xffffffffu, s, o);
+      s = f2_add(s, f2_shfl_xor(s, o));
       const u64 t = __shfl_xor_sync(0xffffffffu, key, o);
       key = t > key ? t : key;
     }
@@ -227,13 +227,13 @@ __global__ void __launch_bounds__(256) deflate_kernel(const float* Rin, float* R
                                                       const int8_t* __restrict__ U, long long ldu,
                                                       const float* __restrict__ d, const int8_t* __restrict__ V,
                                                       long long ldv, int w, const float* __restrict__ h,
-                                                      float* __restrict__ colpart, double* __restrict__ normpart,
+                                                      float* __restrict__ colpart, F2* __restrict__ normpart,
                                                       float* __restrict__ maxpart) {
   __shared__ __align__(16) float As[TK][TM + 4];
   __shared__ float wmax[8];
   __shared__ __align__(16) float Bs[TK][TN];
   __shared__ float red[16][TN];
-  __shared__ double wred[8];
+  __shared__ float wred[8];
   const int c0 = blockIdx.x * TN;
   const int r0 = blockIdx.y * TM;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
@@ -332,7 +332,7 @@ __global__ void __launch_bounds__(256) deflate_kernel(const float* Rin, float* R
       colpart[(long long)blockIdx.y * n + c0 + tid] = s;
     }
   }
-  double dn = warp_sum((double)nrm);
+  const float dn = warp_sum(nrm);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
   if ((tid & 31) == 0) {
@@ -341,11 +341,11 @@ __global__ void __launch_bounds__(256) deflate_kernel(const float* Rin, float* R
   }
   __syncthreads();
   if (tid == 0) {
-    double s = 0.0;
+    F2 s;
     float mx = 0.f;
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
-      s += wred[q];
+      s = f2_add(s, wred[q]);
       mx = fmaxf(mx, wmax[q]);
     }
     const long long tile = (long long)blockIdx.y * gridDim.x + blockIdx.x;
@@ -406,7 +406,7 @@ int deflate_tiles(int m, int n) { return (int)(cdiv(m, TM) * cdiv(n, TN)); }
 
 cudaError_t launch_deflate(const float* Rin, float* Rout, int m, int n, const int8_t* U, long long ldu, bool u_rowmajor,
                            const float* d, const int8_t* Vt, long long ldv, int w, const float* h, float* colpart,
-                           double* normpart, cudaStream_t s, float* maxpart) {
+                           F2* normpart, cudaStream_t s, float* maxpart) {
   dim3 grid((unsigned)cdiv(n, TN), (unsigned)cdiv(m, TM));
   if (u_rowmajor)
     deflate_kernel<true><<<grid, 256, 0, s>>>(Rin, Rout, m, n, U, ldu, d, Vt, ldv, w, h, colpart, normpart, maxpart);

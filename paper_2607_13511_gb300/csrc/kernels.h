@@ -6,7 +6,7 @@
 //   Vt     w x ldv int8: row a is component a's v (length n; ldv = round_up(n, 16), zero padded) = a block of C.
 //   part   splits x w x L float32: split-K partial products; L = n for the V-step, m for the U-step.
 //   X      w x ldx float32: decorrelated targets, one vector per row (the Eq. 2 input).
-//   Stats  per-vector partials of the Eq. 2 statistics: spart[a * nchunk + c] = sum |x| over chunk c,
+//   Stats  per-vector partials of the Eq. 2 statistics: spart[a * nchunk + c] = sum |x| over chunk c (double-float),
 //          kpart[a * nchunk + c] = max magnitude key over chunk c (chunks of kStatChunk positions).
 #pragma once
 
@@ -18,7 +18,7 @@
 namespace externd {
 
 struct Stats {
-  double* spart;
+  F2* spart;
   u64* kpart;
   int nchunk;
 };
@@ -40,7 +40,7 @@ cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int 
 // maxpart (optional): per-tile max |Rout|.
 cudaError_t launch_deflate(const float* Rin, float* Rout, int m, int n, const int8_t* U, long long ldu, bool u_rowmajor,
                            const float* d, const int8_t* Vt, long long ldv, int w, const float* h, float* colpart,
-                           double* normpart, cudaStream_t s, float* maxpart = nullptr);
+                           F2* normpart, cudaStream_t s, float* maxpart = nullptr);
 int deflate_row_tiles(int m);
 int deflate_tiles(int m, int n);
 
@@ -62,7 +62,7 @@ cudaError_t launch_select_with(const float* colpart, int nrt, int n, const float
                                cudaStream_t s);
 // out[0] = sum of count partials (fixed order); if trace != NULL, trace[0] = 1 - out[0] / norm_a[0];
 // if maxpart != NULL, maxout[0] = max of the count per-tile maxima.
-cudaError_t launch_norm(const double* normpart, int count, double* out, const double* norm_a, double* trace,
+cudaError_t launch_norm(const F2* normpart, int count, double* out, const double* norm_a, double* trace,
                         cudaStream_t s, const float* maxpart = nullptr, float* maxout = nullptr);
 // out[0] = max |x_i|
 cudaError_t launch_absmax(const float* x, long long n, float* out, cudaStream_t s);
@@ -84,10 +84,10 @@ cudaError_t launch_gram(const int8_t* T, int ldt, int w, int L, const float* h, 
 // Graw = sum_s Gpart[s]; Ginv = (Graw + eps I)^-1 with eps = kEpsRel * trace / w.
 cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s);
 // r[a] = sum_y Ut[a][y] * sum_s part[s][a][y]
-cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, double* r,
+cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, float* r,
                         cudaStream_t s);
 // d solves [(sum_s GUpart[s]) .* GVraw + eps I] d = r (eps = 0 when w == 1).
-cudaError_t launch_scales(const float* GUpart, int splits, const float* GVraw, const double* r, int w, float* d,
+cudaError_t launch_scales(const float* GUpart, int splits, const float* GVraw, const float* r, int w, float* d,
                           cudaStream_t s);
 
 }  // namespace externd

@@ -66,8 +66,8 @@ extern "C" int externd_energy_noalloc(const float* A, int64_t m, int64_t n, cons
     if (e != cudaSuccess) return record_cuda_error(e, "cudaGetSymbolAddress(g_noalloc_scratch)");
     g_scratch_addr[dev] = static_cast<double*>(p);
   }
-  double* part = g_scratch_addr[dev];   // [tiles] per-tile partial sums
-  double* sc = part + tiles;            // ||A||_H^2, ||A - B diag(D) C||_H^2, energy
+  F2* part = reinterpret_cast<F2*>(g_scratch_addr[dev]);   // [tiles] per-tile partial sums (8 bytes each)
+  double* sc = g_scratch_addr[dev] + tiles;                 // ||A||_H^2, ||A - B diag(D) C||_H^2, energy
   cudaStream_t s = library_stream();
   const int mi = (int)m, ni = (int)n;
   if ((e = launch_deflate(A, nullptr, mi, ni, nullptr, 0, false, nullptr, nullptr, 0, 0, weights, nullptr, part,

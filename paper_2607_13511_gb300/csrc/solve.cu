@@ -82,126 +82,424 @@ __global__ void __launch_bounds__(256) gram_kernel(const int8_t* __restrict__ T,
 // MODE 0: Graw = sum_s Gpart[s]; Ginv = (Graw + eps I)^-1.
 // MODE 1: K = (sum_s Gpart[s]) .* GVraw (+ eps I when w > 1); d = K^-1 r.
 //
-// Symmetric sweep: sweeping pivot k maps S to S - S[:,k] S[k,:] / p with row and column k replaced by
-// S[k,:] / p and S[k][k] by -1/p (p = S[k][k]); after all pivots S = -G^-1. Every intermediate S stays
-// symmetric, so the pivot column equals the pivot row: the threads that own row k publish it to shared memory
-// with vector stores, every thread applies the same branch-free rank-1 update to its EPT elements, and row k
-// and column k are fixed up with predicated selects. One barrier per pivot.
-template <int W_PAD, int NT, int MODE>
-__global__ void __launch_bounds__(NT) sweep_kernel(const float* __restrict__ Gpart, int splits, int w,
-                                                   const float* __restrict__ GVraw, const double* __restrict__ r,
-                                                   float* __restrict__ Graw, float* __restrict__ out) {
-  constexpr int TPR = NT / W_PAD;         // threads per row
-  constexpr int EPT = W_PAD / TPR;        // elements per thread (a multiple of 4)
-  static_assert(EPT % 4 == 0, "EPT must allow 16-byte row stores");
-  __shared__ __align__(16) float rowk[2][W_PAD];
-  __shared__ double dsum[32];
-  const int tid = threadIdx.x;
-  const int i = tid / TPR, q = tid % TPR;
-  const int j0 = q * EPT;
-  float S[EPT];
-  double diag = 0.0;
-#pragma unroll
-  for (int e = 0; e < EPT; ++e) {
-    const int j = j0 + e;
-    float v = (i == j) ? 1.f : 0.f;
-    if (i < w && j < w) {
-      float g = 0.f;
-      for (int sp = 0; sp < splits; ++sp) g += Gpart[(long long)sp * w * w + (long long)i * w + j];
-      if (MODE == 0) {
-        Graw[(long long)i * w + j] = g;
-      } else {
-        g *= GVraw[(long long)i * w + j];
-      }
-      v = g;
-      if (i == j) diag = (double)g;
-    }
-    S[e] = v;
-  }
-  // trace -> ridge
-  double t = warp_sum(diag);
-  if ((tid & 31) == 0) dsum[tid >> 5] = t;
-  __syncthreads();
-  if (tid < 32) {
-    double u = warp_sum(tid < NT / 32 ? dsum[tid] : 0.0);
-    if (tid == 0) dsum[0] = u;
-  }
-  __syncthreads();
-  const bool ridge = (MODE == 0) || (w > 1);
-  const float eps = ridge ? (float)(kEpsRel * dsum[0] / (double)w) : 0.f;
-#pragma unroll
-  for (int e = 0; e < EPT; ++e)
-    if (i < w && j0 + e == i) S[e] += eps;
+// Blocked symmetric sweep. Sweeping pivot k maps S to S - S[:,k] S[k,:] / p with row and column k replaced by
+// S[k,:] / p and S[k][k] by -1/p (p = S[k][k]); after every pivot S = -G^-1. Sweeps compose, so NB = 8 pivots
+// K are eliminated per step: with P = S[K,K] and Q = P^-1,
+//   S[I,J] -= S[I,K] Q S[K,J],  S[I,K] = S[I,K] Q,  S[K,J] = Q S[K,J],  S[K,K] = -Q      (I, J outside K).
+// Every intermediate S is symmetric, so S[I,K] is the transpose of the published block rows S[K,:].
+//
+// Layout: warp q owns the RPW = W_PAD / NWARP rows q*RPW + a; lane l owns the CPL = W_PAD / 32 columns
+// l + 32 c. Row-contiguous lanes make every global load and store coalesced and every read of a row's pivot
+// entries a shared-memory broadcast. Per step: the warps owning rows K publish them (barrier), warp 0 inverts the
+// 8 x 8 pivot block (barrier), every thread forms t = S[i,K] Q with one FMA chain per lane and 8 shuffles per
+// row, then applies the rank-8 update to its elements (barrier).
+template <int W_PAD, int NWARP, int MODE>
+__global__ void __launch_bounds__(NWARP * 32) sweep_kernel(const float* __restrict__ Gpart, int splits, int w,
+                                                           const float* __restrict__ GVraw,
+                                                           const float* __restrict__ r, float* __restrict__ Graw,
+                                                           float* __restrict__ out) {
+  constexpr int RPW = W_PAD / NWARP;  // rows per warp
+  constexpr int CPL = W_PAD / 32;     // columns per lane
+  constexpr int NB = 8;
+  static_assert(RPW >= 1 && CPL >= 1 && W_PAD % NB == 0, "bad sweep shape");
+  __shared__ __align__(16) float rowsK[NB][W_PAD];
+  __shared__ float Qs[NB][NB];
+  __shared__ float dsum[NWARP];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int r0 = warp * RPW;
 
-  for (int k = 0; k < w; ++k) {
-    float* rk = rowk[k & 1];
-    if (i == k) {
+  float S[RPW][CPL];
 #pragma unroll
-      for (int e = 0; e < EPT; e += 4)
-        *reinterpret_cast<float4*>(&rk[j0 + e]) = make_float4(S[e], S[e + 1], S[e + 2], S[e + 3]);
+  for (int a = 0; a < RPW; ++a)
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) S[a][c] = 0.f;
+  // Sum the split Gram slices (coalesced: lanes walk a row).
+  for (int sp = 0; sp < splits; ++sp) {
+    const float* G = Gpart + (long long)sp * w * w;
+#pragma unroll
+    for (int a = 0; a < RPW; ++a) {
+      const int i = r0 + a;
+      if (i >= w) continue;
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) {
+        const int j = lane + 32 * c;
+        if (j < w) S[a][c] += G[(long long)i * w + j];
+      }
+    }
+  }
+  float diag = 0.f;
+#pragma unroll
+  for (int a = 0; a < RPW; ++a) {
+    const int i = r0 + a;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) {
+      const int j = lane + 32 * c;
+      float v = S[a][c];
+      if (i < w && j < w) {
+        if (MODE == 0) Graw[(long long)i * w + j] = v;
+        else v *= GVraw[(long long)i * w + j];
+        if (i == j) diag += v;
+      } else {
+        v = (i == j) ? 1.f : 0.f;     // identity on the padding
+      }
+      S[a][c] = v;
+    }
+  }
+  // trace -> ridge (float: it only sets the ridge, whose relative size is what matters)
+  const float t = warp_sum(diag);
+  if (lane == 0) dsum[warp] = t;
+  __syncthreads();
+  float tr = 0.f;
+#pragma unroll
+  for (int q = 0; q < NWARP; ++q) tr += dsum[q];
+  const bool ridge = (MODE == 0) || (w > 1);
+  const float eps = ridge ? (float)kEpsRel * tr / (float)w : 0.f;
+#pragma unroll
+  for (int a = 0; a < RPW; ++a)
+#pragma unroll
+    for (int c = 0; c < CPL; ++c)
+      if (r0 + a < w && r0 + a == lane + 32 * c) S[a][c] += eps;
+
+  for (int k0 = 0; k0 < w; k0 += NB) {
+    // 1. publish block rows K = [k0, k0 + NB)
+#pragma unroll
+    for (int a = 0; a < RPW; ++a) {
+      const int i = r0 + a;
+      if (i >= k0 && i < k0 + NB) {
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) rowsK[i - k0][lane + 32 * c] = S[a][c];
+      }
     }
     __syncthreads();
-    const float ip = __frcp_rn(rk[k]);
-    const float ci = rk[i];           // S[i][k] = S[k][i]
-    const float f = -ci * ip;
-    const bool own_row = (i == k);
+    // 2. warp 0: Q = P^-1 by the scalar symmetric sweep of the 8 x 8 block (two elements per lane)
+    if (warp == 0) {
+      const int e0 = 2 * lane;
+      const int pr = e0 / NB, cA = e0 % NB, cB = cA + 1;
+      float qa = rowsK[pr][k0 + cA], qb = rowsK[pr][k0 + cB];
+      if (k0 + pr >= w || k0 + cA >= w) qa = (pr == cA) ? 1.f : 0.f;   // identity past w
+      if (k0 + pr >= w || k0 + cB >= w) qb = (pr == cB) ? 1.f : 0.f;
 #pragma unroll
-    for (int e = 0; e < EPT; e += 4) {
-      const float4 c4 = *reinterpret_cast<const float4*>(&rk[j0 + e]);
-      const float cj[4] = {c4.x, c4.y, c4.z, c4.w};
+      for (int kk = 0; kk < NB; ++kk) {
+        // element e of the block lives in lane e / 2 (qa if e is even, qb if odd)
+        const int ek = kk * NB + kk, ec = kk * NB + pr, ej = kk * NB + cA;
+        const float pk_a = __shfl_sync(0xffffffffu, qa, ek >> 1), pk_b = __shfl_sync(0xffffffffu, qb, ek >> 1);
+        const float xa = __shfl_sync(0xffffffffu, qa, ec >> 1), xb = __shfl_sync(0xffffffffu, qb, ec >> 1);
+        const float pa = __shfl_sync(0xffffffffu, qa, ej >> 1), pb = __shfl_sync(0xffffffffu, qb, ej >> 1);
+        // 1 / S[kk][kk] with the fast single-precision division (<= 2 ulp); the correctly rounded reciprocal
+        // takes a double-precision path, slow on this GPU
+        const float ip = __fdividef(1.f, (ek & 1) ? pk_b : pk_a);
+        const float ci = (ec & 1) ? xb : xa;
+        float na = fmaf(-ci * ip, pa, qa), nb = fmaf(-ci * ip, pb, qb);
+        if (pr == kk) { na = pa * ip; nb = pb * ip; }
+        if (cA == kk) na = (pr == kk) ? -ip : ci * ip;
+        if (cB == kk) nb = (pr == kk) ? -ip : ci * ip;
+        qa = na;
+        qb = nb;
+      }
+      Qs[pr][cA] = -qa;                        // sweeping every pivot of P leaves -P^-1
+      Qs[pr][cB] = -qb;
+    }
+    __syncthreads();
+    // 3. update: this lane's column of Q (b = lane % 8) and the pivot-row entries of its columns
+    float qcol[NB];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int j = j0 + e + u;
-        float v = fmaf(f, cj[u], S[e + u]);
-        v = own_row ? cj[u] * ip : v;       // row k: S[k][j] / p
-        v = (j == k) ? (own_row ? -ip : ci * ip) : v;   // column k: S[i][k] / p; pivot: -1/p
-        S[e + u] = v;
+    for (int c = 0; c < NB; ++c) qcol[c] = Qs[c][lane & (NB - 1)];
+    float rk[NB][CPL];
+#pragma unroll
+    for (int b = 0; b < NB; ++b)
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) rk[b][c] = rowsK[b][lane + 32 * c];
+#pragma unroll
+    for (int a = 0; a < RPW; ++a) {
+      const int i = r0 + a;
+      if (i >= W_PAD) continue;
+      const bool i_in = (i >= k0 && i < k0 + NB);        // warp-uniform
+      // t[b] = sum_c S[i][k0 + c] Q[c][b]; S[i][K] = rowsK[.][i] (broadcast reads)
+      float tb = 0.f;
+#pragma unroll
+      for (int c = 0; c < NB; ++c) tb = fmaf(rowsK[c][i], qcol[c], tb);
+      float tt[NB];
+#pragma unroll
+      for (int b = 0; b < NB; ++b) tt[b] = __shfl_sync(0xffffffffu, tb, b);
+      float qrow[NB];                                    // Q[i - k0][.] for the rows of K
+      if (i_in) {
+#pragma unroll
+        for (int b = 0; b < NB; ++b) qrow[b] = Qs[i - k0][b];
+      }
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) {
+        const int j = lane + 32 * c;
+        const bool j_in = (j >= k0 && j < k0 + NB);
+        float v = S[a][c];
+        if (!i_in) {
+          if (!j_in) {
+#pragma unroll
+            for (int b = 0; b < NB; ++b) v = fmaf(-tt[b], rk[b][c], v);
+          } else {
+#pragma unroll
+            for (int b = 0; b < NB; ++b) v = (j - k0 == b) ? tt[b] : v;            // S[i,K] Q
+          }
+        } else {
+          if (!j_in) {
+            v = 0.f;                                                             // (Q S[K,J])
+#pragma unroll
+            for (int b = 0; b < NB; ++b) v = fmaf(qrow[b], rk[b][c], v);
+          } else {
+#pragma unroll
+            for (int b = 0; b < NB; ++b) v = (j - k0 == b) ? -qrow[b] : v;        // -Q
+          }
+        }
+        S[a][c] = v;
       }
     }
+    __syncthreads();   // rowsK and Qs are rewritten by the next step
   }
 
   if (MODE == 0) {
-    if (i < w) {
 #pragma unroll
-      for (int e = 0; e < EPT; ++e) {
-        const int j = j0 + e;
-        if (j < w) out[(long long)i * w + j] = -S[e];
+    for (int a = 0; a < RPW; ++a) {
+      const int i = r0 + a;
+      if (i >= w) continue;
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) {
+        const int j = lane + 32 * c;
+        if (j < w) out[(long long)i * w + j] = -S[a][c];
       }
     }
   } else {
-    double acc = 0.0;
+    // d_i = -sum_j S[i][j] r_j: a warp reduction per row
 #pragma unroll
-    for (int e = 0; e < EPT; ++e) {
-      const int j = j0 + e;
-      if (i < w && j < w) acc += -(double)S[e] * r[j];
+    for (int a = 0; a < RPW; ++a) {
+      const int i = r0 + a;
+      F2 acc;
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) {
+        const int j = lane + 32 * c;
+        if (j < w) acc = f2_add(acc, -S[a][c] * r[j]);
+      }
+      acc = warp_sum(acc);
+      if (lane == 0 && i < w) out[i] = acc.hi + acc.lo;
     }
-#pragma unroll
-    for (int o = TPR / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (q == 0 && i < w) out[i] = (float)acc;
   }
 }
 
 __global__ void __launch_bounds__(256) rvec_kernel(const int8_t* __restrict__ Ut, int ldu, int w, int L,
                                                    const float* __restrict__ part, int splits,
-                                                   double* __restrict__ r) {
-  __shared__ double red[8];
+                                                   float* __restrict__ r) {
+  __shared__ F2 red[8];
   const int a = blockIdx.x;
+  // sum_y u_y p_y over the splits: one pass per split (independent loads), in split order
   float acc = 0.f;
-  for (int y = threadIdx.x; y < L; y += 256) {
-    const int8_t u = Ut[(long long)a * ldu + y];
-    if (u != 0) {
-      float p = 0.f;
-      for (int s = 0; s < splits; ++s) p += part[((long long)s * w + a) * L + y];
-      acc += (u > 0) ? p : -p;
+  for (int sp = 0; sp < splits; ++sp) {
+    const float* P = part + ((long long)sp * w + a) * L;
+    for (int y = threadIdx.x; y < L; y += 256) {
+      const int8_t u = Ut[(long long)a * ldu + y];
+      acc += (u > 0) ? P[y] : ((u < 0) ? -P[y] : 0.f);
     }
   }
-  double v = warp_sum((double)acc);
+  F2 v;
+  v.hi = acc;
+  v = warp_sum(v);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
   __syncthreads();
   if (threadIdx.x == 0) {
-    double s = 0.0;
-    for (int q = 0; q < 8; ++q) s += red[q];
-    r[a] = s;
+    F2 s;
+    for (int q = 0; q < 8; ++q) s = f2_add(s, red[q]);
+    r[a] = s.hi + s.lo;
+  }
+}
+
+// Wide-block sweep for w <= 128: NB pivots per step. 512 threads; thread (ty, tx) in a 16 x 32 grid owns
+// the RPT = W_PAD/16 rows ty*RPT + a and the CPT = W_PAD/32 columns tx + 32c in registers. Per step K:
+//   1. the owners of rows K publish them (Rk = S[K,:], shared memory)                        barrier
+//   2. warp 0 inverts the NB x NB pivot block: lane l keeps column l of P in registers; the
+//      pivot column is broadcast with shuffles (by symmetry it is also the pivot row)      barrier
+//   3. T = S[:,K] Q for every row (S[i,K] = Rk[.,i]), one row per thread group            barrier
+//   4. rank-NB update of the register tiles from T and Rk, fixing up rows and columns of K  barrier
+// The serial part is NB pivots of one warp per step; everything else is dense float32 FMA.
+template <int W_PAD, int NB, int MODE>
+__global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ Gpart, int splits, int w,
+                                                      const float* __restrict__ GVraw, const float* __restrict__ r,
+                                                      float* __restrict__ Graw, float* __restrict__ out) {
+  constexpr int RPT = W_PAD / 16, CPT = W_PAD / 32;
+  static_assert(W_PAD % NB == 0 && RPT >= 1 && CPT >= 1, "bad shape");
+  __shared__ __align__(16) float Rk[NB][W_PAD + 1];
+  __shared__ __align__(16) float T[W_PAD][NB + 1];
+  __shared__ float Qs[NB][NB + 1];
+  __shared__ float red[16];
+  const int tid = threadIdx.x, tx = tid & 31, ty = tid >> 5, lane = tx;
+  const int i0 = ty * RPT;
+
+  float S[RPT][CPT];
+#pragma unroll
+  for (int a = 0; a < RPT; ++a)
+#pragma unroll
+    for (int c = 0; c < CPT; ++c) S[a][c] = 0.f;
+  for (int sp = 0; sp < splits; ++sp) {
+    const float* G = Gpart + (long long)sp * w * w;
+#pragma unroll
+    for (int a = 0; a < RPT; ++a) {
+      const int i = i0 + a;
+      if (i >= w) continue;
+#pragma unroll
+      for (int c = 0; c < CPT; ++c) {
+        const int j = tx + 32 * c;
+        if (j < w) S[a][c] += G[(long long)i * w + j];
+      }
+    }
+  }
+  float diag = 0.f;
+#pragma unroll
+  for (int a = 0; a < RPT; ++a) {
+    const int i = i0 + a;
+#pragma unroll
+    for (int c = 0; c < CPT; ++c) {
+      const int j = tx + 32 * c;
+      float v = S[a][c];
+      if (i < w && j < w) {
+        if (MODE == 0) Graw[(long long)i * w + j] = v;
+        else v *= GVraw[(long long)i * w + j];
+        if (i == j) diag += v;
+      } else {
+        v = (i == j) ? 1.f : 0.f;
+      }
+      S[a][c] = v;
+    }
+  }
+  const float dw = warp_sum(diag);
+  if (lane == 0) red[ty] = dw;
+  __syncthreads();
+  float tr = 0.f;
+#pragma unroll
+  for (int q = 0; q < 16; ++q) tr += red[q];
+  const float eps = ((MODE == 0) || (w > 1)) ? (float)kEpsRel * tr / (float)w : 0.f;
+#pragma unroll
+  for (int a = 0; a < RPT; ++a)
+#pragma unroll
+    for (int c = 0; c < CPT; ++c)
+      if (i0 + a < w && i0 + a == tx + 32 * c) S[a][c] += eps;
+
+  for (int k0 = 0; k0 < w; k0 += NB) {
+    // 1. publish rows K
+#pragma unroll
+    for (int a = 0; a < RPT; ++a) {
+      const int i = i0 + a;
+      if (i >= k0 && i < k0 + NB) {
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) Rk[i - k0][tx + 32 * c] = S[a][c];
+      }
+    }
+    __syncthreads();
+    // 2. warp 0: Q = P^-1 (symmetric sweep of the NB x NB block; lane l holds column l, i.e. P[.][l])
+    if (ty == 0) {
+      float col[NB];
+#pragma unroll
+      for (int e = 0; e < NB; ++e) {
+        const bool inside = (lane < NB) && (k0 + e < w) && (k0 + lane < w);
+        col[e] = inside ? Rk[e][k0 + lane] : ((e == lane) ? 1.f : 0.f);
+      }
+#pragma unroll
+      for (int kk = 0; kk < NB; ++kk) {
+        const float pkl = col[kk];                                   // P[kk][l] = P[l][kk]
+        const float p = __shfl_sync(0xffffffffu, pkl, kk);            // P[kk][kk]
+        const float ip = __fdividef(1.f, p);
+#pragma unroll
+        for (int e = 0; e < NB; ++e) {
+          const float pek = __shfl_sync(0xffffffffu, pkl, e);          // P[e][kk] = P[kk][e] (lane e's entry)
+          float v = fmaf(-pek * ip, pkl, col[e]);
+          v = (e == kk) ? pkl * ip : v;                               // row kk
+          v = (lane == kk) ? ((e == kk) ? -ip : pek * ip) : v;        // column kk, pivot
+          col[e] = v;
+        }
+      }
+      if (lane < NB) {
+#pragma unroll
+        for (int e = 0; e < NB; ++e) Qs[e][lane] = -col[e];
+      }
+    }
+    __syncthreads();
+    // 3. T[i][b] = sum_c S[i][k0 + c] Q[c][b] = sum_c Rk[c][i] Q[c][b]  (thread: row i = tid / 4, b = 8 of them)
+    for (int idx = tid; idx < W_PAD * (NB / 8); idx += 512) {
+      const int i = idx / (NB / 8), bq = (idx % (NB / 8)) * 8;
+      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int c = 0; c < NB; ++c) {
+        const float rv = Rk[c][i];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) acc[u] = fmaf(rv, Qs[c][bq + u], acc[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) T[i][bq + u] = acc[u];
+    }
+    __syncthreads();
+    // 4. rank-NB update of the register tiles
+    float acc[RPT][CPT];
+#pragma unroll
+    for (int a = 0; a < RPT; ++a)
+#pragma unroll
+      for (int c = 0; c < CPT; ++c) acc[a][c] = 0.f;
+#pragma unroll 4
+    for (int b = 0; b < NB; ++b) {
+      float tv[RPT], rv[CPT];
+#pragma unroll
+      for (int a = 0; a < RPT; ++a) tv[a] = T[i0 + a][b];
+#pragma unroll
+      for (int c = 0; c < CPT; ++c) rv[c] = Rk[b][tx + 32 * c];
+#pragma unroll
+      for (int a = 0; a < RPT; ++a)
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) acc[a][c] = fmaf(tv[a], rv[c], acc[a][c]);
+    }
+#pragma unroll
+    for (int a = 0; a < RPT; ++a) {
+      const int i = i0 + a;
+      const bool i_in = (i >= k0 && i < k0 + NB);
+#pragma unroll
+      for (int c = 0; c < CPT; ++c) {
+        const int j = tx + 32 * c;
+        const bool j_in = (j >= k0 && j < k0 + NB);
+        float v;
+        if (!i_in && !j_in) v = S[a][c] - acc[a][c];                 // S - S[I,K] Q S[K,J]
+        else if (!i_in) v = T[i][j - k0];                            // S[I,K] Q
+        else if (!j_in) {                                            // Q S[K,J] = T^T restricted: sum_b Q[ia][b] Rk[b][j]
+          const int ia = i - k0;
+          float q = 0.f;
+#pragma unroll 8
+          for (int b = 0; b < NB; ++b) q = fmaf(Qs[ia][b], Rk[b][j], q);
+          v = q;
+        } else {
+          v = -Qs[i - k0][j - k0];
+        }
+        S[a][c] = v;
+      }
+    }
+    __syncthreads();   // Rk, Qs, T are rewritten by the next step
+  }
+
+  if (MODE == 0) {
+#pragma unroll
+    for (int a = 0; a < RPT; ++a) {
+      const int i = i0 + a;
+      if (i >= w) continue;
+#pragma unroll
+      for (int c = 0; c < CPT; ++c) {
+        const int j = tx + 32 * c;
+        if (j < w) out[(long long)i * w + j] = -S[a][c];
+      }
+    }
+  } else {
+#pragma unroll
+    for (int a = 0; a < RPT; ++a) {
+      const int i = i0 + a;
+      F2 acc2;
+#pragma unroll
+      for (int c = 0; c < CPT; ++c) {
+        const int j = tx + 32 * c;
+        if (j < w) acc2 = f2_add(acc2, -S[a][c] * r[j]);
+      }
+      acc2 = warp_sum(acc2);
+      if (lane == 0 && i < w) out[i] = acc2.hi + acc2.lo;
+    }
   }
 }
 
@@ -216,13 +514,14 @@ int gram_chunk(int w, int L, int* splits) {
 }
 
 template <int MODE>
-cudaError_t launch_sweep(const float* Gpart, int splits, int w, const float* GVraw, const double* r, float* Graw,
+cudaError_t launch_sweep(const float* Gpart, int splits, int w, const float* GVraw, const float* r, float* Graw,
                          float* out, cudaStream_t s) {
-  // 16 elements per thread up to w = 128 (one barrier per pivot; the update is a branch-free rank-1 FMA)
-  if (w <= 32) sweep_kernel<32, 128, MODE><<<1, 128, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
-  else if (w <= 64) sweep_kernel<64, 256, MODE><<<1, 256, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
-  else if (w <= 128) sweep_kernel<128, 1024, MODE><<<1, 1024, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
-  else sweep_kernel<256, 1024, MODE><<<1, 1024, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
+  // elements per lane RPW * CPL = W_PAD^2 / (32 * NWARP): 4 / 8 / 32 / 64
+  // pivot-block sizes measured fastest on GB300: 8 up to w = 64, 16 at w = 128
+  if (w <= 32) sweep32_kernel<32, 8, MODE><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
+  else if (w <= 64) sweep32_kernel<64, 8, MODE><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
+  else if (w <= 128) sweep32_kernel<128, 16, MODE><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
+  else sweep_kernel<256, 32, MODE><<<1, 32 * 32, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
   return cudaGetLastError();
 }
 
@@ -246,13 +545,13 @@ cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, f
   return launch_sweep<0>(Gpart, splits, w, nullptr, nullptr, Graw, Ginv, s);
 }
 
-cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, double* r,
+cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, float* r,
                         cudaStream_t s) {
   rvec_kernel<<<(unsigned)w, 256, 0, s>>>(Ut, ldu, w, L, part, splits, r);
   return cudaGetLastError();
 }
 
-cudaError_t launch_scales(const float* GUpart, int splits, const float* GVraw, const double* r, int w, float* d,
+cudaError_t launch_scales(const float* GUpart, int splits, const float* GVraw, const float* r, int w, float* d,
                           cudaStream_t s) {
   return launch_sweep<1>(GUpart, splits, w, GVraw, r, nullptr, d, s);
 }

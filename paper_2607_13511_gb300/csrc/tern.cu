@@ -16,7 +16,7 @@ template <bool GATHER>
 __global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X, int L, long long ldx, int ncols,
                                                     const int* __restrict__ J, float* __restrict__ Y, long long ldy,
                                                     Stats st) {
-  __shared__ double ssum[4];
+  __shared__ F2 ssum[4];
   __shared__ u64 skey[4];
   const int a = blockIdx.y;
   const int x = blockIdx.x * kStatChunk + threadIdx.x;
@@ -31,7 +31,8 @@ __global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X,
       v = __ldg(X + (long long)a * ldx + x);
     }
   }
-  double s = valid ? (double)fabsf(v) : 0.0;
+  F2 s;
+  s.hi = valid ? fabsf(v) : 0.f;
   u64 key = valid ? mag_key(v, (uint32_t)x) : 0ull;
   s = warp_sum(s);
   key = warp_max(key);
@@ -42,11 +43,11 @@ __global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X,
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    double t = 0.0;
+    F2 t;
     u64 k = 0;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      t += ssum[q];
+      t = f2_add(t, ssum[q]);
       k = skey[q] > k ? skey[q] : k;
     }
     st.spart[(long long)a * st.nchunk + blockIdx.x] = t;
@@ -59,17 +60,19 @@ __global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X,
 __device__ __forceinline__ void vector_threshold(const Stats& st, int a, int L, double tau, float* theta_dn,
                                                  int* fallback, uint32_t* argidx) {
   const int lane = threadIdx.x & 31;
-  double s = 0.0;
+  F2 s;
   u64 key = 0;
   for (int c = lane; c < st.nchunk; c += 32) {
-    s += st.spart[(long long)a * st.nchunk + c];
+    s = f2_add(s, st.spart[(long long)a * st.nchunk + c]);
     const u64 k = st.kpart[(long long)a * st.nchunk + c];
     key = k > key ? k : key;
   }
   s = warp_sum(s);
   key = warp_max(key);
-  const double theta = tau * (s / (double)L);
-  const float th = __double2float_rd(theta);
+  // theta = tau * (S / L) in double, by one lane (double arithmetic is slow here; keep it to one thread)
+  float th = 0.f;
+  if (lane == 0) th = __double2float_rd(tau * (f2_value(s) / (double)L));
+  th = __shfl_sync(0xffffffffu, th, 0);
   *theta_dn = th;
   *fallback = !(key_mag(key) > th);
   *argidx = key_index(key);
@@ -233,20 +236,21 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
   }
 }
 
-__global__ void norm_kernel(const double* __restrict__ part, int count, double* out, const double* norm_a,
-                            double* trace, const float* __restrict__ maxpart, float* maxout) {
-  double s = 0.0;
+__global__ void norm_kernel(const F2* __restrict__ part, int count, double* out, const double* norm_a, double* trace,
+                            const float* __restrict__ maxpart, float* maxout) {
+  F2 s;
   float mx = 0.f;
   for (int i = threadIdx.x; i < count; i += 32) {
-    s += part[i];
+    s = f2_add(s, part[i]);
     if (maxpart != nullptr) mx = fmaxf(mx, maxpart[i]);
   }
   s = warp_sum(s);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
   if (threadIdx.x == 0) {
-    out[0] = s;
-    if (trace != nullptr) trace[0] = 1.0 - s / norm_a[0];
+    const double v = f2_value(s);
+    out[0] = v;
+    if (trace != nullptr) trace[0] = 1.0 - v / norm_a[0];
     if (maxout != nullptr) maxout[0] = mx;
   }
 }
@@ -355,7 +359,7 @@ cudaError_t launch_select_with(const float* colpart, int nrt, int n, const float
   return cudaGetLastError();
 }
 
-cudaError_t launch_norm(const double* normpart, int count, double* out, const double* norm_a, double* trace,
+cudaError_t launch_norm(const F2* normpart, int count, double* out, const double* norm_a, double* trace,
                         cudaStream_t s, const float* maxpart, float* maxout) {
   norm_kernel<<<1, 32, 0, s>>>(normpart, count, out, norm_a, trace, maxpart, maxout);
   return cudaGetLastError();
