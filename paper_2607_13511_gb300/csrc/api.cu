@@ -189,14 +189,16 @@ bool use_tc(int w) {
 int splits_v(int w, int m, int n) { return use_tc(w) ? tc_product_splits(w, n, m) : product_splits(w, n, m); }
 int splits_u(int w, int m, int n) { return use_tc(w) ? tc_product_splits(w, m, n) : product_splits(w, m, n); }
 
-cudaError_t product_v(const float* R, int m, int n, const int8_t* Ut, int ldu, int w, float* part, int splits,
-                      const float* maxabs, unsigned* err, cudaStream_t s) {
-  if (use_tc(w)) return launch_product_v_tc(R, m, n, Ut, ldu, w, part, splits, maxabs, err, s);
+// The factor comes as int8 rows (FMA tiles) and as the same values in fp16 rows (tensor cores), both with
+// leading dimension ld elements.
+cudaError_t product_v(const float* R, int m, int n, const int8_t* Ut, const __half* Ut16, int ldu, int w, float* part,
+                      int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
+  if (use_tc(w)) return launch_product_v_tc(R, m, n, Ut16, ldu, w, part, splits, maxabs, err, s);
   return launch_product_v(R, m, n, Ut, ldu, w, part, splits, s);
 }
-cudaError_t product_u(const float* R, int m, int n, const int8_t* Vt, int ldv, int w, const float* h, float* part,
-                      int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
-  if (use_tc(w)) return launch_product_u_tc(R, m, n, Vt, ldv, w, h, part, splits, maxabs, err, s);
+cudaError_t product_u(const float* R, int m, int n, const int8_t* Vt, const __half* Vt16, int ldv, int w,
+                      const float* h, float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
+  if (use_tc(w)) return launch_product_u_tc(R, m, n, Vt16, ldv, w, h, part, splits, maxabs, err, s);
   return launch_product_u(R, m, n, Vt, ldv, w, h, part, splits, s);
 }
 
@@ -216,9 +218,11 @@ struct Plan {
 };
 
 struct Bufs {
-  float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE, *maxpart, *maxabs;
-  unsigned* err;
+  float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE, *maxpart, *maxabs, *theta;
+  unsigned *err, *arg, *ticket;
+  int *fallback, *GintU, *GintV;
   int8_t *Ut, *Vt;
+  __half *Ut16, *Vt16;   // fp16 copies of Ut, Vt for the tensor-core products (nullptr when unused)
   F2 *spart, *normpart;
   float* r;
   double *norm_a, *norm_r, *trace;
@@ -232,6 +236,11 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "R", (size_t)p.m * p.n, &B->R));
   TRY(need(ws, "Ut", (size_t)w * p.ldm, &B->Ut, true));
   TRY(need(ws, "Vt", (size_t)w * p.ldn, &B->Vt, true));
+  B->Ut16 = B->Vt16 = nullptr;
+  if (use_tc(p.b)) {
+    TRY(need(ws, "Ut16", (size_t)w * p.ldm, &B->Ut16, true));
+    TRY(need(ws, "Vt16", (size_t)w * p.ldn, &B->Vt16, true));
+  }
   // split-K partials for both block widths that occur (b and the tail k mod b)
   size_t part = 0;
   for (long long wi : {(long long)p.b, p.k % p.b}) {
@@ -243,6 +252,12 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "maxpart", (size_t)deflate_tiles(p.m, p.n), &B->maxpart));
   TRY(need(ws, "maxabs", 2, &B->maxabs));
   TRY(need(ws, "err", 1, &B->err, true));
+  TRY(need(ws, "theta", (size_t)w, &B->theta));
+  TRY(need(ws, "fallback", (size_t)w, &B->fallback));
+  TRY(need(ws, "arg", (size_t)w, &B->arg));
+  TRY(need(ws, "ticket", 1, &B->ticket, true));
+  TRY(need(ws, "GintU", (size_t)w * w, &B->GintU, true));
+  TRY(need(ws, "GintV", (size_t)w * w, &B->GintV, true));
   TRY(need(ws, "X", (size_t)w * L, &B->X));
   TRY(need(ws, "spart", (size_t)w * std::max(p.nchunk_m, p.nchunk_n), &B->spart));
   TRY(need(ws, "kpart", (size_t)w * std::max(p.nchunk_m, p.nchunk_n), &B->kpart));
@@ -317,10 +332,13 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
                       float* Dout, int8_t* Cout, cudaStream_t s) {
   cudaStream_t side = ws.side;
   const int m = p.m, n = p.n;
-  // each producer of Eq. 2 statistics and its apply agree on the chunk count
-  const Stats st_g{B.spart, B.kpart, (int)cdiv(m, kStatChunk)};    // gather (block start)
-  const Stats st_m{B.spart, B.kpart, decorrelate_chunks(m)};       // U-step decorrelation
-  const Stats st_n{B.spart, B.kpart, decorrelate_chunks(n)};       // V-step decorrelation
+  // each producer of Eq. 2 statistics and its apply agree on the chunk count; the producer's last CTA writes the
+  // thresholds the apply reads
+  const Thresh th_m{B.theta, B.fallback, B.arg, B.ticket, p.tau, m};
+  const Thresh th_n{B.theta, B.fallback, B.arg, B.ticket, p.tau, n};
+  const Stats st_g{B.spart, B.kpart, (int)cdiv(m, kStatChunk), th_m};   // gather (block start)
+  const Stats st_m{B.spart, B.kpart, decorrelate_chunks(m), th_m};       // U-step decorrelation
+  const Stats st_n{B.spart, B.kpart, decorrelate_chunks(n), th_n};       // V-step decorrelation
   const int nrt = deflate_row_tiles(m), ntiles = deflate_tiles(m, n);
   g_prof.used = 0;
   g_prof.launches = 0;
@@ -333,34 +351,56 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
     const long long j0 = (long long)blk * p.b;
     const int w = (int)std::min<long long>(p.b, p.k - j0);
     const int sv = splits_v(w, m, n), su = splits_u(w, m, n);
+    // Exact Gram matrices of unweighted ternary factors are accumulated by the apply that writes the factor
+    // (integer atomics) up to 128 components; wider blocks and the weighted V^T H V use the Gram kernel.
+    const bool fusedU = w <= 128, fusedV = w <= 128 && h == nullptr;
     KL(kStart, 2, launch_select_with(B.colpart, nrt, n, h, w, B.J, B.colE, s));
     KL(kStart, 1, launch_gather(B.R, m, n, B.J, w, B.X, m, st_g, s));
-    KL(kApply, 1, launch_apply(B.X, w, m, m, st_g, p.tau, B.Ut, (int)p.ldm, s));
+    __half* const U16 = use_tc(w) ? B.Ut16 : nullptr;
+    __half* const V16 = use_tc(w) ? B.Vt16 : nullptr;
+    KL(kApply, 1, launch_apply(B.X, w, m, m, th_m, B.Ut, (int)p.ldm, (fusedU && w > 1) ? B.GintU : nullptr, s, U16,
+                               p.ldm));
     for (int it = 0; it < p.iters; ++it) {
+      const bool last = it == p.iters - 1;
       // V-step: V <- T([(U^T U + eps I)^-1 U^T R]^T)   (plain R even when weighted, §2.5).
       // The Gram inverse depends only on U: it runs on the side branch while the product streams R.
       if (w > 1) {
         FORK();
-        KLS(kGram, 1, side, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, side));
-        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side));
+        if (fusedU) {
+          KLS(kSolve, 1, side, launch_inverse_int(B.GintU, w, B.GrawU, B.Ginv, side));
+        } else {
+          KLS(kGram, 1, side, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, side));
+          KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side));
+        }
       }
-      KL(kVstep, 1, product_v(B.R, m, n, B.Ut, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
+      KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
       if (w > 1) JOIN();
       KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, sv, n, B.X, n, st_n, s));
-      KL(kApply, 1, launch_apply(B.X, w, n, n, st_n, p.tau, B.Vt, (int)p.ldn, s));
+      KL(kApply, 1, launch_apply(B.X, w, n, n, th_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, s, V16, p.ldn));
       // U-step: U <- T(R H V (V^T H V + eps I)^-1)
       FORK();
-      KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
-      KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side));
-      KL(kUstep, 1, product_u(B.R, m, n, B.Vt, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s));
+      if (fusedV) {
+        KLS(kSolve, 1, side, launch_inverse_int(B.GintV, w, B.GrawV, B.Ginv, side));
+      } else {
+        KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
+        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side));
+      }
+      KL(kUstep, 1, product_u(B.R, m, n, B.Vt, V16, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s));
       JOIN();
       KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, su, m, B.X, m, st_m, s));
-      KL(kApply, 1, launch_apply(B.X, w, m, m, st_m, p.tau, B.Ut, (int)p.ldm, s));
+      // the next V-step's inverse (w > 1) or, after the last iteration, Eq. 4 consumes U's Gram
+      // (the fp16 copy of U is not needed after the last iteration)
+      KL(kApply, 1, launch_apply(B.X, w, m, m, th_m, B.Ut, (int)p.ldm, (fusedU && (w > 1 || last)) ? B.GintU : nullptr,
+                                 s, last ? nullptr : U16, p.ldm));
     }
     // Eq. 4: [(U^T U) .* (V^T H V)] d = diag(U^T R H V), with R H V the last U-step product
-    KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
     KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, su, B.r, s));
-    KL(kSolve, 1, launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s));
+    if (fusedU) {
+      KL(kSolve, 1, launch_scales_int(B.GintU, B.GrawV, B.r, w, B.d, s));
+    } else {
+      KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
+      KL(kSolve, 1, launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s));
+    }
     // R <- R - U diag(d) V^T
     KL(kDeflate, 1, launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart, B.normpart,
                                    s, B.maxpart));
@@ -494,16 +534,31 @@ int step_scalars(Workspace& ws, const float* R, long long count, const float* h,
   return EXTERND_OK;
 }
 
-// Per-step helpers: bring a caller's m x w U into the internal Ut layout, and a w x n Cb into Vt.
-int stage_u(Workspace& ws, const int8_t* U, long long m, int w, int8_t** Ut) {
+// Per-step helpers: bring a caller's m x w U into the internal Ut layout, and a w x n Cb into Vt; with T16 given,
+// also the fp16 copy the tensor-core products read (nullptr when the FMA tiles run).
+int stage_u(Workspace& ws, const int8_t* U, long long m, int w, int8_t** Ut, __half** T16 = nullptr) {
   TRY(need(ws, "Ut", (size_t)w * ld16(m), Ut, true));
   LK(launch_transpose_i8(U, w, (int)m, w, *Ut, ld16(m), g_stream));
+  if (T16 != nullptr) {
+    *T16 = nullptr;
+    if (use_tc(w)) {
+      TRY(need(ws, "Ut16", (size_t)w * ld16(m), T16, true));
+      LK(launch_i8_to_f16(*Ut, ld16(m), w, (int)m, *T16, ld16(m), g_stream));
+    }
+  }
   return EXTERND_OK;
 }
 
-int stage_v(Workspace& ws, const int8_t* Cb, long long n, int w, int8_t** Vt) {
+int stage_v(Workspace& ws, const int8_t* Cb, long long n, int w, int8_t** Vt, __half** T16 = nullptr) {
   TRY(need(ws, "Vt", (size_t)w * ld16(n), Vt, true));
   LK(cudaMemcpy2DAsync(*Vt, (size_t)ld16(n), Cb, (size_t)n, (size_t)n, (size_t)w, cudaMemcpyDeviceToDevice, g_stream));
+  if (T16 != nullptr) {
+    *T16 = nullptr;
+    if (use_tc(w)) {
+      TRY(need(ws, "Vt16", (size_t)w * ld16(n), T16, true));
+      LK(launch_i8_to_f16(Cb, n, w, (int)n, *T16, ld16(n), g_stream));
+    }
+  }
   return EXTERND_OK;
 }
 
@@ -670,12 +725,20 @@ int externd_ternarize(const float* X, int64_t rows, int64_t cols, int axis, doub
   const int nchunk = (int)cdiv(L, kStatChunk);
   F2* sp;
   u64* kp;
+  float* theta;
+  int* fb;
+  unsigned *arg, *ticket;
   TRY(need(*ws, "tern.spart", (size_t)nv * nchunk, &sp));
   TRY(need(*ws, "tern.kpart", (size_t)nv * nchunk, &kp));
-  Stats st{sp, kp, nchunk};
+  TRY(need(*ws, "tern.theta", (size_t)nv, &theta));
+  TRY(need(*ws, "tern.fallback", (size_t)nv, &fb));
+  TRY(need(*ws, "tern.arg", (size_t)nv, &arg));
+  TRY(need(*ws, "ticket", 1, &ticket, true));
+  const Thresh th{theta, fb, arg, ticket, tau, (int)L};
+  Stats st{sp, kp, nchunk, th};
   if (axis == 1) {
     LK(launch_stats(X, (int)nv, (int)L, (int)L, st, g_stream));
-    LK(launch_apply(X, (int)nv, (int)L, L, st, tau, T, (int)L, g_stream));
+    LK(launch_apply(X, (int)nv, (int)L, L, th, T, (int)L, nullptr, g_stream));
   } else {
     float* Xt;
     int8_t* Tt;
@@ -683,7 +746,7 @@ int externd_ternarize(const float* X, int64_t rows, int64_t cols, int axis, doub
     TRY(need(*ws, "tern.T", (size_t)nv * L, &Tt));
     LK(launch_transpose_f32(X, cols, (int)rows, (int)cols, Xt, L, g_stream));
     LK(launch_stats(Xt, (int)nv, (int)L, (int)L, st, g_stream));
-    LK(launch_apply(Xt, (int)nv, (int)L, L, st, tau, Tt, (int)L, g_stream));
+    LK(launch_apply(Xt, (int)nv, (int)L, L, th, Tt, (int)L, nullptr, g_stream));
     LK(launch_transpose_i8(Tt, L, (int)nv, (int)L, T, cols, g_stream));
   }
   CK(cudaGetLastError());
@@ -703,13 +766,14 @@ int externd_vstep_product(const float* R, int64_t m, int64_t n, const int8_t* U,
   Workspace* ws;
   TRY(current_ws(&ws));
   int8_t* Ut;
+  __half* U16;
   float *part, *mx;
   unsigned* err;
-  TRY(stage_u(*ws, U, m, (int)w, &Ut));
+  TRY(stage_u(*ws, U, m, (int)w, &Ut, &U16));
   TRY(step_scalars(*ws, R, m * n, nullptr, 0, &mx, &err));
   const int sv = splits_v((int)w, (int)m, (int)n);
   TRY(need(*ws, "part", (size_t)sv * w * n, &part));
-  LK(product_v(R, (int)m, (int)n, Ut, (int)ld16(m), (int)w, part, sv, mx, err, g_stream));
+  LK(product_v(R, (int)m, (int)n, Ut, U16, (int)ld16(m), (int)w, part, sv, mx, err, g_stream));
   LK(launch_sum_splits(part, sv, (int)w, (int)n, PV, n, g_stream));
   return check_device_error(*ws, err, g_stream);
 }
@@ -724,14 +788,15 @@ int externd_ustep_product(const float* R, int64_t m, int64_t n, const int8_t* Cb
   Workspace* ws;
   TRY(current_ws(&ws));
   int8_t* Vt;
+  __half* V16;
   float *part, *X, *mx;
   unsigned* err;
-  TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
+  TRY(stage_v(*ws, Cb, n, (int)w, &Vt, &V16));
   TRY(step_scalars(*ws, R, m * n, weights, n, &mx, &err));
   const int su = splits_u((int)w, (int)m, (int)n);
   TRY(need(*ws, "part", (size_t)su * w * m, &part));
   TRY(need(*ws, "X", (size_t)w * m, &X));
-  LK(product_u(R, (int)m, (int)n, Vt, (int)ld16(n), (int)w, weights, part, su, mx, err, g_stream));
+  LK(product_u(R, (int)m, (int)n, Vt, V16, (int)ld16(n), (int)w, weights, part, su, mx, err, g_stream));
   LK(launch_sum_splits(part, su, (int)w, (int)m, X, m, g_stream));
   LK(launch_transpose_f32(X, m, (int)w, (int)m, PU, w, g_stream));
   return check_device_error(*ws, err, g_stream);
@@ -745,11 +810,12 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   const long long L = vstep ? n : m;
   const int nchunk = decorrelate_chunks((int)L);
   int8_t* T;
+  __half* T16;
   float *part, *X, *Gpart, *Graw, *Ginv, *one;
   F2* sp;
   u64* kp;
-  if (vstep) TRY(stage_u(*ws, F, m, w, &T));
-  else TRY(stage_v(*ws, F, n, w, &T));
+  if (vstep) TRY(stage_u(*ws, F, m, w, &T, &T16));
+  else TRY(stage_v(*ws, F, n, w, &T, &T16));
   const long long ldt = vstep ? ld16(m) : ld16(n);
   const long long Lred = vstep ? m : n;
   float* mx;
@@ -765,13 +831,20 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   TRY(need(*ws, "spart", (size_t)w * nchunk, &sp));
   TRY(need(*ws, "kpart", (size_t)w * nchunk, &kp));
   TRY(get_one(*ws, &one));
-  if (vstep) LK(product_v(R, (int)m, (int)n, T, (int)ldt, w, part, splits, mx, err, g_stream));
-  else LK(product_u(R, (int)m, (int)n, T, (int)ldt, w, h, part, splits, mx, err, g_stream));
+  if (vstep) LK(product_v(R, (int)m, (int)n, T, T16, (int)ldt, w, part, splits, mx, err, g_stream));
+  else LK(product_u(R, (int)m, (int)n, T, T16, (int)ldt, w, h, part, splits, mx, err, g_stream));
   if (w > 1) {
     LK(launch_gram(T, (int)ldt, w, (int)Lred, vstep ? nullptr : h, Gpart, gs, g_stream));
     LK(launch_inverse(Gpart, gs, w, Graw, Ginv, g_stream));
   }
-  Stats st{sp, kp, nchunk};
+  float* theta;
+  int* fb;
+  unsigned *arg, *ticket;
+  TRY(need(*ws, "theta", (size_t)w, &theta));
+  TRY(need(*ws, "fallback", (size_t)w, &fb));
+  TRY(need(*ws, "arg", (size_t)w, &arg));
+  TRY(need(*ws, "ticket", 1, &ticket, true));
+  Stats st{sp, kp, nchunk, Thresh{theta, fb, arg, ticket, 0.0, (int)L}};
   if (vstep) {
     LK(launch_decorrelate(w > 1 ? Ginv : one, w, part, splits, (int)L, out, (int)L, st, g_stream));
   } else {
@@ -811,11 +884,12 @@ int externd_block_scales(const float* R, int64_t m, int64_t n, const int8_t* U, 
   Workspace* ws;
   TRY(current_ws(&ws));
   int8_t *Ut, *Vt;
+  __half* V16;
   float *part, *Gpart, *GrawV, *Ginv, *mx;
   unsigned* err;
   float* r;
   TRY(stage_u(*ws, U, m, (int)w, &Ut));
-  TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
+  TRY(stage_v(*ws, Cb, n, (int)w, &Vt, &V16));
   TRY(step_scalars(*ws, R, m * n, weights, n, &mx, &err));
   const int su = splits_u((int)w, (int)m, (int)n);
   const int gm = gram_splits((int)w, (int)m), gn = gram_splits((int)w, (int)n);
@@ -824,7 +898,7 @@ int externd_block_scales(const float* R, int64_t m, int64_t n, const int8_t* U, 
   TRY(need(*ws, "GrawV", (size_t)w * w, &GrawV));
   TRY(need(*ws, "Ginv", (size_t)w * w, &Ginv));
   TRY(need(*ws, "r", (size_t)w, &r));
-  LK(product_u(R, (int)m, (int)n, Vt, (int)ld16(n), (int)w, weights, part, su, mx, err, g_stream));
+  LK(product_u(R, (int)m, (int)n, Vt, V16, (int)ld16(n), (int)w, weights, part, su, mx, err, g_stream));
   LK(launch_gram(Vt, (int)ld16(n), (int)w, (int)n, weights, Gpart, gn, g_stream));
   LK(launch_inverse(Gpart, gn, (int)w, GrawV, Ginv, g_stream));
   LK(launch_gram(Ut, (int)ld16(m), (int)w, (int)m, nullptr, Gpart, gm, g_stream));

@@ -130,65 +130,92 @@ __global__ void __launch_bounds__(256) product_kernel(const float* __restrict__ 
 }
 
 // X tile of 64 components x 32 positions: thread (ty, tx) owns components ty*4..+3 at positions tx*2, tx*2+1.
-// Narrow tiles give enough CTAs to read the split-K partials in parallel at small L.
+// Narrow tiles give enough CTAs to read the split-K partials in parallel at small L. The CTA first stages, with
+// every load of a batch in flight before any is used,
+//   Ps[b][x]  = sum_s part[s][b][x0 + x]   for all w components b (split order)
+//   Gs[b][a]  = Ginv[b][a0 + a]            (Ginv is symmetric: row b holds column b)
+// in dynamic shared memory, then runs the w-deep product out of shared memory.
 constexpr int DX = 32;
+constexpr int kGsLd = TM + 4;
+
+size_t decorrelate_smem(int w) { return (size_t)w * (DX + kGsLd) * sizeof(float); }
 
 __global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restrict__ Ginv, int w,
                                                           const float* __restrict__ part, int splits, int L,
                                                           float* __restrict__ X, int ldx, Stats st) {
-  __shared__ __align__(16) float Ps[TK][DX];
-  __shared__ __align__(16) float Gs[TK][TM + 4];
+  extern __shared__ __align__(16) float dsm[];
+  float* const Ps = dsm;                 // [w][DX]
+  float* const Gs = dsm + w * DX;        // [w][kGsLd]
   const int x0 = blockIdx.x * DX;
   const int a0 = blockIdx.y * TM;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
-  float acc[4][2] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
 
-  for (int b0 = 0; b0 < w; b0 += TK) {
-    {
-      // Ps[kb][kx..kx+1] = sum_s part[s][b0 + kb][x0 + kx..]: 16 x 32 floats, 2 per thread
-      const int kb = tid >> 4, kx = (tid & 15) * 2;
-      const int b = b0 + kb, x = x0 + kx;
-      float v0 = 0.f, v1 = 0.f;
-      if (b < w) {
-        // independent loads first (8 splits at a time), then the sum in split order
-        const float* p = part + (long long)b * L + x;
-        const long long stride = (long long)w * L;
-        for (int q0 = 0; q0 < splits; q0 += 8) {
-          float a0[8], a1[8];
+  // Ginv rows: w x 16 float4 slots
+  {
+    const bool gvec = (w & 3) == 0;
+    for (int i0 = 0; i0 < w * 16; i0 += 4 * 256) {
+      float4 g[4];
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            const bool in = q0 + q < splits;
-            a0[q] = (in && x < L) ? p[(q0 + q) * stride] : 0.f;
-            a1[q] = (in && x + 1 < L) ? p[(q0 + q) * stride + 1] : 0.f;
-          }
-#pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            v0 += a0[q];
-            v1 += a1[q];
-          }
-        }
+      for (int q = 0; q < 4; ++q) {
+        const int i = i0 + q * 256 + tid;
+        g[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i < w * 16) g[q] = load4(Ginv + (long long)(i >> 4) * w, a0 + (i & 15) * 4, w, gvec);
       }
-      Ps[kb][kx] = v0;
-      Ps[kb][kx + 1] = v1;
-    }
-    {
-      const int kb = tid >> 4, a4 = (tid & 15) * 4;
-      const int b = b0 + kb;
-      float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (b < w) g = load4(Ginv + (long long)b * w, a0 + a4, w, (w & 3) == 0);
-      *reinterpret_cast<float4*>(&Gs[kb][a4]) = g;
-    }
-    __syncthreads();
 #pragma unroll
-    for (int k = 0; k < TK; ++k) {
-      const float4 g = *reinterpret_cast<const float4*>(&Gs[k][ty * 4]);
-      const float2 p = *reinterpret_cast<const float2*>(&Ps[k][tx * 2]);
-      acc[0][0] = fmaf(g.x, p.x, acc[0][0]); acc[0][1] = fmaf(g.x, p.y, acc[0][1]);
-      acc[1][0] = fmaf(g.y, p.x, acc[1][0]); acc[1][1] = fmaf(g.y, p.y, acc[1][1]);
-      acc[2][0] = fmaf(g.z, p.x, acc[2][0]); acc[2][1] = fmaf(g.z, p.y, acc[2][1]);
-      acc[3][0] = fmaf(g.w, p.x, acc[3][0]); acc[3][1] = fmaf(g.w, p.y, acc[3][1]);
+      for (int q = 0; q < 4; ++q) {
+        const int i = i0 + q * 256 + tid;
+        if (i < w * 16) *reinterpret_cast<float4*>(&Gs[(i >> 4) * kGsLd + (i & 15) * 4]) = g[q];
+      }
     }
-    __syncthreads();
+  }
+  // split sums: w x 8 float4 slots, 4 slots x 4 splits of loads in flight per thread
+  {
+    constexpr int E = 4, SB = 4;
+    const bool pvec = (L & 3) == 0;
+    const long long sstride = (long long)w * L;
+    for (int i0 = 0; i0 < w * 8; i0 += E * 256) {
+      float4 acc[E];
+#pragma unroll
+      for (int e = 0; e < E; ++e) acc[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int s0 = 0; s0 < splits; s0 += SB) {
+        float4 v[SB][E];
+#pragma unroll
+        for (int q = 0; q < SB; ++q)
+#pragma unroll
+          for (int e = 0; e < E; ++e) {
+            const int i = i0 + e * 256 + tid;
+            v[q][e] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (s0 + q < splits && i < w * 8)
+              v[q][e] = load4(part + (s0 + q) * sstride + (long long)(i >> 3) * L, x0 + (i & 7) * 4, L, pvec);
+          }
+#pragma unroll
+        for (int q = 0; q < SB; ++q)
+#pragma unroll
+          for (int e = 0; e < E; ++e) {
+            acc[e].x += v[q][e].x;
+            acc[e].y += v[q][e].y;
+            acc[e].z += v[q][e].z;
+            acc[e].w += v[q][e].w;
+          }
+      }
+#pragma unroll
+      for (int e = 0; e < E; ++e) {
+        const int i = i0 + e * 256 + tid;
+        if (i < w * 8) *reinterpret_cast<float4*>(&Ps[(i >> 3) * DX + (i & 7) * 4]) = acc[e];
+      }
+    }
+  }
+  __syncthreads();
+
+  float acc[4][2] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+#pragma unroll 4
+  for (int b = 0; b < w; ++b) {
+    const float4 g = *reinterpret_cast<const float4*>(&Gs[b * kGsLd + ty * 4]);
+    const float2 p = *reinterpret_cast<const float2*>(&Ps[b * DX + tx * 2]);
+    acc[0][0] = fmaf(g.x, p.x, acc[0][0]); acc[0][1] = fmaf(g.x, p.y, acc[0][1]);
+    acc[1][0] = fmaf(g.y, p.x, acc[1][0]); acc[1][1] = fmaf(g.y, p.y, acc[1][1]);
+    acc[2][0] = fmaf(g.z, p.x, acc[2][0]); acc[2][1] = fmaf(g.z, p.y, acc[2][1]);
+    acc[3][0] = fmaf(g.w, p.x, acc[3][0]); acc[3][1] = fmaf(g.w, p.y, acc[3][1]);
   }
 
 #pragma unroll
@@ -220,6 +247,7 @@ __global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restric
       st.kpart[(long long)a * st.nchunk + blockIdx.x] = key;
     }
   }
+  stats_done(st, w);
 }
 
 template <bool UROW>
@@ -396,8 +424,15 @@ int decorrelate_chunks(int L) { return (int)cdiv(L, DX); }
 
 cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
                                Stats st, cudaStream_t s) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(decorrelate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)decorrelate_smem(kMaxBlock));
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
   dim3 grid((unsigned)cdiv(L, DX), (unsigned)cdiv(w, TM));
-  decorrelate_kernel<<<grid, 256, 0, s>>>(Ginv, w, part, splits, L, X, ldx, st);
+  decorrelate_kernel<<<grid, 256, decorrelate_smem(w), s>>>(Ginv, w, part, splits, L, X, ldx, st);
   return cudaGetLastError();
 }
 

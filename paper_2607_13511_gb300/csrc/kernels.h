@@ -10,6 +10,7 @@
 //          kpart[a * nchunk + c] = max magnitude key over chunk c (chunks of kStatChunk positions).
 #pragma once
 
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -17,11 +18,88 @@
 
 namespace externd {
 
+// Eq. 2 thresholds of nv vectors of length L: theta = RD_float(tau * S / L), whether nothing passes, and the
+// fallback index. The last CTA of the statistics producer writes them (ticket counts finished CTAs and is reset
+// to zero by that CTA).
+struct Thresh {
+  float* theta;
+  int* fallback;
+  unsigned* arg;
+  unsigned* ticket;
+  double tau;
+  int L;
+};
+
 struct Stats {
   F2* spart;
   u64* kpart;
   int nchunk;
+  Thresh th;
 };
+
+// Run by the CTA that finished last: sums every vector's chunk partials (double-float) and writes its threshold.
+// G threads per vector (a power of two, as many as the CTA allows up to a warp) each take chunks g, g + G, ...
+// with all of a batch's loads issued before any is used, then combine with a butterfly inside the group: a fixed
+// order, so the result is reproducible. The double-precision division happens once per vector.
+__device__ __forceinline__ void finalize_thresholds(const Stats& st, int nv) {
+  constexpr int kBatch = 16;
+  const int nt = blockDim.x;
+  int G = 32;
+  while (G > 1 && G * nv > nt) G >>= 1;
+  const int g = threadIdx.x & (G - 1);
+  for (int a0 = 0; a0 < nv; a0 += nt / G) {   // uniform across the CTA: every lane reaches the shuffles
+    const int a = a0 + (int)threadIdx.x / G;
+    const bool act = a < nv;
+    const F2* sp = st.spart + (long long)a * st.nchunk;
+    const u64* kp = st.kpart + (long long)a * st.nchunk;
+    F2 s;
+    u64 key = 0;
+    for (int c0 = 0; c0 < st.nchunk; c0 += kBatch * G) {
+      F2 sv[kBatch];
+      u64 kv[kBatch];
+#pragma unroll
+      for (int i = 0; i < kBatch; ++i) {
+        const int c = c0 + i * G + g;
+        const bool in = act && c < st.nchunk;
+        sv[i] = in ? sp[c] : F2{};
+        kv[i] = in ? kp[c] : 0ull;
+      }
+#pragma unroll
+      for (int i = 0; i < kBatch; ++i) {
+        s = f2_add(s, sv[i]);
+        key = kv[i] > key ? kv[i] : key;
+      }
+    }
+    for (int o = G >> 1; o > 0; o >>= 1) {
+      s = f2_add(s, f2_shfl_xor(s, o));
+      const u64 t = __shfl_xor_sync(0xffffffffu, key, o);
+      key = t > key ? t : key;
+    }
+    if (act && g == 0) {
+      const float th = __double2float_rd(st.th.tau * (f2_value(s) / (double)st.th.L));
+      st.th.theta[a] = th;
+      st.th.fallback[a] = !(key_mag(key) > th);
+      st.th.arg[a] = key_index(key);
+    }
+  }
+}
+
+// Last-CTA protocol: every CTA calls this after writing its partials; the last one to arrive finalizes.
+__device__ __forceinline__ void stats_done(const Stats& st, int nv) {
+  __shared__ int s_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const unsigned total = gridDim.x * gridDim.y * gridDim.z;
+    s_last = (atomicAdd(st.th.ticket, 1u) == total - 1u);
+  }
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    finalize_thresholds(st, nv);
+    if (threadIdx.x == 0) *st.th.ticket = 0u;
+  }
+}
 
 // ---- products (gemm.cu)
 // Split-K factor of a product with Lx output positions per component and reduction length Ly.
@@ -44,17 +122,25 @@ cudaError_t launch_deflate(const float* Rin, float* Rout, int m, int n, const in
 int deflate_row_tiles(int m);
 int deflate_tiles(int m, int n);
 
-// ---- tensor-core products (product_tc.cu): w >= 16; maxabs = {max |R|, max h}; err = device error word
+// ---- tensor-core products (product_tc.cu): w >= 16; the factor as fp16 rows (ld elements, 16-byte aligned, zero
+// padded); maxabs = {max |R|, max h}; err = device error word
 int tc_product_splits(int w, int Lx, int Ly);
-cudaError_t launch_product_v_tc(const float* R, int m, int n, const int8_t* Ut, int ldu, int w, float* part,
+cudaError_t launch_product_v_tc(const float* R, int m, int n, const __half* Ut, int ldu, int w, float* part,
                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s);
-cudaError_t launch_product_u_tc(const float* R, int m, int n, const int8_t* Vt, int ldv, int w, const float* h,
+cudaError_t launch_product_u_tc(const float* R, int m, int n, const __half* Vt, int ldv, int w, const float* h,
                                 float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s);
+// dst[r][c] = (half) src[r][c] for an rows x cols int8 matrix
+cudaError_t launch_i8_to_f16(const int8_t* src, long long lds, int rows, int cols, __half* dst, long long ldd,
+                             cudaStream_t s);
 
 // ---- ternarization and bookkeeping (tern.cu)
 cudaError_t launch_stats(const float* X, int nv, int L, int ldx, Stats st, cudaStream_t s);
-cudaError_t launch_apply(const float* X, int nv, int L, int ldx, Stats st, double tau, int8_t* T, int ldt,
-                         cudaStream_t s);
+// T = T_tau(X) from finalized thresholds. If gram != NULL (requires nv <= 256) also accumulates the exact Gram
+// matrix of the ternary vectors into the upper triangle gram[a * nv + b] (a <= b) with integer atomics (gram
+// must hold zeros or a running sum).
+// T16 (optional): the same ternary values as fp16 rows with leading dimension ldt16.
+cudaError_t launch_apply(const float* X, int nv, int L, int ldx, const Thresh& th, int8_t* T, int ldt, int* gram,
+                         cudaStream_t s, __half* T16 = nullptr, long long ldt16 = 0);
 cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, float* Y, int ldy, Stats st,
                           cudaStream_t s);
 // J = the w columns of largest h_c * sum_t colpart[t][c] (ties to the lower c), ascending; e (n floats) is scratch.
@@ -83,11 +169,15 @@ cudaError_t launch_gram(const int8_t* T, int ldt, int w, int L, const float* h, 
                         cudaStream_t s);
 // Graw = sum_s Gpart[s]; Ginv = (Graw + eps I)^-1 with eps = kEpsRel * trace / w.
 cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s);
+// Same from an integer upper-triangle Gram (as written by launch_apply), which is reset to zero after reading.
+cudaError_t launch_inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s);
 // r[a] = sum_y Ut[a][y] * sum_s part[s][a][y]
 cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, float* r,
                         cudaStream_t s);
 // d solves [(sum_s GUpart[s]) .* GVraw + eps I] d = r (eps = 0 when w == 1).
 cudaError_t launch_scales(const float* GUpart, int splits, const float* GVraw, const float* r, int w, float* d,
                           cudaStream_t s);
+// Same with G_U from an integer upper-triangle Gram, reset to zero after reading.
+cudaError_t launch_scales_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s);
 
 }  // namespace externd

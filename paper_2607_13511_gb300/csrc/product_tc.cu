@@ -10,10 +10,11 @@
 // accumulator, which the epilogue scales back by 2^-s. That keeps ~22 significant bits of every residual entry
 // (the float32 product bar is 1e-5 relative), at twice the MMA count of a plain fp16 product.
 //
-// Warps 0-7 convert: they load float32 R with coalesced 16-byte loads, convert, and store straight into the
-// 128-byte-swizzled K-major tiles the MMA reads (the V-step transposes on the way: its A rows are R's columns).
-// Warp 8 allocates tensor memory and one of its threads issues the MMAs. Stages hand over through mbarriers:
-// full[s] (256 producer arrivals), empty[s] (tcgen05.commit after the stage's MMAs), done (after the last).
+// Warps 0-15 convert: they load float32 R with coalesced 16-byte loads, convert two values per instruction, and
+// store straight into the 128-byte-swizzled K-major tiles the MMA reads (the V-step transposes on the way: its A
+// rows are R's columns); the ternary factor arrives as fp16 rows written by the ternarization and is copied.
+// Warp 16 allocates tensor memory and one of its threads issues the MMAs. Stages hand over through mbarriers:
+// full[s] (512 producer arrivals), empty[s] (tcgen05.commit after the stage's MMAs), done (after the last).
 #include "kernels.h"
 #include "umma.cuh"
 
@@ -21,15 +22,16 @@ namespace externd {
 
 namespace {
 
-constexpr int kThreads = 288;     // 8 converter/epilogue warps + 1 MMA warp
-constexpr int kProducers = 256;
+constexpr int kProducerWarps = 16;
+constexpr int kProducers = kProducerWarps * 32;
+constexpr int kThreads = kProducers + 32;   // converter/epilogue warps + 1 MMA warp
 constexpr int kStageK = 64;       // reduction elements per stage: one 128-byte swizzle row of fp16
 constexpr uint32_t kTileA = 128u * 128u;   // 128 rows x 64 fp16
 
 struct TcArgs {
   const float* R;
   int m, n;
-  const int8_t* T;        // ternary factor, component-major (w rows, ldt bytes each, zero padded)
+  const __half* T;        // ternary factor as fp16, component-major (w rows, ldt elements each, zero padded)
   int ldt, w, wpad;
   const float* h;         // U-step importances or nullptr
   float* part;            // split-K partials [splits][w][Lx]
@@ -44,31 +46,29 @@ __device__ __forceinline__ void st_shared16(uint8_t* p, uint32_t a, uint32_t b, 
   *reinterpret_cast<uint4*>(p) = make_uint4(a, b, c, d);
 }
 
-// 8 scaled values -> one hi chunk and one lo chunk (4 x half2 each).
-__device__ __forceinline__ void split_chunk(const float (&x)[8], uint32_t (&hi)[4], uint32_t (&lo)[4]) {
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    __half h0, l0, h1, l1;
-    split_f16(x[2 * e], h0, l0);
-    split_f16(x[2 * e + 1], h1, l1);
-    hi[e] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-    lo[e] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
-  }
+// Scaled pairs -> fp16 hi = RN(x) and lo = RN(x - hi), packed two per 32-bit word (one conversion per pair).
+__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __half2 h = __floats2half2_rn(x0, x1);
+  const float2 hb = __half22float2(h);
+  const __half2 l = __floats2half2_rn(x0 - hb.x, x1 - hb.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
-// Loads this thread's 32 residual values of stage k into registers (zeros outside the matrix / split).
-// V-step: rows y0 + 8o + j (j < 8) at columns x0 + 4q .. +3, v[4j + i]. U-step: rows x0 + row_t (t < 4) at
-// columns y0 + 8 (lane & 7) .. +7, v[8t + e].
+// Loads this thread's 16 residual values of stage k into registers (zeros outside the matrix / split).
+// V-step: rows y0 + 8o + 4hf + j (j < 4) at columns x0 + 4q .. +3 -> v[4j + i], with o = lane % 8,
+//         q = (warp % 8) * 4 + lane / 8, hf = warp / 8.
+// U-step: rows x0 + warp * 8 + lane / 8 + 4t (t < 2) at columns y0 + 8 (lane % 8) .. +7 -> v[8t + e].
 template <bool USTEP>
 __device__ __forceinline__ void load_stage(const TcArgs& p, int k, int ybeg, int yend, int x0, int warp, int lane,
-                                           bool vec, float (&v)[32]) {
+                                           bool vec, float (&v)[16]) {
   const int y0 = ybeg + k * kStageK;
   if (!USTEP) {
-    const int o = lane & 7, q = warp * 4 + (lane >> 3);
+    const int o = lane & 7, q = (warp & 7) * 4 + (lane >> 3), hf = warp >> 3;
     const int c = x0 + 4 * q;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int y = y0 + 8 * o + j;
+    for (int j = 0; j < 4; ++j) {
+      const int y = y0 + 8 * o + 4 * hf + j;
       float4 t = make_float4(0.f, 0.f, 0.f, 0.f);
       if (y < yend) t = load4(p.R + (long long)y * p.n, c, p.n, vec);
       v[4 * j + 0] = t.x;
@@ -79,8 +79,8 @@ __device__ __forceinline__ void load_stage(const TcArgs& p, int k, int ybeg, int
   } else {
     const int c = y0 + 8 * (lane & 7);
 #pragma unroll
-    for (int t = 0; t < 4; ++t) {
-      const int r = x0 + warp * 16 + (lane >> 3) + 4 * t;
+    for (int t = 0; t < 2; ++t) {
+      const int r = x0 + warp * 8 + (lane >> 3) + 4 * t;
       float4 v0 = make_float4(0.f, 0.f, 0.f, 0.f), v1 = v0;
       if (r < p.m) {
         v0 = load4(p.R + (long long)r * p.n, c, yend, vec);
@@ -98,12 +98,12 @@ __device__ __forceinline__ void load_stage(const TcArgs& p, int k, int ybeg, int
   }
 }
 
-// Waits for stage slot k % S to be free, converts the loaded values into the swizzled fp16 hi/lo A tiles and the
-// ternary B tile, and arrives on full[slot]. False if the wait timed out.
+// Waits for stage slot k % S to be free, converts the loaded values into the swizzled fp16 hi/lo A tiles, copies
+// the fp16 ternary B tile, and arrives on full[slot]. False if the wait timed out.
 template <bool USTEP>
 __device__ __forceinline__ bool convert_stage(const TcArgs& p, int k, int S, uint32_t stage_bytes, uint8_t* gbase,
                                               uint32_t bars, int ybeg, int yend, int x0, int tid, int warp, int lane,
-                                              bool vec, float scale, const float (&v)[32]) {
+                                              bool vec, float scale, const float (&v)[16]) {
   const int s = k % S, round = k / S;
   if (round > 0 && !mbar_wait(bars + 8u * (S + s), (uint32_t)(round - 1) & 1u, p.err)) return false;
   uint8_t* a_hi = gbase + (uint32_t)s * stage_bytes;
@@ -111,17 +111,16 @@ __device__ __forceinline__ bool convert_stage(const TcArgs& p, int k, int S, uin
   uint8_t* bt = a_hi + 2u * kTileA;
   const int y0 = ybeg + k * kStageK;
   if (!USTEP) {
-    const int o = lane & 7, q = warp * 4 + (lane >> 3);
+    // A row = local column 4q + i; this thread writes the 8-byte half hf of chunk o (rows 8o + 4hf .. +3)
+    const int o = lane & 7, q = (warp & 7) * 4 + (lane >> 3), hf = warp >> 3;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      float x[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) x[j] = v[4 * j + i] * scale;
-      uint32_t hi[4], lo[4];
-      split_chunk(x, hi, lo);
-      const uint32_t off = sw128_offset((uint32_t)(4 * q + i), (uint32_t)o);
-      st_shared16(a_hi + off, hi[0], hi[1], hi[2], hi[3]);
-      st_shared16(a_lo + off, lo[0], lo[1], lo[2], lo[3]);
+      uint32_t h0, l0, h1, l1;
+      split_pair(v[i] * scale, v[4 + i] * scale, h0, l0);
+      split_pair(v[8 + i] * scale, v[12 + i] * scale, h1, l1);
+      const uint32_t off = sw128_offset((uint32_t)(4 * q + i), (uint32_t)o) + 8u * hf;
+      *reinterpret_cast<uint2*>(a_hi + off) = make_uint2(h0, h1);
+      *reinterpret_cast<uint2*>(a_lo + off) = make_uint2(l0, l1);
     }
   } else {
     const int j = lane & 7;
@@ -133,36 +132,35 @@ __device__ __forceinline__ bool convert_stage(const TcArgs& p, int k, int S, uin
       hv[4] = h1.x; hv[5] = h1.y; hv[6] = h1.z; hv[7] = h1.w;
     }
 #pragma unroll
-    for (int t = 0; t < 4; ++t) {
-      const int row = warp * 16 + (lane >> 3) + 4 * t;
-      float x[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) x[e] = v[8 * t + e] * hv[e] * scale;
+    for (int t = 0; t < 2; ++t) {
+      const int row = warp * 8 + (lane >> 3) + 4 * t;
       uint32_t hi[4], lo[4];
-      split_chunk(x, hi, lo);
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        split_pair(v[8 * t + 2 * e] * hv[2 * e] * scale, v[8 * t + 2 * e + 1] * hv[2 * e + 1] * scale, hi[e], lo[e]);
       const uint32_t off = sw128_offset((uint32_t)row, (uint32_t)j);
       st_shared16(a_hi + off, hi[0], hi[1], hi[2], hi[3]);
       st_shared16(a_lo + off, lo[0], lo[1], lo[2], lo[3]);
     }
   }
-  // B rows = components; chunk oc holds reduction elements y0 + 8 oc .. +7 (exact in fp16)
+  // B rows = components: chunk oc holds reduction elements y0 + 8 oc .. +7, copied from the fp16 factor
   for (int id = tid; id < p.wpad * 8; id += kProducers) {
     const int a = id >> 3, oc = id & 7;
     const int y = y0 + 8 * oc;
-    unsigned long long raw8 = 0;
+    uint4 raw = make_uint4(0u, 0u, 0u, 0u);
     if (a < p.w && y < yend) {
-      raw8 = *reinterpret_cast<const unsigned long long*>(p.T + (long long)a * p.ldt + y);
+      raw = *reinterpret_cast<const uint4*>(p.T + (long long)a * p.ldt + y);
       const int valid = yend - y;
-      if (valid < 8) raw8 &= (1ull << (8 * valid)) - 1ull;
-    }
-    uint32_t hb[4];
+      if (valid < 8) {   // zero the elements of the next split
+        uint32_t* wv = reinterpret_cast<uint32_t*>(&raw);
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float t0 = (float)(int8_t)((raw8 >> (16 * e)) & 0xff);
-      const float t1 = (float)(int8_t)((raw8 >> (16 * e + 8)) & 0xff);
-      hb[e] = pack_half2(t0, t1);
+        for (int e = 0; e < 4; ++e) {
+          if (2 * e >= valid) wv[e] = 0u;
+          else if (2 * e + 1 >= valid) wv[e] &= 0xffffu;
+        }
+      }
     }
-    st_shared16(bt + sw128_offset((uint32_t)a, (uint32_t)oc), hb[0], hb[1], hb[2], hb[3]);
+    st_shared16(bt + sw128_offset((uint32_t)a, (uint32_t)oc), raw.x, raw.y, raw.z, raw.w);
   }
   fence_async_shared();
   mbar_arrive(bars + 8u * s);
@@ -207,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1) product_tc_kernel(const TcArgs p)
     mbar_init(done_bar, 1);
     fence_barrier_init();
   }
-  if (warp == 8) {
+  if (warp == kProducerWarps) {
     tmem_alloc(tmem_slot, p.tmem_cols);
     tmem_relinquish();
   }
@@ -217,10 +215,10 @@ __global__ void __launch_bounds__(kThreads, 1) product_tc_kernel(const TcArgs p)
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(gbase + (tmem_slot - sbase));
 
   bool ok = true;
-  if (warp < 8) {
+  if (warp < kProducerWarps) {
     // ------------------------------------------------------------------ converters
     // Loads run one stage ahead of the conversion (two rotating register buffers).
-    float b0[32], b1[32];
+    float b0[16], b1[16];
     if (nk > 0) load_stage<USTEP>(p, 0, ybeg, yend, x0, warp, lane, vec, b0);
     for (int k = 0; k < nk && ok; k += 2) {
       if (k + 1 < nk) load_stage<USTEP>(p, k + 1, ybeg, yend, x0, warp, lane, vec, b1);
@@ -251,17 +249,17 @@ __global__ void __launch_bounds__(kThreads, 1) product_tc_kernel(const TcArgs p)
     mma_commit(done_bar);                 // every MMA of this CTA has completed
   }
 
-  // ------------------------------------------------------------------ epilogue (warps 0-7)
+  // ------------------------------------------------------------------ epilogue (converter warps)
   const int all_ok = __syncthreads_and(ok ? 1 : 0);
-  if (warp < 8) {
+  if (warp < kProducerWarps) {
     bool have = nk > 0 && all_ok;
     const bool waited = mbar_wait(done_bar, 0u, p.err);
     have = __all_sync(0xffffffffu, have && waited);
     tc_fence_after();
-    const int quad = warp & 3, half = warp >> 2;
+    const int quad = warp & 3, group = warp >> 2;   // 4 warps per TMEM lane quadrant
     const int xi = x0 + quad * 32 + lane;
     float* out = p.part + (long long)blockIdx.z * p.w * Lx;
-    for (int ch = half; ch < p.wpad / 16; ch += 2) {
+    for (int ch = group; ch < p.wpad / 16; ch += kProducerWarps / 4) {
       uint32_t v[16];
       if (have) {
         tmem_ld16(tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(ch * 16), v);
@@ -281,7 +279,7 @@ __global__ void __launch_bounds__(kThreads, 1) product_tc_kernel(const TcArgs p)
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 8) {
+  if (warp == kProducerWarps) {
     tc_fence_after();
     tmem_dealloc(tmem, p.tmem_cols);
   }
@@ -313,7 +311,7 @@ TcPlan tc_plan(int w, int Lx, int Ly) {
 }
 
 template <bool USTEP>
-cudaError_t launch_tc(const float* R, int m, int n, const int8_t* T, int ldt, int w, const float* h, float* part,
+cudaError_t launch_tc(const float* R, int m, int n, const __half* T, int ldt, int w, const float* h, float* part,
                       int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
   const int Lx = USTEP ? m : n, Ly = USTEP ? n : m;
   TcPlan t = tc_plan(w, Lx, Ly);
@@ -335,12 +333,12 @@ cudaError_t launch_tc(const float* R, int m, int n, const int8_t* T, int ldt, in
 
 int tc_product_splits(int w, int Lx, int Ly) { return tc_plan(w, Lx, Ly).splits; }
 
-cudaError_t launch_product_v_tc(const float* R, int m, int n, const int8_t* Ut, int ldu, int w, float* part,
+cudaError_t launch_product_v_tc(const float* R, int m, int n, const __half* Ut, int ldu, int w, float* part,
                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
   return launch_tc<false>(R, m, n, Ut, ldu, w, nullptr, part, splits, maxabs, err, s);
 }
 
-cudaError_t launch_product_u_tc(const float* R, int m, int n, const int8_t* Vt, int ldv, int w, const float* h,
+cudaError_t launch_product_u_tc(const float* R, int m, int n, const __half* Vt, int ldv, int w, const float* h,
                                 float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
   return launch_tc<true>(R, m, n, Vt, ldv, w, h, part, splits, maxabs, err, s);
 }

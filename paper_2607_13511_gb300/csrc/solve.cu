@@ -283,19 +283,43 @@ __global__ void __launch_bounds__(NWARP * 32) sweep_kernel(const float* __restri
   }
 }
 
-__global__ void __launch_bounds__(256) rvec_kernel(const int8_t* __restrict__ Ut, int ldu, int w, int L,
+// r_a = sum_y u_a[y] (sum_s part[s][a][y]): one CTA per component; each thread takes 4 positions at a time
+// and sums their split partials in split order with a batch of loads in flight.
+__global__ void __launch_bounds__(512) rvec_kernel(const int8_t* __restrict__ Ut, int ldu, int w, int L,
                                                    const float* __restrict__ part, int splits,
                                                    float* __restrict__ r) {
-  __shared__ F2 red[8];
+  constexpr int NT = 512, PY = 4, SB = 8;
+  __shared__ F2 red[NT / 32];
   const int a = blockIdx.x;
-  // sum_y u_y p_y over the splits: one pass per split (independent loads), in split order
+  const int8_t* u = Ut + (long long)a * ldu;
+  const long long sstride = (long long)w * L;
+  const float* P = part + (long long)a * L;
   float acc = 0.f;
-  for (int sp = 0; sp < splits; ++sp) {
-    const float* P = part + ((long long)sp * w + a) * L;
-    for (int y = threadIdx.x; y < L; y += 256) {
-      const int8_t u = Ut[(long long)a * ldu + y];
-      acc += (u > 0) ? P[y] : ((u < 0) ? -P[y] : 0.f);
+  for (int y0 = 0; y0 < L; y0 += NT * PY) {
+    float p[PY];
+    int uv[PY];
+#pragma unroll
+    for (int j = 0; j < PY; ++j) {
+      const int y = y0 + j * NT + threadIdx.x;
+      p[j] = 0.f;
+      uv[j] = y < L ? (int)u[y] : 0;
     }
+    for (int s0 = 0; s0 < splits; s0 += SB) {
+      float v[SB][PY];
+#pragma unroll
+      for (int q = 0; q < SB; ++q)
+#pragma unroll
+        for (int j = 0; j < PY; ++j) {
+          const int y = y0 + j * NT + threadIdx.x;
+          v[q][j] = (s0 + q < splits && y < L) ? P[(s0 + q) * sstride + y] : 0.f;
+        }
+#pragma unroll
+      for (int q = 0; q < SB; ++q)
+#pragma unroll
+        for (int j = 0; j < PY; ++j) p[j] += v[q][j];
+    }
+#pragma unroll
+    for (int j = 0; j < PY; ++j) acc += uv[j] > 0 ? p[j] : (uv[j] < 0 ? -p[j] : 0.f);
   }
   F2 v;
   v.hi = acc;
@@ -304,7 +328,7 @@ __global__ void __launch_bounds__(256) rvec_kernel(const int8_t* __restrict__ Ut
   __syncthreads();
   if (threadIdx.x == 0) {
     F2 s;
-    for (int q = 0; q < 8; ++q) s = f2_add(s, red[q]);
+    for (int q = 0; q < NT / 32; ++q) s = f2_add(s, red[q]);
     r[a] = s.hi + s.lo;
   }
 }
@@ -312,17 +336,22 @@ __global__ void __launch_bounds__(256) rvec_kernel(const int8_t* __restrict__ Ut
 // Wide-block sweep for w <= 128: NB pivots per step. 512 threads; thread (ty, tx) in a 16 x 32 grid owns
 // the RPT = W_PAD/16 rows ty*RPT + a and the CPT = W_PAD/32 columns tx + 32c in registers. Per step K:
 //   1. the owners of rows K publish them (Rk = S[K,:], shared memory)                        barrier
-//   2. warp 0 inverts the NB x NB pivot block: lane l keeps column l of P in registers; the
-//      pivot column is broadcast with shuffles (by symmetry it is also the pivot row)      barrier
-//   3. T = S[:,K] Q for every row (S[i,K] = Rk[.,i]), one row per thread group            barrier
-//   4. rank-NB update of the register tiles from T and Rk, fixing up rows and columns of K  barrier
-// The serial part is NB pivots of one warp per step; everything else is dense float32 FMA.
-template <int W_PAD, int NB, int MODE>
+//   2. warp 0 inverts the NB x NB pivot block P: Q = P^-1 (lane l keeps column l in registers; the pivot
+//      column is broadcast with shuffles, by symmetry it is also the pivot row)                barrier
+//   3. T'[i,:] = S[i,K] Q for rows outside K and -Q[i,:] for rows in K                        barrier
+//   4. one uniform rank-NB update S <- D S - T' Rk, D zeroing the rows of K: outside K this is the Schur
+//      complement S - S[I,K] Q S[K,J], on the rows of K it gives Q S[K,J]; then the columns of K take T'
+//      (S[I,K] Q, and -Q on the pivot block)                                                   barrier
+// The serial part is NB pivots of one warp per step; everything else is the same dense float32 FMA work on
+// every thread. After the last step S = -(G + eps I)^-1.
+// IN_INT: the Gram comes as an integer upper triangle Gint[a * w + b] (a <= b), reset to zero after reading;
+// each thread reads its upper-triangle entries and the lower ones come back mirrored through shared memory.
+template <int W_PAD, int NB, int MODE, bool IN_INT>
 __global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ Gpart, int splits, int w,
                                                       const float* __restrict__ GVraw, const float* __restrict__ r,
-                                                      float* __restrict__ Graw, float* __restrict__ out) {
+                                                      float* __restrict__ Graw, float* __restrict__ out, int* Gint) {
   constexpr int RPT = W_PAD / 16, CPT = W_PAD / 32;
-  static_assert(W_PAD % NB == 0 && RPT >= 1 && CPT >= 1, "bad shape");
+  static_assert(W_PAD % NB == 0 && 32 % NB == 0 && RPT >= 1 && CPT >= 1, "bad shape");
   __shared__ __align__(16) float Rk[NB][W_PAD + 1];
   __shared__ __align__(16) float T[W_PAD][NB + 1];
   __shared__ float Qs[NB][NB + 1];
@@ -335,16 +364,42 @@ __global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ 
   for (int a = 0; a < RPT; ++a)
 #pragma unroll
     for (int c = 0; c < CPT; ++c) S[a][c] = 0.f;
-  for (int sp = 0; sp < splits; ++sp) {
-    const float* G = Gpart + (long long)sp * w * w;
+  if (IN_INT) {
+    extern __shared__ float mirror[];   // [W_PAD][W_PAD + 1]: mirror[j][i] = G[i][j] for i < j
 #pragma unroll
     for (int a = 0; a < RPT; ++a) {
       const int i = i0 + a;
-      if (i >= w) continue;
 #pragma unroll
       for (int c = 0; c < CPT; ++c) {
         const int j = tx + 32 * c;
-        if (j < w) S[a][c] += G[(long long)i * w + j];
+        if (i <= j && j < w) {
+          S[a][c] = (float)Gint[(long long)i * w + j];
+          mirror[j * (W_PAD + 1) + i] = S[a][c];
+        }
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int a = 0; a < RPT; ++a) {
+      const int i = i0 + a;
+#pragma unroll
+      for (int c = 0; c < CPT; ++c) {
+        const int j = tx + 32 * c;
+        if (j < i && i < w) S[a][c] = mirror[i * (W_PAD + 1) + j];
+      }
+    }
+  } else {
+    for (int sp = 0; sp < splits; ++sp) {
+      const float* G = Gpart + (long long)sp * w * w;
+#pragma unroll
+      for (int a = 0; a < RPT; ++a) {
+        const int i = i0 + a;
+        if (i >= w) continue;
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) {
+          const int j = tx + 32 * c;
+          if (j < w) S[a][c] += G[(long long)i * w + j];
+        }
       }
     }
   }
@@ -418,21 +473,26 @@ __global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ 
       }
     }
     __syncthreads();
-    // 3. T[i][b] = sum_c S[i][k0 + c] Q[c][b] = sum_c Rk[c][i] Q[c][b]  (thread: row i = tid / 4, b = 8 of them)
+    // 3. T'[i][b] = sum_c S[i][k0 + c] Q[c][b] = sum_c Rk[c][i] Q[c][b] outside K, -Q[i - k0][b] on K
     for (int idx = tid; idx < W_PAD * (NB / 8); idx += 512) {
       const int i = idx / (NB / 8), bq = (idx % (NB / 8)) * 8;
       float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      if (i >= k0 && i < k0 + NB) {
 #pragma unroll
-      for (int c = 0; c < NB; ++c) {
-        const float rv = Rk[c][i];
+        for (int u = 0; u < 8; ++u) acc[u] = -Qs[i - k0][bq + u];
+      } else {
 #pragma unroll
-        for (int u = 0; u < 8; ++u) acc[u] = fmaf(rv, Qs[c][bq + u], acc[u]);
+        for (int c = 0; c < NB; ++c) {
+          const float rv = Rk[c][i];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) acc[u] = fmaf(rv, Qs[c][bq + u], acc[u]);
+        }
       }
 #pragma unroll
       for (int u = 0; u < 8; ++u) T[i][bq + u] = acc[u];
     }
     __syncthreads();
-    // 4. rank-NB update of the register tiles
+    // 4. S <- D S - T' Rk, then the columns of K (all in register column cK: NB divides 32) take T'
     float acc[RPT][CPT];
 #pragma unroll
     for (int a = 0; a < RPT; ++a)
@@ -450,25 +510,20 @@ __global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ 
 #pragma unroll
         for (int c = 0; c < CPT; ++c) acc[a][c] = fmaf(tv[a], rv[c], acc[a][c]);
     }
+    const int cK = k0 >> 5;
+    const int jk = tx + 32 * cK - k0;                 // this lane's column within K, when in [0, NB)
+    const bool lane_in = jk >= 0 && jk < NB;
+    const int jb = min(max(jk, 0), NB - 1);
 #pragma unroll
     for (int a = 0; a < RPT; ++a) {
       const int i = i0 + a;
-      const bool i_in = (i >= k0 && i < k0 + NB);
+      const bool i_in = (i >= k0 && i < k0 + NB);   // uniform across the warp
 #pragma unroll
       for (int c = 0; c < CPT; ++c) {
-        const int j = tx + 32 * c;
-        const bool j_in = (j >= k0 && j < k0 + NB);
-        float v;
-        if (!i_in && !j_in) v = S[a][c] - acc[a][c];                 // S - S[I,K] Q S[K,J]
-        else if (!i_in) v = T[i][j - k0];                            // S[I,K] Q
-        else if (!j_in) {                                            // Q S[K,J] = T^T restricted: sum_b Q[ia][b] Rk[b][j]
-          const int ia = i - k0;
-          float q = 0.f;
-#pragma unroll 8
-          for (int b = 0; b < NB; ++b) q = fmaf(Qs[ia][b], Rk[b][j], q);
-          v = q;
-        } else {
-          v = -Qs[i - k0][j - k0];
+        float v = (i_in ? 0.f : S[a][c]) - acc[a][c];
+        if (c == cK) {
+          const float tk = T[i][jb];
+          v = lane_in ? tk : v;
         }
         S[a][c] = v;
       }
@@ -500,6 +555,14 @@ __global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ 
       acc2 = warp_sum(acc2);
       if (lane == 0 && i < w) out[i] = acc2.hi + acc2.lo;
     }
+  }  if (IN_INT) {   // every thread has read its entries (barrier after the last step): reset the upper triangle
+#pragma unroll
+    for (int a = 0; a < RPT; ++a)
+#pragma unroll
+      for (int c = 0; c < CPT; ++c) {
+        const int i = i0 + a, j = tx + 32 * c;
+        if (i <= j && j < w) Gint[(long long)i * w + j] = 0;
+      }
   }
 }
 
@@ -513,14 +576,38 @@ int gram_chunk(int w, int L, int* splits) {
   return chunk;
 }
 
+template <int W_PAD, int NB, int MODE>
+cudaError_t launch_sweep_int_w(int* Gint, int w, const float* GVraw, const float* r, float* Graw, float* out,
+                               cudaStream_t s) {
+  const size_t smem = (size_t)W_PAD * (W_PAD + 1) * sizeof(float);   // the lower-triangle mirror
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(sweep32_kernel<W_PAD, NB, MODE, true>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  sweep32_kernel<W_PAD, NB, MODE, true><<<1, 512, smem, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint);
+  return cudaGetLastError();
+}
+
+template <int MODE>
+cudaError_t launch_sweep_int(int* Gint, int w, const float* GVraw, const float* r, float* Graw, float* out,
+                             cudaStream_t s) {
+  if (w <= 32) return launch_sweep_int_w<32, 8, MODE>(Gint, w, GVraw, r, Graw, out, s);
+  if (w <= 64) return launch_sweep_int_w<64, 8, MODE>(Gint, w, GVraw, r, Graw, out, s);
+  if (w <= 128) return launch_sweep_int_w<128, 16, MODE>(Gint, w, GVraw, r, Graw, out, s);
+  return cudaErrorInvalidValue;   // callers use the float-partial Gram above 128 components
+}
+
 template <int MODE>
 cudaError_t launch_sweep(const float* Gpart, int splits, int w, const float* GVraw, const float* r, float* Graw,
                          float* out, cudaStream_t s) {
   // elements per lane RPW * CPL = W_PAD^2 / (32 * NWARP): 4 / 8 / 32 / 64
   // pivot-block sizes measured fastest on GB300: 8 up to w = 64, 16 at w = 128
-  if (w <= 32) sweep32_kernel<32, 8, MODE><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
-  else if (w <= 64) sweep32_kernel<64, 8, MODE><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
-  else if (w <= 128) sweep32_kernel<128, 16, MODE><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
+  if (w <= 32) sweep32_kernel<32, 8, MODE, false><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
+  else if (w <= 64) sweep32_kernel<64, 8, MODE, false><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
+  else if (w <= 128) sweep32_kernel<128, 16, MODE, false><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
   else sweep_kernel<256, 32, MODE><<<1, 32 * 32, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
   return cudaGetLastError();
 }
@@ -545,9 +632,17 @@ cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, f
   return launch_sweep<0>(Gpart, splits, w, nullptr, nullptr, Graw, Ginv, s);
 }
 
+cudaError_t launch_inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s) {
+  return launch_sweep_int<0>(Gint, w, nullptr, nullptr, Graw, Ginv, s);
+}
+
+cudaError_t launch_scales_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s) {
+  return launch_sweep_int<1>(GUint, w, GVraw, r, nullptr, d, s);
+}
+
 cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, float* r,
                         cudaStream_t s) {
-  rvec_kernel<<<(unsigned)w, 256, 0, s>>>(Ut, ldu, w, L, part, splits, r);
+  rvec_kernel<<<(unsigned)w, 512, 0, s>>>(Ut, ldu, w, L, part, splits, r);
   return cudaGetLastError();
 }
 

@@ -5,6 +5,8 @@
 // (first index) is kept. The sum is gathered as per-chunk partials (compensated float, combined in double) by
 // whichever kernel produces x, then summed in a fixed order by the apply kernel: theta = tau * (S / L) in double,
 // compared in float against RD_float(theta), which decides exactly like a double comparison for float x.
+#include <algorithm>
+
 #include "kernels.h"
 
 namespace externd {
@@ -53,74 +55,92 @@ __global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X,
     st.spart[(long long)a * st.nchunk + blockIdx.x] = t;
     st.kpart[(long long)a * st.nchunk + blockIdx.x] = k;
   }
+  stats_done(st, gridDim.y);
 }
 
-// Threshold of vector a from its chunk partials (warp 0, fixed order): RD_float(tau * S / L), fallback flag and
-// the fallback index.
-__device__ __forceinline__ void vector_threshold(const Stats& st, int a, int L, double tau, float* theta_dn,
-                                                 int* fallback, uint32_t* argidx) {
-  const int lane = threadIdx.x & 31;
-  F2 s;
-  u64 key = 0;
-  for (int c = lane; c < st.nchunk; c += 32) {
-    s = f2_add(s, st.spart[(long long)a * st.nchunk + c]);
-    const u64 k = st.kpart[(long long)a * st.nchunk + c];
-    key = k > key ? k : key;
+// T = T_tau(X) for up to 256 vectors per CTA over positions [x0, x0 + P), in 64-position chunks. Each warp
+// ternarizes 32 positions of one vector at a time (coalesced reads and byte writes) and records the +1 and -1
+// positions as ballot masks; with GRAM the CTA then adds the chunk's exact Gram entries
+//   G_ab += popc(P_a & P_b) + popc(N_a & N_b) - popc(P_a & N_b) - popc(N_a & P_b)
+// into per-thread integer accumulators (thread: vector a = tid % VB, VB*VB/256 consecutive b), and finally
+// atomically adds the upper triangle to gram. Integer sums are exact, so the order of the atomics does not matter.
+template <int VB, bool GRAM>
+__global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X, int nv, int L, long long ldx,
+                                                    Thresh th, int8_t* __restrict__ T, long long ldt,
+                                                    int* __restrict__ gram, int P, __half* __restrict__ T16,
+                                                    long long ldt16) {
+  constexpr int PPT = (VB * VB) / 256 > 0 ? (VB * VB) / 256 : 1;   // Gram pairs per thread
+  constexpr int IT = VB / 4;                                      // warp passes per 64-position chunk
+  __shared__ unsigned mpos[VB][2], mneg[VB][2];
+  __shared__ float s_theta[VB];
+  __shared__ unsigned s_arg[VB];   // fallback position, or ~0u when some entry passes the threshold
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int v0 = blockIdx.y * VB;
+  const int nvb = min(VB, nv - v0);
+  const int xbeg = blockIdx.x * P, xend = min(L, xbeg + P);
+  const int ga = tid % VB, gb0 = (tid / VB) * PPT;
+  for (int a = tid; a < nvb; a += 256) {
+    s_theta[a] = th.theta[v0 + a];
+    s_arg[a] = th.fallback[v0 + a] ? th.arg[v0 + a] : 0xffffffffu;
   }
-  s = warp_sum(s);
-  key = warp_max(key);
-  // theta = tau * (S / L) in double, by one lane (double arithmetic is slow here; keep it to one thread)
-  float th = 0.f;
-  if (lane == 0) th = __double2float_rd(tau * (f2_value(s) / (double)L));
-  th = __shfl_sync(0xffffffffu, th, 0);
-  *theta_dn = th;
-  *fallback = !(key_mag(key) > th);
-  *argidx = key_index(key);
-}
-
-__global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X, int L, long long ldx, Stats st,
-                                                    double tau, int8_t* __restrict__ T, long long ldt) {
-  __shared__ float s_theta;
-  __shared__ int s_fallback;
-  __shared__ uint32_t s_arg;
-  const int a = blockIdx.y;
-  if (threadIdx.x < 32) {
-    float th;
-    int fb;
-    uint32_t ai;
-    vector_threshold(st, a, L, tau, &th, &fb, &ai);
-    if (threadIdx.x == 0) {
-      s_theta = th;
-      s_fallback = fb;
-      s_arg = ai;
-    }
-  }
+  int acc[PPT];
+#pragma unroll
+  for (int k = 0; k < PPT; ++k) acc[k] = 0;
   __syncthreads();
-  const float th = s_theta;
-  const int fb = s_fallback;
-  const uint32_t ai = s_arg;
-  const int x0 = (blockIdx.x * 256 + threadIdx.x) * 4;
-  if (x0 >= L) return;
-  const float* src = X + (long long)a * ldx;
-  int8_t t[4];
+  for (int x0 = xbeg; x0 < xend; x0 += 64) {
+    // pass i of warp covers vector a = (warp + 8i) / 2, positions x0 + 32 * ((warp + 8i) % 2) + lane; the
+    // loads of a batch of passes are all issued before the first is used
+    constexpr int IB = IT < 16 ? IT : 16;
+#pragma unroll 1
+    for (int i0 = 0; i0 < IT; i0 += IB) {
+      float xv[IB];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const int x = x0 + j;
-    t[j] = 0;
-    if (x < L) {
-      const float v = src[x];
-      t[j] = ternary_of(v, th);
-      if (fb && (uint32_t)x == ai) t[j] = v < 0.f ? (int8_t)-1 : (int8_t)1;
+      for (int i = 0; i < IB; ++i) {
+        const int u = warp + 8 * (i0 + i), a = u >> 1;
+        const int x = x0 + 32 * (u & 1) + lane;
+        xv[i] = (a < nvb && x < xend) ? X[(long long)(v0 + a) * ldx + x] : 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < IB; ++i) {
+        const int u = warp + 8 * (i0 + i), a = u >> 1, half = u & 1;
+        const int x = x0 + 32 * half + lane;
+        int8_t t = 0;
+        if (a < nvb && x < xend) {
+          const int v = v0 + a;
+          t = ternary_of(xv[i], s_theta[a]);
+          if ((uint32_t)x == s_arg[a]) t = xv[i] < 0.f ? (int8_t)-1 : (int8_t)1;
+          T[(long long)v * ldt + x] = t;
+          if (T16 != nullptr) T16[(long long)v * ldt16 + x] = __short2half_rn((short)t);
+        }
+        if (GRAM) {
+          const unsigned pm = __ballot_sync(0xffffffffu, t > 0), nm = __ballot_sync(0xffffffffu, t < 0);
+          if (lane == 0) {
+            mpos[a][half] = pm;
+            mneg[a][half] = nm;
+          }
+        }
+      }
+    }
+    if (GRAM) {
+      __syncthreads();
+      const unsigned long long pa = mpos[ga][0] | ((unsigned long long)mpos[ga][1] << 32);
+      const unsigned long long na = mneg[ga][0] | ((unsigned long long)mneg[ga][1] << 32);
+#pragma unroll
+      for (int k = 0; k < PPT; ++k) {
+        const int b = gb0 + k;
+        const unsigned long long pb = mpos[b][0] | ((unsigned long long)mpos[b][1] << 32);
+        const unsigned long long nb = mneg[b][0] | ((unsigned long long)mneg[b][1] << 32);
+        acc[k] += __popcll(pa & pb) + __popcll(na & nb) - __popcll(pa & nb) - __popcll(na & pb);
+      }
+      __syncthreads();
     }
   }
-  int8_t* dst = T + (long long)a * ldt + x0;
-  if ((ldt & 3) == 0 && x0 + 3 < L) {
-    *reinterpret_cast<int*>(dst) = (int)(uint8_t)t[0] | ((int)(uint8_t)t[1] << 8) | ((int)(uint8_t)t[2] << 16) |
-                                   ((int)(uint8_t)t[3] << 24);
-  } else {
+  if (GRAM) {
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
-      if (x0 + j < L) dst[j] = t[j];
+    for (int k = 0; k < PPT; ++k) {
+      const int b = gb0 + k;
+      if (ga < nvb && b < nvb && ga <= b && acc[k] != 0) atomicAdd(&gram[(long long)ga * nv + b], acc[k]);
+    }
   }
 }
 
@@ -342,10 +362,42 @@ cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, flo
   return cudaGetLastError();
 }
 
-cudaError_t launch_apply(const float* X, int nv, int L, int ldx, Stats st, double tau, int8_t* T, int ldt,
-                         cudaStream_t s) {
-  dim3 grid((unsigned)cdiv(L, 1024), (unsigned)nv);
-  apply_kernel<<<grid, 256, 0, s>>>(X, L, ldx, st, tau, T, ldt);
+cudaError_t launch_apply(const float* X, int nv, int L, int ldx, const Thresh& th, int8_t* T, int ldt, int* gram,
+                         cudaStream_t s, __half* T16, long long ldt16) {
+  // about 64 CTAs along the vectors' length, in whole 64-position chunks
+  const int P = 64 * (int)std::max<long long>(1, cdiv(L, 64 * 64));
+  const int gx = (int)cdiv(L, P);
+  const bool g = gram != nullptr && nv <= 128;   // 256 vectors would need 256 accumulators per thread
+#define APPLY_LAUNCH(VB)                                                                                 \
+  do {                                                                                                   \
+    dim3 grid((unsigned)gx, (unsigned)cdiv(nv, VB));                                                     \
+    if (g) apply_kernel<VB, true><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, gram, P, T16, ldt16);  \
+    else apply_kernel<VB, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16); \
+  } while (0)
+  if (nv <= 16) APPLY_LAUNCH(16);
+  else if (nv <= 32) APPLY_LAUNCH(32);
+  else if (nv <= 64) APPLY_LAUNCH(64);
+  else if (nv <= 128) APPLY_LAUNCH(128);
+  else {
+    dim3 grid((unsigned)gx, (unsigned)cdiv(nv, 256));
+    apply_kernel<256, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16);
+  }
+#undef APPLY_LAUNCH
+  return cudaGetLastError();
+}
+
+__global__ void i8_to_f16_kernel(const int8_t* __restrict__ src, long long lds, int rows, int cols,
+                                 __half* __restrict__ dst, long long ldd) {
+  const int r = blockIdx.y;
+  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < cols; c += gridDim.x * blockDim.x)
+    dst[(long long)r * ldd + c] = __short2half_rn((short)src[(long long)r * lds + c]);
+}
+
+cudaError_t launch_i8_to_f16(const int8_t* src, long long lds, int rows, int cols, __half* dst, long long ldd,
+                             cudaStream_t s) {
+  if (rows < 1 || cols < 1) return cudaSuccess;
+  dim3 grid((unsigned)std::min<long long>(64, cdiv(cols, 256)), (unsigned)rows);
+  i8_to_f16_kernel<<<grid, 256, 0, s>>>(src, lds, rows, cols, dst, ldd);
   return cudaGetLastError();
 }
 
