@@ -223,10 +223,12 @@ struct Bufs {
   int *fallback, *GintU, *GintV;
   int8_t *Ut, *Vt;
   __half *Ut16, *Vt16;   // fp16 copies of Ut, Vt for the tensor-core products (nullptr when unused)
-  F2 *spart, *normpart;
+  __half *Uk16, *Vk16;   // K-major fp16 copies of the final U, V of a block for the tensor-core deflation
+  long long ldk;
+  StatPart* spart;
+  F2* normpart;
   float* r;
   double *norm_a, *norm_r, *trace;
-  u64* kpart;
   int* J;
 };
 
@@ -236,10 +238,13 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "R", (size_t)p.m * p.n, &B->R));
   TRY(need(ws, "Ut", (size_t)w * p.ldm, &B->Ut, true));
   TRY(need(ws, "Vt", (size_t)w * p.ldn, &B->Vt, true));
-  B->Ut16 = B->Vt16 = nullptr;
+  B->Ut16 = B->Vt16 = B->Uk16 = B->Vk16 = nullptr;
+  B->ldk = round_up(w, 16);
   if (use_tc(p.b)) {
     TRY(need(ws, "Ut16", (size_t)w * p.ldm, &B->Ut16, true));
     TRY(need(ws, "Vt16", (size_t)w * p.ldn, &B->Vt16, true));
+    TRY(need(ws, "Uk16", (size_t)p.m * B->ldk, &B->Uk16, true));
+    TRY(need(ws, "Vk16", (size_t)p.n * B->ldk, &B->Vk16, true));
   }
   // split-K partials for both block widths that occur (b and the tail k mod b)
   size_t part = 0;
@@ -260,7 +265,6 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "GintV", (size_t)w * w, &B->GintV, true));
   TRY(need(ws, "X", (size_t)w * L, &B->X));
   TRY(need(ws, "spart", (size_t)w * std::max(p.nchunk_m, p.nchunk_n), &B->spart));
-  TRY(need(ws, "kpart", (size_t)w * std::max(p.nchunk_m, p.nchunk_n), &B->kpart));
   TRY(need(ws, "Gpart", (size_t)std::max(p.gm, p.gn) * w * w, &B->Gpart));
   TRY(need(ws, "GrawU", (size_t)w * w, &B->GrawU));
   TRY(need(ws, "GrawV", (size_t)w * w, &B->GrawV));
@@ -288,8 +292,8 @@ Plan make_plan(long long m, long long n, long long k, int block, int iters, doub
   p.nblocks = (int)cdiv(k, p.b);
   p.gm = gram_splits(p.b, p.m);
   p.gn = gram_splits(p.b, p.n);
-  p.nchunk_m = std::max((int)cdiv(p.m, kStatChunk), decorrelate_chunks(p.m));
-  p.nchunk_n = std::max((int)cdiv(p.n, kStatChunk), decorrelate_chunks(p.n));
+  p.nchunk_m = (int)cdiv(p.m, 16);   // bounds every producer's chunk count (decorrelation tiles >= 16)
+  p.nchunk_n = (int)cdiv(p.n, 16);
   p.ldm = ld16(m);
   p.ldn = ld16(n);
   return p;
@@ -336,9 +340,9 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
   // thresholds the apply reads
   const Thresh th_m{B.theta, B.fallback, B.arg, B.ticket, p.tau, m};
   const Thresh th_n{B.theta, B.fallback, B.arg, B.ticket, p.tau, n};
-  const Stats st_g{B.spart, B.kpart, (int)cdiv(m, kStatChunk), th_m};   // gather (block start)
-  const Stats st_m{B.spart, B.kpart, decorrelate_chunks(m), th_m};       // U-step decorrelation
-  const Stats st_n{B.spart, B.kpart, decorrelate_chunks(n), th_n};       // V-step decorrelation
+  const Stats st_g{B.spart, (int)cdiv(m, kStatChunk), th_m};   // gather (block start)
+  Stats st_m{B.spart, 0, th_m};       // U-step decorrelation (chunk count set per block width)
+  Stats st_n{B.spart, 0, th_n};       // V-step decorrelation
   const int nrt = deflate_row_tiles(m), ntiles = deflate_tiles(m, n);
   g_prof.used = 0;
   g_prof.launches = 0;
@@ -351,6 +355,8 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
     const long long j0 = (long long)blk * p.b;
     const int w = (int)std::min<long long>(p.b, p.k - j0);
     const int sv = splits_v(w, m, n), su = splits_u(w, m, n);
+    st_m.nchunk = decorrelate_chunks(m, w);
+    st_n.nchunk = decorrelate_chunks(n, w);
     // Exact Gram matrices of unweighted ternary factors are accumulated by the apply that writes the factor
     // (integer atomics) up to 128 components; wider blocks and the weighted V^T H V use the Gram kernel.
     const bool fusedU = w <= 128, fusedV = w <= 128 && h == nullptr;
@@ -376,7 +382,8 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
       KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
       if (w > 1) JOIN();
       KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, sv, n, B.X, n, st_n, s));
-      KL(kApply, 1, launch_apply(B.X, w, n, n, th_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, s, V16, p.ldn));
+      KL(kApply, 1, launch_apply(B.X, w, n, n, th_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, s, V16, p.ldn,
+                                 (last && use_tc(w)) ? B.Vk16 : nullptr, B.ldk));
       // U-step: U <- T(R H V (V^T H V + eps I)^-1)
       FORK();
       if (fusedV) {
@@ -391,7 +398,7 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
       // the next V-step's inverse (w > 1) or, after the last iteration, Eq. 4 consumes U's Gram
       // (the fp16 copy of U is not needed after the last iteration)
       KL(kApply, 1, launch_apply(B.X, w, m, m, th_m, B.Ut, (int)p.ldm, (fusedU && (w > 1 || last)) ? B.GintU : nullptr,
-                                 s, last ? nullptr : U16, p.ldm));
+                                 s, last ? nullptr : U16, p.ldm, (last && use_tc(w)) ? B.Uk16 : nullptr, B.ldk));
     }
     // Eq. 4: [(U^T U) .* (V^T H V)] d = diag(U^T R H V), with R H V the last U-step product
     KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, su, B.r, s));
@@ -402,8 +409,13 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
       KL(kSolve, 1, launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s));
     }
     // R <- R - U diag(d) V^T
-    KL(kDeflate, 1, launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart, B.normpart,
-                                   s, B.maxpart));
+    if (use_tc(w)) {
+      KL(kDeflate, 1, launch_deflate_tc(B.R, m, n, B.Uk16, B.Vk16, B.ldk, B.d, w, h, B.colpart, B.normpart, B.maxpart,
+                                        B.err, s));
+    } else {
+      KL(kDeflate, 1, launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart,
+                                     B.normpart, s, B.maxpart));
+    }
     KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_r, B.norm_a, B.trace + blk, s, B.maxpart, B.maxabs));
     KL(0, 1, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, s));
     LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
@@ -723,19 +735,17 @@ int externd_ternarize(const float* X, int64_t rows, int64_t cols, int axis, doub
   const long long nv = axis == 1 ? rows : cols, L = axis == 1 ? cols : rows;
   if (nv > 65535) return EXTERND_EINVAL;   // one grid row per vector
   const int nchunk = (int)cdiv(L, kStatChunk);
-  F2* sp;
-  u64* kp;
+  StatPart* sp;
   float* theta;
   int* fb;
   unsigned *arg, *ticket;
   TRY(need(*ws, "tern.spart", (size_t)nv * nchunk, &sp));
-  TRY(need(*ws, "tern.kpart", (size_t)nv * nchunk, &kp));
   TRY(need(*ws, "tern.theta", (size_t)nv, &theta));
   TRY(need(*ws, "tern.fallback", (size_t)nv, &fb));
   TRY(need(*ws, "tern.arg", (size_t)nv, &arg));
   TRY(need(*ws, "ticket", 1, &ticket, true));
   const Thresh th{theta, fb, arg, ticket, tau, (int)L};
-  Stats st{sp, kp, nchunk, th};
+  Stats st{sp, nchunk, th};
   if (axis == 1) {
     LK(launch_stats(X, (int)nv, (int)L, (int)L, st, g_stream));
     LK(launch_apply(X, (int)nv, (int)L, L, th, T, (int)L, nullptr, g_stream));
@@ -808,12 +818,11 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   Workspace* ws;
   TRY(current_ws(&ws));
   const long long L = vstep ? n : m;
-  const int nchunk = decorrelate_chunks((int)L);
+  const int nchunk = decorrelate_chunks((int)L, w);
   int8_t* T;
   __half* T16;
   float *part, *X, *Gpart, *Graw, *Ginv, *one;
-  F2* sp;
-  u64* kp;
+  StatPart* sp;
   if (vstep) TRY(stage_u(*ws, F, m, w, &T, &T16));
   else TRY(stage_v(*ws, F, n, w, &T, &T16));
   const long long ldt = vstep ? ld16(m) : ld16(n);
@@ -829,7 +838,6 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   TRY(need(*ws, "GrawV", (size_t)w * w, &Graw));
   TRY(need(*ws, "Ginv", (size_t)w * w, &Ginv));
   TRY(need(*ws, "spart", (size_t)w * nchunk, &sp));
-  TRY(need(*ws, "kpart", (size_t)w * nchunk, &kp));
   TRY(get_one(*ws, &one));
   if (vstep) LK(product_v(R, (int)m, (int)n, T, T16, (int)ldt, w, part, splits, mx, err, g_stream));
   else LK(product_u(R, (int)m, (int)n, T, T16, (int)ldt, w, h, part, splits, mx, err, g_stream));
@@ -844,7 +852,7 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   TRY(need(*ws, "fallback", (size_t)w, &fb));
   TRY(need(*ws, "arg", (size_t)w, &arg));
   TRY(need(*ws, "ticket", 1, &ticket, true));
-  Stats st{sp, kp, nchunk, Thresh{theta, fb, arg, ticket, 0.0, (int)L}};
+  Stats st{sp, nchunk, Thresh{theta, fb, arg, ticket, 0.0, (int)L}};
   if (vstep) {
     LK(launch_decorrelate(w > 1 ? Ginv : one, w, part, splits, (int)L, out, (int)L, st, g_stream));
   } else {
@@ -917,17 +925,32 @@ int externd_deflate(float* R, int64_t m, int64_t n, const int8_t* U, const float
   if (weights) TRY(check_dev(weights));
   Workspace* ws;
   TRY(current_ws(&ws));
-  int8_t *Ut, *Vt;
   F2* part;
   double* sc;
-  TRY(stage_u(*ws, U, m, (int)w, &Ut));
-  TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
   const int tiles = deflate_tiles((int)m, (int)n);
   TRY(need(*ws, "energy.part", (size_t)tiles, &part));
   TRY(need(*ws, "energy.sc", 4, &sc));
-  LK(launch_deflate(R, R, (int)m, (int)n, Ut, ld16(m), false, d, Vt, ld16(n), (int)w, weights, nullptr, part,
-                    g_stream));
-  LK(launch_norm(part, tiles, sc, nullptr, nullptr, g_stream));
+  if (use_tc((int)w)) {
+    const long long ldk = round_up(w, 16);
+    __half *Uk, *Vk;
+    unsigned* err;
+    TRY(need(*ws, "step.Uk16", (size_t)m * ldk, &Uk, true));
+    TRY(need(*ws, "step.Vk16", (size_t)n * ldk, &Vk, true));
+    TRY(need(*ws, "err", 1, &err, true));
+    LK(launch_kmajor(U, 1, w, (int)w, (int)m, Uk, ldk, g_stream));    // U is m x w row-major
+    LK(launch_kmajor(Cb, n, 1, (int)w, (int)n, Vk, ldk, g_stream));   // Cb is w x n row-major
+    LK(launch_deflate_tc(R, (int)m, (int)n, Uk, Vk, ldk, d, (int)w, weights, nullptr, part, nullptr, err,
+                         g_stream));
+    LK(launch_norm(part, tiles, sc, nullptr, nullptr, g_stream));
+    TRY(check_device_error(*ws, err, g_stream));
+  } else {
+    int8_t *Ut, *Vt;
+    TRY(stage_u(*ws, U, m, (int)w, &Ut));
+    TRY(stage_v(*ws, Cb, n, (int)w, &Vt));
+    LK(launch_deflate(R, R, (int)m, (int)n, Ut, ld16(m), false, d, Vt, ld16(n), (int)w, weights, nullptr, part,
+                      g_stream));
+    LK(launch_norm(part, tiles, sc, nullptr, nullptr, g_stream));
+  }
   if (norm2 != nullptr) return read_double(*ws, sc, norm2);
   return EXTERND_OK;
 }

@@ -129,93 +129,133 @@ __global__ void __launch_bounds__(256) product_kernel(const float* __restrict__ 
   }
 }
 
-// X tile of 64 components x 32 positions: thread (ty, tx) owns components ty*4..+3 at positions tx*2, tx*2+1.
-// Narrow tiles give enough CTAs to read the split-K partials in parallel at small L. The CTA first stages, with
-// every load of a batch in flight before any is used,
+// X tile of 64 components x DXT positions (DXT = 16 ... 128, chosen per shape so that the grid fills the GPU
+// once or twice): thread (ty, tx) owns components ty*4..+3 at positions tx*PX .. +PX-1, PX = DXT / 16. The CTA
+// first stages, with every load of a batch in flight before any is used,
 //   Ps[b][x]  = sum_s part[s][b][x0 + x]   for all w components b (split order)
 //   Gs[b][a]  = Ginv[b][a0 + a]            (Ginv is symmetric: row b holds column b)
-// in dynamic shared memory, then runs the w-deep product out of shared memory.
-constexpr int DX = 32;
+// in dynamic shared memory, then runs the w-deep product out of shared memory. One Eq. 2 statistics chunk per
+// CTA column: DXT positions.
 constexpr int kGsLd = TM + 4;
 
-size_t decorrelate_smem(int w) { return (size_t)w * (DX + kGsLd) * sizeof(float); }
+size_t decorrelate_smem(int w, int dxt) { return (size_t)w * (dxt + kGsLd) * sizeof(float); }
 
-__global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restrict__ Ginv, int w,
+int decorrelate_dx(int L, int w) {
+  int sms = 152, dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int dx = 16;
+  while (dx < 128 && cdiv(L, dx) * cdiv(w, TM) > 2LL * sms) dx *= 2;
+  return dx;
+}
+
+template <int DXT>
+__global__ void __launch_bounds__(256, 2) decorrelate_kernel(const float* __restrict__ Ginv, int w,
                                                           const float* __restrict__ part, int splits, int L,
                                                           float* __restrict__ X, int ldx, Stats st) {
+  constexpr int PX = DXT / 16;
   extern __shared__ __align__(16) float dsm[];
-  float* const Ps = dsm;                 // [w][DX]
-  float* const Gs = dsm + w * DX;        // [w][kGsLd]
-  const int x0 = blockIdx.x * DX;
+  float* const Ps = dsm;                 // [w][DXT]
+  float* const Gs = dsm + w * DXT;       // [w][kGsLd]
+  const int x0 = blockIdx.x * DXT;
   const int a0 = blockIdx.y * TM;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
 
-  // Ginv rows: w x 16 float4 slots
+  // Ps: w x DXT/4 float4 slots; a thread owns slots tid + 256 e and walks its (slot, split) pairs in batches of
+  // 8 loads, adding each slot's splits in split order through shared memory. The first Ginv rows (w x 16 float4
+  // slots) are issued with the first batch. Two CTAs fit on an SM (<= 128 registers).
   {
-    const bool gvec = (w & 3) == 0;
-    for (int i0 = 0; i0 < w * 16; i0 += 4 * 256) {
-      float4 g[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int i = i0 + q * 256 + tid;
-        g[q] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (i < w * 16) g[q] = load4(Ginv + (long long)(i >> 4) * w, a0 + (i & 15) * 4, w, gvec);
-      }
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int i = i0 + q * 256 + tid;
-        if (i < w * 16) *reinterpret_cast<float4*>(&Gs[(i >> 4) * kGsLd + (i & 15) * 4]) = g[q];
-      }
-    }
-  }
-  // split sums: w x 8 float4 slots, 4 slots x 4 splits of loads in flight per thread
-  {
-    constexpr int E = 4, SB = 4;
-    const bool pvec = (L & 3) == 0;
+    constexpr int Q = DXT / 4, NB = 8;
+    const bool pvec = (L & 3) == 0, gvec = (w & 3) == 0;
     const long long sstride = (long long)w * L;
-    for (int i0 = 0; i0 < w * 8; i0 += E * 256) {
-      float4 acc[E];
+    const int nps = w * Q, pper = (nps + 255) / 256, nld = pper * splits;
+    const int ngs = w * 16, gper = (ngs + 255) / 256;
+    constexpr int GB = 4;
+    float4 g[GB];
 #pragma unroll
-      for (int e = 0; e < E; ++e) acc[e] = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int s0 = 0; s0 < splits; s0 += SB) {
-        float4 v[SB][E];
+    for (int q = 0; q < GB; ++q) {
+      const int i = q * 256 + tid;
+      g[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (q < gper && i < ngs) g[q] = load4(Ginv + (long long)(i >> 4) * w, a0 + (i & 15) * 4, w, gvec);
+    }
+    for (int f0 = 0; f0 < nld; f0 += NB) {
+      float4 v[NB];
+      int e = f0 / splits, sp = f0 - e * splits;
 #pragma unroll
-        for (int q = 0; q < SB; ++q)
-#pragma unroll
-          for (int e = 0; e < E; ++e) {
-            const int i = i0 + e * 256 + tid;
-            v[q][e] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (s0 + q < splits && i < w * 8)
-              v[q][e] = load4(part + (s0 + q) * sstride + (long long)(i >> 3) * L, x0 + (i & 7) * 4, L, pvec);
-          }
-#pragma unroll
-        for (int q = 0; q < SB; ++q)
-#pragma unroll
-          for (int e = 0; e < E; ++e) {
-            acc[e].x += v[q][e].x;
-            acc[e].y += v[q][e].y;
-            acc[e].z += v[q][e].z;
-            acc[e].w += v[q][e].w;
-          }
+      for (int k = 0; k < NB; ++k) {
+        const int i = e * 256 + tid;
+        v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (f0 + k < nld && i < nps)
+          v[k] = load4(part + sp * sstride + (long long)(i / Q) * L, x0 + (i % Q) * 4, L, pvec);
+        if (++sp == splits) {
+          sp = 0;
+          ++e;
+        }
       }
+      e = f0 / splits;
+      sp = f0 - e * splits;
 #pragma unroll
-      for (int e = 0; e < E; ++e) {
-        const int i = i0 + e * 256 + tid;
-        if (i < w * 8) *reinterpret_cast<float4*>(&Ps[(i >> 3) * DX + (i & 7) * 4]) = acc[e];
+      for (int k = 0; k < NB; ++k) {
+        const int i = e * 256 + tid;
+        if (f0 + k < nld && i < nps) {
+          float4* dst = reinterpret_cast<float4*>(&Ps[(i / Q) * DXT + (i % Q) * 4]);
+          if (sp == 0) {
+            *dst = v[k];
+          } else {
+            float4 t = *dst;
+            t.x += v[k].x;
+            t.y += v[k].y;
+            t.z += v[k].z;
+            t.w += v[k].w;
+            *dst = t;
+          }
+        }
+        if (++sp == splits) {
+          sp = 0;
+          ++e;
+        }
       }
     }
+#pragma unroll
+    for (int q = 0; q < GB; ++q) {
+      const int i = q * 256 + tid;
+      if (q < gper && i < ngs) *reinterpret_cast<float4*>(&Gs[(i >> 4) * kGsLd + (i & 15) * 4]) = g[q];
+    }
+    for (int i = GB * 256 + tid; i < ngs; i += 256)   // w > 64 only
+      *reinterpret_cast<float4*>(&Gs[(i >> 4) * kGsLd + (i & 15) * 4]) =
+          load4(Ginv + (long long)(i >> 4) * w, a0 + (i & 15) * 4, w, gvec);
   }
   __syncthreads();
 
-  float acc[4][2] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+  float acc[4][PX];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < PX; ++j) acc[i][j] = 0.f;
 #pragma unroll 4
   for (int b = 0; b < w; ++b) {
     const float4 g = *reinterpret_cast<const float4*>(&Gs[b * kGsLd + ty * 4]);
-    const float2 p = *reinterpret_cast<const float2*>(&Ps[b * DX + tx * 2]);
-    acc[0][0] = fmaf(g.x, p.x, acc[0][0]); acc[0][1] = fmaf(g.x, p.y, acc[0][1]);
-    acc[1][0] = fmaf(g.y, p.x, acc[1][0]); acc[1][1] = fmaf(g.y, p.y, acc[1][1]);
-    acc[2][0] = fmaf(g.z, p.x, acc[2][0]); acc[2][1] = fmaf(g.z, p.y, acc[2][1]);
-    acc[3][0] = fmaf(g.w, p.x, acc[3][0]); acc[3][1] = fmaf(g.w, p.y, acc[3][1]);
+    float p[PX];
+    if (PX == 1) {
+      p[0] = Ps[b * DXT + tx];
+    } else if (PX == 2) {
+      const float2 t = *reinterpret_cast<const float2*>(&Ps[b * DXT + tx * 2]);
+      p[0] = t.x;
+      p[PX - 1] = t.y;
+    } else {
+#pragma unroll
+      for (int j = 0; j < PX; j += 4) {
+        const float4 t = *reinterpret_cast<const float4*>(&Ps[b * DXT + tx * PX + j]);
+        p[j] = t.x;
+        p[j + 1] = t.y;
+        p[j + 2] = t.z;
+        p[j + 3] = t.w;
+      }
+    }
+    const float gv[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < PX; ++j) acc[i][j] = fmaf(gv[i], p[j], acc[i][j]);
   }
 
 #pragma unroll
@@ -225,8 +265,8 @@ __global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restric
     u64 key = 0;
     if (a < w) {
 #pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int x = x0 + tx * 2 + j;
+      for (int j = 0; j < PX; ++j) {
+        const int x = x0 + tx * PX + j;
         if (x < L) {
           X[(long long)a * ldx + x] = acc[i][j];
           sum.add(acc[i][j]);
@@ -242,12 +282,24 @@ __global__ void __launch_bounds__(256) decorrelate_kernel(const float* __restric
       const u64 t = __shfl_xor_sync(0xffffffffu, key, o);
       key = t > key ? t : key;
     }
-    if (tx == 0 && a < w) {
-      st.spart[(long long)a * st.nchunk + blockIdx.x] = s;
-      st.kpart[(long long)a * st.nchunk + blockIdx.x] = key;
-    }
+    if (tx == 0 && a < w) put_stat(st, a, blockIdx.x, s, key);
   }
   stats_done(st, w);
+}
+
+template <int DXT>
+cudaError_t launch_decorrelate_dx(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
+                                  Stats st, cudaStream_t s) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(decorrelate_kernel<DXT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)decorrelate_smem(kMaxBlock, DXT));
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  dim3 grid((unsigned)cdiv(L, DXT), (unsigned)cdiv(w, TM));
+  decorrelate_kernel<DXT><<<grid, 256, decorrelate_smem(w, DXT), s>>>(Ginv, w, part, splits, L, X, ldx, st);
+  return cudaGetLastError();
 }
 
 template <bool UROW>
@@ -420,20 +472,16 @@ cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int
   return cudaGetLastError();
 }
 
-int decorrelate_chunks(int L) { return (int)cdiv(L, DX); }
+int decorrelate_chunks(int L, int w) { return (int)cdiv(L, decorrelate_dx(L, w)); }
 
 cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
                                Stats st, cudaStream_t s) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(decorrelate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)decorrelate_smem(kMaxBlock));
-    if (e != cudaSuccess) return e;
-    configured = true;
+  switch (decorrelate_dx(L, w)) {
+    case 16: return launch_decorrelate_dx<16>(Ginv, w, part, splits, L, X, ldx, st, s);
+    case 32: return launch_decorrelate_dx<32>(Ginv, w, part, splits, L, X, ldx, st, s);
+    case 64: return launch_decorrelate_dx<64>(Ginv, w, part, splits, L, X, ldx, st, s);
+    default: return launch_decorrelate_dx<128>(Ginv, w, part, splits, L, X, ldx, st, s);
   }
-  dim3 grid((unsigned)cdiv(L, DX), (unsigned)cdiv(w, TM));
-  decorrelate_kernel<<<grid, 256, decorrelate_smem(w), s>>>(Ginv, w, part, splits, L, X, ldx, st);
-  return cudaGetLastError();
 }
 
 int deflate_row_tiles(int m) { return (int)cdiv(m, TM); }

@@ -6,8 +6,8 @@
 //   Vt     w x ldv int8: row a is component a's v (length n; ldv = round_up(n, 16), zero padded) = a block of C.
 //   part   splits x w x L float32: split-K partial products; L = n for the V-step, m for the U-step.
 //   X      w x ldx float32: decorrelated targets, one vector per row (the Eq. 2 input).
-//   Stats  per-vector partials of the Eq. 2 statistics: spart[a * nchunk + c] = sum |x| over chunk c (double-float),
-//          kpart[a * nchunk + c] = max magnitude key over chunk c (chunks of kStatChunk positions).
+//   Stats  per-vector partials of the Eq. 2 statistics: part[a * nchunk + c] = {sum |x| over chunk c (double-float),
+//          max magnitude key over chunk c}, 16 bytes, one chunk per producer CTA column.
 #pragma once
 
 #include <cuda_fp16.h>
@@ -30,17 +30,29 @@ struct Thresh {
   int L;
 };
 
+// One chunk's partial statistics, written and read as a single 16-byte access.
+struct __align__(16) StatPart {
+  F2 s;
+  u64 key;
+};
+
 struct Stats {
-  F2* spart;
-  u64* kpart;
+  StatPart* part;
   int nchunk;
   Thresh th;
 };
 
+__device__ __forceinline__ void put_stat(const Stats& st, int a, int c, F2 s, u64 key) {
+  const uint2 sv = make_uint2(__float_as_uint(s.hi), __float_as_uint(s.lo));
+  *reinterpret_cast<uint4*>(st.part + (long long)a * st.nchunk + c) =
+      make_uint4(sv.x, sv.y, (unsigned)(key & 0xffffffffu), (unsigned)(key >> 32));
+}
+
 // Run by the CTA that finished last: sums every vector's chunk partials (double-float) and writes its threshold.
-// G threads per vector (a power of two, as many as the CTA allows up to a warp) each take chunks g, g + G, ...
-// with all of a batch's loads issued before any is used, then combine with a butterfly inside the group: a fixed
-// order, so the result is reproducible. The double-precision division happens once per vector.
+// G threads per vector (a power of two, as many as the CTA allows up to a warp) each take chunks g, g + G, ... in
+// batches of 16 whose loads are all issued before any is used and which are summed as a pairwise tree; batches
+// add in order, then the group combines with a butterfly. The order is fixed, so the result is reproducible. The
+// double-precision division happens once per vector.
 __device__ __forceinline__ void finalize_thresholds(const Stats& st, int nv) {
   constexpr int kBatch = 16;
   const int nt = blockDim.x;
@@ -50,8 +62,7 @@ __device__ __forceinline__ void finalize_thresholds(const Stats& st, int nv) {
   for (int a0 = 0; a0 < nv; a0 += nt / G) {   // uniform across the CTA: every lane reaches the shuffles
     const int a = a0 + (int)threadIdx.x / G;
     const bool act = a < nv;
-    const F2* sp = st.spart + (long long)a * st.nchunk;
-    const u64* kp = st.kpart + (long long)a * st.nchunk;
+    const uint4* pp = reinterpret_cast<const uint4*>(st.part + (long long)(act ? a : 0) * st.nchunk);
     F2 s;
     u64 key = 0;
     for (int c0 = 0; c0 < st.nchunk; c0 += kBatch * G) {
@@ -60,15 +71,21 @@ __device__ __forceinline__ void finalize_thresholds(const Stats& st, int nv) {
 #pragma unroll
       for (int i = 0; i < kBatch; ++i) {
         const int c = c0 + i * G + g;
-        const bool in = act && c < st.nchunk;
-        sv[i] = in ? sp[c] : F2{};
-        kv[i] = in ? kp[c] : 0ull;
+        uint4 r = make_uint4(0u, 0u, 0u, 0u);
+        if (act && c < st.nchunk) r = pp[c];
+        sv[i].hi = __uint_as_float(r.x);
+        sv[i].lo = __uint_as_float(r.y);
+        kv[i] = ((u64)r.w << 32) | r.z;
       }
 #pragma unroll
-      for (int i = 0; i < kBatch; ++i) {
-        s = f2_add(s, sv[i]);
-        key = kv[i] > key ? kv[i] : key;
-      }
+      for (int h = 1; h < kBatch; h <<= 1)
+#pragma unroll
+        for (int i = 0; i + h < kBatch; i += 2 * h) {
+          sv[i] = f2_add(sv[i], sv[i + h]);
+          kv[i] = kv[i + h] > kv[i] ? kv[i + h] : kv[i];
+        }
+      s = f2_add(s, sv[0]);
+      key = kv[0] > key ? kv[0] : key;
     }
     for (int o = G >> 1; o > 0; o >>= 1) {
       s = f2_add(s, f2_shfl_xor(s, o));
@@ -84,18 +101,20 @@ __device__ __forceinline__ void finalize_thresholds(const Stats& st, int nv) {
   }
 }
 
-// Last-CTA protocol: every CTA calls this after writing its partials; the last one to arrive finalizes.
+// Last-CTA protocol: every CTA calls this after writing its partials. After a barrier, thread 0 takes a ticket
+// with an acquire-release atomic at device scope (ordering the CTA's partial writes before it and the
+// finalizer's reads after it); the CTA that takes the last ticket finalizes and resets the ticket.
 __device__ __forceinline__ void stats_done(const Stats& st, int nv) {
   __shared__ int s_last;
-  __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) {
     const unsigned total = gridDim.x * gridDim.y * gridDim.z;
-    s_last = (atomicAdd(st.th.ticket, 1u) == total - 1u);
+    unsigned old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(st.th.ticket) : "memory");
+    s_last = (old == total - 1u);
   }
   __syncthreads();
   if (s_last) {
-    __threadfence();
     finalize_thresholds(st, nv);
     if (threadIdx.x == 0) *st.th.ticket = 0u;
   }
@@ -108,8 +127,9 @@ cudaError_t launch_product_v(const float* R, int m, int n, const int8_t* Ut, int
                              cudaStream_t s);
 cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int ldv, int w, const float* h,
                              float* part, int splits, cudaStream_t s);
-// Statistics chunks the decorrelation writes per vector of length L.
-int decorrelate_chunks(int L);
+// Statistics chunks the decorrelation writes per vector of length L for a block of w components (at most
+// cdiv(L, 16)).
+int decorrelate_chunks(int L, int w);
 cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
                                Stats st, cudaStream_t s);
 // Rout = Rin - U diag(d) V (Rout may alias Rin or be NULL); U is Ut (component-major, ldu) or, when
@@ -129,6 +149,15 @@ cudaError_t launch_product_v_tc(const float* R, int m, int n, const __half* Ut, 
                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s);
 cudaError_t launch_product_u_tc(const float* R, int m, int n, const __half* Vt, int ldv, int w, const float* h,
                                 float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s);
+// ---- tensor-core deflation (deflate_tc.cu): R -= U diag(d) V^T in place with the factors as K-major fp16
+// (Uk[r * ldk + a], Vk[c * ldk + a]; ldk a multiple of 8 and >= round_up(w, 16)); the statistics outputs have
+// the layout of launch_deflate's (64-row x 128-column tiles).
+cudaError_t launch_deflate_tc(float* R, int m, int n, const __half* Uk, const __half* Vk, long long ldk,
+                              const float* d, int w, const float* h, float* colpart, F2* normpart, float* maxpart,
+                              unsigned* err, cudaStream_t s);
+// dst[pos * ldk + a] = (half) src[a * lda + pos * ldp] for a < w, pos < L (K-major fp16 copy of a ternary factor)
+cudaError_t launch_kmajor(const int8_t* src, long long lda, long long ldp, int w, int L, __half* dst, long long ldk,
+                          cudaStream_t s);
 // dst[r][c] = (half) src[r][c] for an rows x cols int8 matrix
 cudaError_t launch_i8_to_f16(const int8_t* src, long long lds, int rows, int cols, __half* dst, long long ldd,
                              cudaStream_t s);
@@ -138,9 +167,11 @@ cudaError_t launch_stats(const float* X, int nv, int L, int ldx, Stats st, cudaS
 // T = T_tau(X) from finalized thresholds. If gram != NULL (requires nv <= 256) also accumulates the exact Gram
 // matrix of the ternary vectors into the upper triangle gram[a * nv + b] (a <= b) with integer atomics (gram
 // must hold zeros or a running sum).
-// T16 (optional): the same ternary values as fp16 rows with leading dimension ldt16.
+// T16 (optional): the same ternary values as fp16 rows with leading dimension ldt16. Tk (optional): as fp16 in
+// K-major layout, Tk[x * ldk + a] for a < nv (ldk a multiple of 8, >= round_up(nv, 8); 16-byte aligned).
 cudaError_t launch_apply(const float* X, int nv, int L, int ldx, const Thresh& th, int8_t* T, int ldt, int* gram,
-                         cudaStream_t s, __half* T16 = nullptr, long long ldt16 = 0);
+                         cudaStream_t s, __half* T16 = nullptr, long long ldt16 = 0, __half* Tk = nullptr,
+                         long long ldk = 0);
 cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, float* Y, int ldy, Stats st,
                           cudaStream_t s);
 // J = the w columns of largest h_c * sum_t colpart[t][c] (ties to the lower c), ascending; e (n floats) is scratch.

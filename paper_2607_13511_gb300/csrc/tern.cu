@@ -52,8 +52,7 @@ __global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X,
       t = f2_add(t, ssum[q]);
       k = skey[q] > k ? skey[q] : k;
     }
-    st.spart[(long long)a * st.nchunk + blockIdx.x] = t;
-    st.kpart[(long long)a * st.nchunk + blockIdx.x] = k;
+    put_stat(st, a, blockIdx.x, t, k);
   }
   stats_done(st, gridDim.y);
 }
@@ -68,37 +67,38 @@ template <int VB, bool GRAM>
 __global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X, int nv, int L, long long ldx,
                                                     Thresh th, int8_t* __restrict__ T, long long ldt,
                                                     int* __restrict__ gram, int P, __half* __restrict__ T16,
-                                                    long long ldt16) {
+                                                    long long ldt16, __half* __restrict__ Tk, long long ldk) {
   constexpr int PPT = (VB * VB) / 256 > 0 ? (VB * VB) / 256 : 1;   // Gram pairs per thread
   constexpr int IT = VB / 4;                                      // warp passes per 64-position chunk
+  constexpr int KLD = VB + 8;                                     // sK row (halves): 16-byte rows, 4-way stores
   __shared__ unsigned mpos[VB][2], mneg[VB][2];
-  __shared__ float s_theta[VB];
-  __shared__ unsigned s_arg[VB];   // fallback position, or ~0u when some entry passes the threshold
+  __shared__ __align__(16) __half sK[64][KLD];                    // the chunk as [position][component]
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int v0 = blockIdx.y * VB;
   const int nvb = min(VB, nv - v0);
   const int xbeg = blockIdx.x * P, xend = min(L, xbeg + P);
   const int ga = tid % VB, gb0 = (tid / VB) * PPT;
-  for (int a = tid; a < nvb; a += 256) {
-    s_theta[a] = th.theta[v0 + a];
-    s_arg[a] = th.fallback[v0 + a] ? th.arg[v0 + a] : 0xffffffffu;
-  }
   int acc[PPT];
 #pragma unroll
   for (int k = 0; k < PPT; ++k) acc[k] = 0;
-  __syncthreads();
   for (int x0 = xbeg; x0 < xend; x0 += 64) {
     // pass i of warp covers vector a = (warp + 8i) / 2, positions x0 + 32 * ((warp + 8i) % 2) + lane; the
-    // loads of a batch of passes are all issued before the first is used
+    // loads of a batch of passes (values and thresholds) are all issued before the first is used
     constexpr int IB = IT < 16 ? IT : 16;
 #pragma unroll 1
     for (int i0 = 0; i0 < IT; i0 += IB) {
-      float xv[IB];
+      float xv[IB], thv[IB];
+      int fbv[IB];
+      unsigned argv[IB];
 #pragma unroll
       for (int i = 0; i < IB; ++i) {
         const int u = warp + 8 * (i0 + i), a = u >> 1;
         const int x = x0 + 32 * (u & 1) + lane;
-        xv[i] = (a < nvb && x < xend) ? X[(long long)(v0 + a) * ldx + x] : 0.f;
+        const bool in = a < nvb && x < xend;
+        xv[i] = in ? X[(long long)(v0 + a) * ldx + x] : 0.f;
+        thv[i] = a < nvb ? th.theta[v0 + a] : 0.f;
+        fbv[i] = a < nvb ? th.fallback[v0 + a] : 0;
+        argv[i] = a < nvb ? th.arg[v0 + a] : 0u;
       }
 #pragma unroll
       for (int i = 0; i < IB; ++i) {
@@ -107,8 +107,8 @@ __global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X,
         int8_t t = 0;
         if (a < nvb && x < xend) {
           const int v = v0 + a;
-          t = ternary_of(xv[i], s_theta[a]);
-          if ((uint32_t)x == s_arg[a]) t = xv[i] < 0.f ? (int8_t)-1 : (int8_t)1;
+          t = ternary_of(xv[i], thv[i]);
+          if (fbv[i] && (uint32_t)x == argv[i]) t = xv[i] < 0.f ? (int8_t)-1 : (int8_t)1;
           T[(long long)v * ldt + x] = t;
           if (T16 != nullptr) T16[(long long)v * ldt16 + x] = __short2half_rn((short)t);
         }
@@ -119,7 +119,19 @@ __global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X,
             mneg[a][half] = nm;
           }
         }
+        if (Tk != nullptr) sK[32 * half + lane][a] = __short2half_rn((short)t);
       }
+    }
+    if (Tk != nullptr) {   // K-major fp16 copy: rows of the chunk's positions, 16-byte chunks of 8 components
+      __syncthreads();
+      const int kc = (nvb + 7) / 8;
+      for (int id = tid; id < 64 * kc; id += 256) {
+        const int xl = id / kc, j = id - xl * kc;
+        if (x0 + xl < xend)
+          *reinterpret_cast<uint4*>(Tk + (long long)(x0 + xl) * ldk + 8 * j) =
+              *reinterpret_cast<const uint4*>(&sK[xl][8 * j]);
+      }
+      __syncthreads();
     }
     if (GRAM) {
       __syncthreads();
@@ -363,16 +375,19 @@ cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, flo
 }
 
 cudaError_t launch_apply(const float* X, int nv, int L, int ldx, const Thresh& th, int8_t* T, int ldt, int* gram,
-                         cudaStream_t s, __half* T16, long long ldt16) {
-  // about 64 CTAs along the vectors' length, in whole 64-position chunks
-  const int P = 64 * (int)std::max<long long>(1, cdiv(L, 64 * 64));
+                         cudaStream_t s, __half* T16, long long ldt16, __half* Tk, long long ldk) {
+  if (Tk != nullptr && (ldk < round_up(nv, 8) || (ldk & 7) != 0)) return cudaErrorInvalidValue;
+  // one 64-position chunk per CTA up to one CTA per SM, whole chunks per CTA beyond
+  int sms = 152, dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int P = 64 * (int)std::max<long long>(1, cdiv(L, 64LL * sms));
   const int gx = (int)cdiv(L, P);
   const bool g = gram != nullptr && nv <= 128;   // 256 vectors would need 256 accumulators per thread
 #define APPLY_LAUNCH(VB)                                                                                 \
   do {                                                                                                   \
     dim3 grid((unsigned)gx, (unsigned)cdiv(nv, VB));                                                     \
-    if (g) apply_kernel<VB, true><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, gram, P, T16, ldt16);  \
-    else apply_kernel<VB, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16); \
+    if (g) apply_kernel<VB, true><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, gram, P, T16, ldt16, Tk, ldk);  \
+    else apply_kernel<VB, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16, Tk, ldk); \
   } while (0)
   if (nv <= 16) APPLY_LAUNCH(16);
   else if (nv <= 32) APPLY_LAUNCH(32);
@@ -380,7 +395,7 @@ cudaError_t launch_apply(const float* X, int nv, int L, int ldx, const Thresh& t
   else if (nv <= 128) APPLY_LAUNCH(128);
   else {
     dim3 grid((unsigned)gx, (unsigned)cdiv(nv, 256));
-    apply_kernel<256, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16);
+    apply_kernel<256, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16, Tk, ldk);
   }
 #undef APPLY_LAUNCH
   return cudaGetLastError();
