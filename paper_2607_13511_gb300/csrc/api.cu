@@ -186,6 +186,14 @@ bool use_tc(int w) {
   }();
   return enabled && w >= 16;
 }
+// The TMA-fed tensor-core products where the layout allows them; EXTERND_TMA=0 keeps the register-fed ones.
+bool use_tma() {
+  static const bool enabled = [] {
+    const char* e = std::getenv("EXTERND_TMA");
+    return !(e && std::strcmp(e, "0") == 0);
+  }();
+  return enabled;
+}
 int splits_v(int w, int m, int n) { return use_tc(w) ? tc_product_splits(w, n, m) : product_splits(w, n, m); }
 int splits_u(int w, int m, int n) { return use_tc(w) ? tc_product_splits(w, m, n) : product_splits(w, m, n); }
 
@@ -193,12 +201,20 @@ int splits_u(int w, int m, int n) { return use_tc(w) ? tc_product_splits(w, m, n
 // leading dimension ld elements.
 cudaError_t product_v(const float* R, int m, int n, const int8_t* Ut, const __half* Ut16, int ldu, int w, float* part,
                       int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
-  if (use_tc(w)) return launch_product_v_tc(R, m, n, Ut16, ldu, w, part, splits, maxabs, err, s);
+  if (use_tc(w)) {
+    if (use_tma() && tma_product_ok(R, n, Ut16, ldu))
+      return launch_product_v_tma(R, m, n, Ut16, ldu, w, part, splits, maxabs, err, s);
+    return launch_product_v_tc(R, m, n, Ut16, ldu, w, part, splits, maxabs, err, s);
+  }
   return launch_product_v(R, m, n, Ut, ldu, w, part, splits, s);
 }
 cudaError_t product_u(const float* R, int m, int n, const int8_t* Vt, const __half* Vt16, int ldv, int w,
                       const float* h, float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
-  if (use_tc(w)) return launch_product_u_tc(R, m, n, Vt16, ldv, w, h, part, splits, maxabs, err, s);
+  if (use_tc(w)) {
+    if (use_tma() && tma_product_ok(R, n, Vt16, ldv))
+      return launch_product_u_tma(R, m, n, Vt16, ldv, w, h, part, splits, maxabs, err, s);
+    return launch_product_u_tc(R, m, n, Vt16, ldv, w, h, part, splits, maxabs, err, s);
+  }
   return launch_product_u(R, m, n, Vt, ldv, w, h, part, splits, s);
 }
 

@@ -158,6 +158,15 @@ cudaError_t launch_deflate_tc(float* R, int m, int n, const __half* Uk, const __
 // dst[pos * ldk + a] = (half) src[a * lda + pos * ldp] for a < w, pos < L (K-major fp16 copy of a ternary factor)
 cudaError_t launch_kmajor(const int8_t* src, long long lda, long long ldp, int w, int L, __half* dst, long long ldk,
                           cudaStream_t s);
+// Split plan shared by both tensor-core product kernels: split count and reduction elements per split.
+void tc_split(int w, int Lx, int Ly, int* splits, int* chunk);
+// TMA-fed products (product_tma.cu): same contract as the launch_product_*_tc above; usable when
+// tma_product_ok (R and the factor 16-byte aligned, n % 4 == 0, factor ld a multiple of 8).
+bool tma_product_ok(const float* R, int n, const __half* T, int ldt);
+cudaError_t launch_product_v_tma(const float* R, int m, int n, const __half* Ut, int ldu, int w, float* part,
+                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s);
+cudaError_t launch_product_u_tma(const float* R, int m, int n, const __half* Vt, int ldv, int w, const float* h,
+                                 float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s);
 // dst[r][c] = (half) src[r][c] for an rows x cols int8 matrix
 cudaError_t launch_i8_to_f16(const int8_t* src, long long lds, int rows, int cols, __half* dst, long long ldd,
                              cudaStream_t s);

@@ -333,6 +333,12 @@ cudaError_t launch_tc(const float* R, int m, int n, const __half* T, int ldt, in
 
 int tc_product_splits(int w, int Lx, int Ly) { return tc_plan(w, Lx, Ly).splits; }
 
+void tc_split(int w, int Lx, int Ly, int* splits, int* chunk) {
+  const TcPlan t = tc_plan(w, Lx, Ly);
+  *splits = t.splits;
+  *chunk = t.chunk;
+}
+
 cudaError_t launch_product_v_tc(const float* R, int m, int n, const __half* Ut, int ldu, int w, float* part,
                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
   return launch_tc<false>(R, m, n, Ut, ldu, w, nullptr, part, splits, maxabs, err, s);

@@ -1,0 +1,377 @@
+// Residual products on the tensor cores, fed by the Tensor Memory Accelerator (same products and accuracy scheme
+// as product_tc.cu; used when R's rows are 16-byte aligned, i.e. n % 4 == 0):
+//
+//   V-step  part[s][a][c] = sum_{r in split s} U[r][a] R[r][c]       (§2.3 step 1, §2.4)
+//   U-step  part[s][a][r] = sum_{c in split s} R[r][c] h[c] V[c][a]  (§2.3 step 1, §2.5)
+//
+// A CTA owns 128 output positions (MMA M) and all w components (N = w rounded up to 16), reducing over one
+// split of the other dimension in stages of 64. Roles, all hand-offs through mbarriers with bounded waits:
+//   producer (one thread)  TMA loads of the float32 R tile of a stage (128-byte swizzled boxes of 32 floats)
+//                          into a ring of S32 slots, and of the stage's fp16 ternary tile (the MMA's B operand,
+//                          128-byte swizzled K-major) into a ring of SB slots
+//   converters (8 warps)   read a staged R tile (lanes on consecutive positions: conflict-free), scale it by
+//                          2^s, split it into fp16 hi and lo, and write the two swizzled K-major A tiles into a
+//                          ring of S16 slots; the same warps run the epilogue (TMEM -> split-K partials)
+//   MMA (one thread)       two kind::f16 MMAs per 16-deep K step (hi and lo against the same B), commits that
+//                          free the A and B slots
+// R never passes through registers on its way into shared memory, so the loads of several stages are in flight
+// per SM without any register cost.
+#include <cuda.h>
+
+#include "kernels.h"
+#include "umma.cuh"
+
+namespace externd {
+
+namespace {
+
+constexpr int kConvWarps = 8;
+constexpr int kConv = kConvWarps * 32;
+constexpr int kProducerWarp = kConvWarps, kMmaWarp = kConvWarps + 1;
+constexpr int kThreads = (kConvWarps + 2) * 32;
+constexpr int kStageK = 64;
+constexpr uint32_t kTileA = 128u * 128u;      // 128 rows x 64 fp16
+constexpr uint32_t kStage32 = 128u * 64u * 4u;   // float32 R tile of one stage
+
+struct TmaArgs {
+  int m, n, w, wpad;
+  const float* h;
+  float* part;
+  int ychunk;
+  const float* maxabs;
+  unsigned* err;
+  int s32, sb, s16;
+  uint32_t tmem_cols;
+};
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+          "r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+// Byte offset of float c (0..31) of row r in a box of 128-byte rows with the 128-byte swizzle.
+__device__ __forceinline__ uint32_t sw128_f32(uint32_t r, uint32_t c) {
+  return r * 128u + ((((c >> 2) ^ (r & 7u)) << 4) | ((c & 3u) << 2));
+}
+
+__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __half2 h = __floats2half2_rn(x0, x1);
+  const float2 hb = __half22float2(h);
+  const __half2 l = __floats2half2_rn(x0 - hb.x, x1 - hb.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
+template <bool USTEP>
+__global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_constant__ CUtensorMap mapR,
+                                                                  const __grid_constant__ CUtensorMap mapT,
+                                                                  const TmaArgs p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t sbase = (raw + 1023u) & ~1023u;
+  uint8_t* const gbase = smem_raw + (sbase - raw);
+  const uint32_t tileB = (uint32_t)p.wpad * 128u;
+  const uint32_t r32 = sbase;                                   // S32 x 32 KB
+  const uint32_t rb = r32 + (uint32_t)p.s32 * kStage32;         // SB x tileB (1024-aligned: tileB = wpad * 128)
+  const uint32_t ra = rb + (uint32_t)round_up((long long)p.sb * tileB, 1024);   // S16 x (2 x 16 KB)
+  const uint32_t bars = ra + (uint32_t)p.s16 * 2u * kTileA;
+  const uint32_t full32 = bars, empty32 = full32 + 8u * p.s32;
+  const uint32_t fullB = empty32 + 8u * p.s32, emptyB = fullB + 8u * p.sb;
+  const uint32_t full16 = emptyB + 8u * p.sb, empty16 = full16 + 8u * p.s16;
+  const uint32_t done_bar = empty16 + 8u * p.s16;
+  const uint32_t tmem_slot = done_bar + 8u;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int Lx = USTEP ? p.m : p.n;
+  const int Ly = USTEP ? p.n : p.m;
+  const int x0 = blockIdx.x * 128;
+  const int ybeg = blockIdx.z * p.ychunk;
+  const int yend = min(Ly, ybeg + p.ychunk);
+  const int nk = ybeg < yend ? (int)cdiv(yend - ybeg, kStageK) : 0;
+
+  float mx = __ldg(p.maxabs);
+  if (USTEP && p.h != nullptr) mx *= __ldg(p.maxabs + 1);
+  int ex = 0;
+  if (mx > 0.f && mx <= 3.0e38f) frexpf(mx, &ex);
+  const int sexp = max(-100, min(100, 14 - ex));
+  const float scale = ldexpf(1.f, sexp), inv_scale = ldexpf(1.f, -sexp);
+
+  if (tid == 0) {
+    for (int s = 0; s < p.s32; ++s) {
+      mbar_init(full32 + 8u * s, 1);
+      mbar_init(empty32 + 8u * s, kConvWarps);
+    }
+    for (int s = 0; s < p.sb; ++s) {
+      mbar_init(fullB + 8u * s, 1);
+      mbar_init(emptyB + 8u * s, 1);
+    }
+    for (int s = 0; s < p.s16; ++s) {
+      mbar_init(full16 + 8u * s, kConvWarps);
+      mbar_init(empty16 + 8u * s, 1);
+    }
+    mbar_init(done_bar, 1);
+    fence_barrier_init();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(tmem_slot, p.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(gbase + (tmem_slot - sbase));
+
+  bool ok = true;
+  if (warp == kProducerWarp) {
+    // ------------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int k = 0, kb = 0;   // stages whose R copies / B copies were issued
+      for (; k < nk; ++k) {
+        const int s = k % p.s32, sb = k % p.sb;
+        if (k >= p.s32 && !mbar_wait(empty32 + 8u * s, (uint32_t)(k / p.s32 - 1) & 1u, p.err)) break;
+        const int y0 = ybeg + k * kStageK;
+        mbar_expect_tx(full32 + 8u * s, kStage32);
+        if (!USTEP) {
+#pragma unroll
+          for (int b = 0; b < 4; ++b) tma_load_2d(r32 + s * kStage32 + b * 8192u, &mapR, x0 + 32 * b, y0, full32 + 8u * s);
+        } else {
+#pragma unroll
+          for (int b = 0; b < 2; ++b) tma_load_2d(r32 + s * kStage32 + b * 16384u, &mapR, y0 + 32 * b, x0, full32 + 8u * s);
+        }
+        if (k >= p.sb && !mbar_wait(emptyB + 8u * sb, (uint32_t)(k / p.sb - 1) & 1u, p.err)) {
+          ++k;   // stage k's R copies are in flight, its B copy is not
+          break;
+        }
+        mbar_expect_tx(fullB + 8u * sb, tileB);
+        tma_load_2d(rb + sb * tileB, &mapT, y0, 0, fullB + 8u * sb);
+        kb = k + 1;
+      }
+      // every copy this thread issued lands before the CTA can exit (bounded waits)
+      for (int j = max(0, k - p.s32); j < k; ++j) mbar_wait(full32 + 8u * (j % p.s32), (uint32_t)(j / p.s32) & 1u, p.err);
+      for (int j = max(0, kb - p.sb); j < kb; ++j) mbar_wait(fullB + 8u * (j % p.sb), (uint32_t)(j / p.sb) & 1u, p.err);
+    }
+  } else if (warp == kMmaWarp) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = f16_idesc(128, (uint32_t)p.wpad);
+      for (int k = 0; k < nk; ++k) {
+        const int s = k % p.s16, sb = k % p.sb;
+        if (!mbar_wait(full16 + 8u * s, (uint32_t)(k / p.s16) & 1u, p.err) ||
+            !mbar_wait(fullB + 8u * sb, (uint32_t)(k / p.sb) & 1u, p.err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a_hi = ra + (uint32_t)s * 2u * kTileA, a_lo = a_hi + kTileA, bt = rb + (uint32_t)sb * tileB;
+#pragma unroll
+        for (int kk = 0; kk < kStageK / 16; ++kk) {
+          const uint64_t bd = sw128_desc(bt + 32u * kk);
+          mma_f16(tmem, sw128_desc(a_hi + 32u * kk), bd, idesc, (k > 0 || kk > 0) ? 1u : 0u);
+          mma_f16(tmem, sw128_desc(a_lo + 32u * kk), bd, idesc, 1u);
+        }
+        mma_commit(empty16 + 8u * s);
+        mma_commit(emptyB + 8u * sb);
+      }
+      mma_commit(done_bar);
+    }
+  } else {
+    // ------------------------------------------------------------------ converters
+    // item i = tid + 256 q (q < 4): A row x = i % 128 (lanes on consecutive rows), K chunk o = i / 128
+    for (int k = 0; k < nk && ok; ++k) {
+      const int s = k % p.s32, s16 = k % p.s16;
+      const bool got = mbar_wait(full32 + 8u * s, (uint32_t)(k / p.s32) & 1u, p.err) &&
+                       (k < p.s16 || mbar_wait(empty16 + 8u * s16, (uint32_t)(k / p.s16 - 1) & 1u, p.err));
+      ok = __all_sync(0xffffffffu, got) != 0;
+      if (!ok) break;
+      const uint8_t* st = gbase + (r32 - sbase) + (size_t)s * kStage32;
+      uint8_t* a_hi = gbase + (ra - sbase) + (size_t)s16 * 2u * kTileA;
+      uint8_t* a_lo = a_hi + kTileA;
+      const int y0 = ybeg + k * kStageK;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int i = tid + kConv * q;
+        const int x = i & 127, o = i >> 7;
+        const int valid = yend - (y0 + 8 * o);   // elements of this chunk inside the split
+        float v[8];
+        if (!USTEP) {
+          // R[y0 + 8o + j][x0 + x]: box x / 32, row 8o + j, float x % 32
+          const uint8_t* bx = st + (x >> 5) * 8192;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) v[j] = *reinterpret_cast<const float*>(bx + sw128_f32(8 * o + j, x & 31));
+        } else {
+          // R[x0 + x][y0 + 8o .. +7]: box o / 4, row x, floats 8 (o % 4) .. +7 (two 16-byte chunks)
+          const uint8_t* bx = st + (o >> 2) * 16384;
+          const float4 a = *reinterpret_cast<const float4*>(bx + sw128_f32(x, 8 * (o & 3)));
+          const float4 b = *reinterpret_cast<const float4*>(bx + sw128_f32(x, 8 * (o & 3) + 4));
+          v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+          v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+          if (p.h != nullptr) {
+            const int c = y0 + 8 * o;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) v[j] *= (c + j < Ly) ? __ldg(p.h + c + j) : 0.f;
+          }
+        }
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float x0v = 2 * e < valid ? v[2 * e] * scale : 0.f;
+          const float x1v = 2 * e + 1 < valid ? v[2 * e + 1] * scale : 0.f;
+          split_pair(x0v, x1v, hi[e], lo[e]);
+        }
+        const uint32_t off = sw128_offset((uint32_t)x, (uint32_t)o);
+        *reinterpret_cast<uint4*>(a_hi + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<uint4*>(a_lo + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+      }
+      fence_async_shared();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(full16 + 8u * s16);
+        mbar_arrive(empty32 + 8u * s);
+      }
+    }
+  }
+
+  // ------------------------------------------------------------------ epilogue (converter warps)
+  const int all_ok = __syncthreads_and(ok ? 1 : 0);
+  if (warp < kConvWarps) {
+    bool have = nk > 0 && all_ok;
+    const bool waited = mbar_wait(done_bar, 0u, p.err);
+    have = __all_sync(0xffffffffu, have && waited);
+    tc_fence_after();
+    const int quad = warp & 3, group = warp >> 2;   // 2 warps per TMEM lane quadrant
+    const int xi = x0 + quad * 32 + lane;
+    float* out = p.part + (long long)blockIdx.z * p.w * Lx;
+    for (int ch = group; ch < p.wpad / 16; ch += kConvWarps / 4) {
+      uint32_t v[16];
+      if (have) {
+        tmem_ld16(tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(ch * 16), v);
+        tmem_wait_ld();
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = 0u;
+      }
+      if (xi < Lx) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int a = ch * 16 + i;
+          if (a < p.w) out[(long long)a * Lx + xi] = __uint_as_float(v[i]) * inv_scale;
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem, p.tmem_cols);
+  }
+}
+
+typedef CUresult (*EncodeTiled)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiled encoder() {
+  static EncodeTiled fn = [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+      cudaGetLastError();
+      return (EncodeTiled) nullptr;
+    }
+    return reinterpret_cast<EncodeTiled>(f);
+  }();
+  return fn;
+}
+
+struct TmaPlan {
+  int wpad, s32, sb, s16;
+  size_t smem;
+};
+
+TmaPlan tma_plan(int w) {
+  TmaPlan t;
+  t.wpad = (int)round_up(w, 16);
+  const size_t tileB = (size_t)t.wpad * 128;
+  t.s16 = 2;
+  const size_t budget = 227 * 1024 - 1024 - 512 - (size_t)t.s16 * 2 * kTileA;
+  int s = 4;
+  while (s > 1 && (size_t)s * kStage32 + round_up((long long)s * tileB, 1024) > budget) --s;
+  t.s32 = t.sb = s;
+  t.smem = 1024 + (size_t)s * kStage32 + round_up((long long)s * tileB, 1024) + (size_t)t.s16 * 2 * kTileA + 512;
+  return t;
+}
+
+template <bool USTEP>
+cudaError_t launch_tma(const float* R, int m, int n, const __half* T, int ldt, int w, const float* h, float* part,
+                       int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
+  EncodeTiled enc = encoder();
+  if (enc == nullptr) return cudaErrorNotSupported;
+  const int Lx = USTEP ? m : n, Ly = USTEP ? n : m;
+  int chunk, sp;
+  tc_split(w, Lx, Ly, &sp, &chunk);
+  if (splits != sp) return cudaErrorInvalidValue;
+  const TmaPlan t = tma_plan(w);
+  CUtensorMap mapR, mapT;
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)n, (cuuint64_t)m};
+    const cuuint64_t strides[1] = {(cuuint64_t)n * 4};
+    const cuuint32_t box[2] = {32u, USTEP ? 128u : 64u};
+    const cuuint32_t es[2] = {1u, 1u};
+    if (enc(&mapR, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(R), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)Ly, (cuuint64_t)w};
+    const cuuint64_t strides[1] = {(cuuint64_t)ldt * 2};
+    const cuuint32_t box[2] = {64u, (cuuint32_t)t.wpad};
+    const cuuint32_t es[2] = {1u, 1u};
+    if (enc(&mapT, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half*>(T), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  static bool configured[2] = {false, false};
+  if (!configured[USTEP]) {
+    cudaError_t e = cudaFuncSetAttribute(product_tma_kernel<USTEP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         227 * 1024);
+    if (e != cudaSuccess) return e;
+    configured[USTEP] = true;
+  }
+  uint32_t cols = 32;
+  while ((int)cols < t.wpad) cols <<= 1;
+  TmaArgs a{m, n, w, t.wpad, h, part, chunk, maxabs, err, t.s32, t.sb, t.s16, cols};
+  dim3 grid((unsigned)cdiv(Lx, 128), 1, (unsigned)splits);
+  product_tma_kernel<USTEP><<<grid, kThreads, t.smem, s>>>(mapR, mapT, a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool tma_product_ok(const float* R, int n, const __half* T, int ldt) {
+  return encoder() != nullptr && (n % 4) == 0 && ((uintptr_t)R & 15u) == 0 && ((uintptr_t)T & 15u) == 0 &&
+         (ldt % 8) == 0;
+}
+
+cudaError_t launch_product_v_tma(const float* R, int m, int n, const __half* Ut, int ldu, int w, float* part,
+                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
+  return launch_tma<false>(R, m, n, Ut, ldu, w, nullptr, part, splits, maxabs, err, s);
+}
+
+cudaError_t launch_product_u_tma(const float* R, int m, int n, const __half* Vt, int ldv, int w, const float* h,
+                                 float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
+  return launch_tma<true>(R, m, n, Vt, ldv, w, h, part, splits, maxabs, err, s);
+}
+
+}  // namespace externd
