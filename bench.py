@@ -33,11 +33,12 @@ from paper_2607_13511_gb300 import workloads as W  # noqa: E402
 METRIC = "ternary components fitted/sec per matrix"
 UNIT = "components/s"
 DEFAULT_WORKLOAD = W.OUTLIER_2048.name
-ROOFLINE_KIND = "vstep"   # the kernel class with the largest share of device time (profiles/launches_*.md)
+ROOFLINE_KIND = "vstep"   # the largest HBM stream of the path: the V-step residual product (profiles/)
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch of the profiled kernel, from one ncu capture, valid
 # only while the kernel's source is unchanged (sha256 of the file that holds it).
-NCU_TRAFFIC: dict = {}
+NCU_TRAFFIC: dict = {"kind": "vstep", "file": "product_tma.cu", "sha": "d4d5f9a979ef2b69", "workload": "outlier2048_mu3_b64",
+               "bytes_per_launch": 17077888}
 
 
 def env_int(name, default):
