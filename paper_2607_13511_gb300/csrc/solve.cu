@@ -333,31 +333,63 @@ __global__ void __launch_bounds__(512) rvec_kernel(const int8_t* __restrict__ Ut
   }
 }
 
-// Wide-block sweep for w <= 128: NB pivots per step. 512 threads; thread (ty, tx) in a 16 x 32 grid owns
-// the RPT = W_PAD/16 rows ty*RPT + a and the CPT = W_PAD/32 columns tx + 32c in registers. Per step K:
-//   1. the owners of rows K publish them (Rk = S[K,:], shared memory)                        barrier
-//   2. warp 0 inverts the NB x NB pivot block P: Q = P^-1 (lane l keeps column l in registers; the pivot
-//      column is broadcast with shuffles, by symmetry it is also the pivot row)                barrier
-//   3. T'[i,:] = S[i,K] Q for rows outside K and -Q[i,:] for rows in K                        barrier
-//   4. one uniform rank-NB update S <- D S - T' Rk, D zeroing the rows of K: outside K this is the Schur
-//      complement S - S[I,K] Q S[K,J], on the rows of K it gives Q S[K,J]; then the columns of K take T'
-//      (S[I,K] Q, and -Q on the pivot block)                                                   barrier
-// The serial part is NB pivots of one warp per step; everything else is the same dense float32 FMA work on
-// every thread. After the last step S = -(G + eps I)^-1.
+// One warp inverts an NB x NB SPD block by the symmetric sweep: lane l holds EPL = NB^2/32 entries of row
+// l / LPR (LPR = NB / EPL lanes per row), columns (l % LPR) * EPL + e. Per pivot kk every lane fetches with
+// shuffles the pivot-row entries of its columns (from the lane of row kk with the same column group), the pivot,
+// and its row's pivot-column entry (by symmetry the entry of row r in column kk sits at a register index that is
+// the same for every lane), then updates its entries. On return A holds -P^-1.
+template <int NB>
+__device__ __forceinline__ void warp_sweep(float (&A)[NB * NB / 32], int lane) {
+  constexpr int EPL = NB * NB / 32, LPR = NB / EPL;
+  const int r = lane / LPR, cg = lane % LPR, cb = cg * EPL;
+#pragma unroll
+  for (int kk = 0; kk < NB; ++kk) {
+    float akc[EPL];
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) akc[e] = __shfl_sync(0xffffffffu, A[e], kk * LPR + cg);
+    const float p = __shfl_sync(0xffffffffu, A[kk % EPL], kk * LPR + kk / EPL);
+    const float ark0 = __shfl_sync(0xffffffffu, A[kk % EPL], r * LPR + kk / EPL);
+    const float ip = __fdividef(1.f, p);
+    const float ark = ark0 * ip;   // P[r][kk] / p
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) {
+      const int c = cb + e;
+      float v = fmaf(-ark, akc[e], A[e]);
+      v = (c == kk) ? ark : v;
+      v = (r == kk) ? ((c == kk) ? -ip : akc[e] * ip) : v;
+      A[e] = v;
+    }
+  }
+}
+
+// Wide-block sweep for w <= 128 with lookahead: NB pivots per step. 16 tile warps (512 threads; thread (ty, tx)
+// owns the RPT = W_PAD/16 rows ty*RPT + a and the CPT = W_PAD/32 columns tx + 32c in registers) and one pivot
+// warp. With Q = P^-1 of the current pivot block K (computed one step ahead), per step:
+//   a. tile warps: T'[i,:] = S[i,K] Q for rows outside K (S[i,K] = Rk[.,i] by symmetry), -Q[i,:] on K; the
+//      owners of the next block K+ also publish S[K+,K+] as it stands before this step's update      barrier
+//   b. tile warps: one uniform rank-NB update S <- D S - T' Rk (D zeroes the rows of K: outside K this is the
+//      Schur complement S - S[I,K] Q S[K,J], on K it gives Q S[K,J]), then the columns of K take T'
+//      (S[I,K] Q, and -Q on the pivot block); the owners of K+ publish the updated rows K+.
+//      Pivot warp, meanwhile: the updated next pivot block S[K+,K+] - T'[K+,:] Rk[:,K+] (the same operations
+//      in the same order as the tile owners) and its inverse by warp_sweep, for the next step          barrier
+// After the last step S = -(G + eps I)^-1.
 // IN_INT: the Gram comes as an integer upper triangle Gint[a * w + b] (a <= b), reset to zero after reading;
 // each thread reads its upper-triangle entries and the lower ones come back mirrored through shared memory.
 template <int W_PAD, int NB, int MODE, bool IN_INT>
-__global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ Gpart, int splits, int w,
+__global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ Gpart, int splits, int w,
                                                       const float* __restrict__ GVraw, const float* __restrict__ r,
                                                       float* __restrict__ Graw, float* __restrict__ out, int* Gint) {
-  constexpr int RPT = W_PAD / 16, CPT = W_PAD / 32;
-  static_assert(W_PAD % NB == 0 && 32 % NB == 0 && RPT >= 1 && CPT >= 1, "bad shape");
-  __shared__ __align__(16) float Rk[NB][W_PAD + 1];
-  __shared__ __align__(16) float T[W_PAD][NB + 1];
-  __shared__ float Qs[NB][NB + 1];
+  constexpr int RPT = W_PAD / 16, CPT = W_PAD / 32, EPL = NB * NB / 32, LPR = NB / EPL, TLD = NB + 4;
+  static_assert(W_PAD % NB == 0 && 32 % NB == 0 && (NB * NB) % 32 == 0 && NB % 4 == 0 && RPT >= 1 && CPT >= 1,
+                "bad shape");
+  __shared__ __align__(16) float Rk[2][NB][W_PAD];   // published rows of the pivot block (two buffers)
+  __shared__ __align__(16) float T[W_PAD][TLD];      // T' of the step (padded rows: conflict-free float4 stores)
+  __shared__ __align__(16) float Qs[2][NB][NB];      // pivot-block inverses (two buffers)
+  __shared__ float Pn[NB][NB];                        // next pivot block before this step's update
   __shared__ float red[16];
-  const int tid = threadIdx.x, tx = tid & 31, ty = tid >> 5, lane = tx;
-  const int i0 = ty * RPT;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const bool tile = warp < 16;
+  const int tx = lane, ty = tile ? warp : 0, i0 = ty * RPT;
 
   float S[RPT][CPT];
 #pragma unroll
@@ -366,29 +398,39 @@ __global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ 
     for (int c = 0; c < CPT; ++c) S[a][c] = 0.f;
   if (IN_INT) {
     extern __shared__ float mirror[];   // [W_PAD][W_PAD + 1]: mirror[j][i] = G[i][j] for i < j
+    if (tile) {   // every load issued before the first mirror store
 #pragma unroll
-    for (int a = 0; a < RPT; ++a) {
-      const int i = i0 + a;
+      for (int a = 0; a < RPT; ++a) {
+        const int i = i0 + a;
 #pragma unroll
-      for (int c = 0; c < CPT; ++c) {
-        const int j = tx + 32 * c;
-        if (i <= j && j < w) {
-          S[a][c] = (float)Gint[(long long)i * w + j];
-          mirror[j * (W_PAD + 1) + i] = S[a][c];
+        for (int c = 0; c < CPT; ++c) {
+          const int j = tx + 32 * c;
+          S[a][c] = (i <= j && j < w) ? (float)Gint[(long long)i * w + j] : 0.f;
+        }
+      }
+#pragma unroll
+      for (int a = 0; a < RPT; ++a) {
+        const int i = i0 + a;
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) {
+          const int j = tx + 32 * c;
+          if (i < j && j < w) mirror[j * (W_PAD + 1) + i] = S[a][c];
         }
       }
     }
     __syncthreads();
+    if (tile) {
 #pragma unroll
-    for (int a = 0; a < RPT; ++a) {
-      const int i = i0 + a;
+      for (int a = 0; a < RPT; ++a) {
+        const int i = i0 + a;
 #pragma unroll
-      for (int c = 0; c < CPT; ++c) {
-        const int j = tx + 32 * c;
-        if (j < i && i < w) S[a][c] = mirror[i * (W_PAD + 1) + j];
+        for (int c = 0; c < CPT; ++c) {
+          const int j = tx + 32 * c;
+          if (j < i && i < w) S[a][c] = mirror[i * (W_PAD + 1) + j];
+        }
       }
     }
-  } else {
+  } else if (tile) {
     for (int sp = 0; sp < splits; ++sp) {
       const float* G = Gpart + (long long)sp * w * w;
 #pragma unroll
@@ -404,133 +446,169 @@ __global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ 
     }
   }
   float diag = 0.f;
+  if (tile) {
 #pragma unroll
-  for (int a = 0; a < RPT; ++a) {
-    const int i = i0 + a;
+    for (int a = 0; a < RPT; ++a) {
+      const int i = i0 + a;
 #pragma unroll
-    for (int c = 0; c < CPT; ++c) {
-      const int j = tx + 32 * c;
-      float v = S[a][c];
-      if (i < w && j < w) {
-        if (MODE == 0) Graw[(long long)i * w + j] = v;
-        else v *= GVraw[(long long)i * w + j];
-        if (i == j) diag += v;
-      } else {
-        v = (i == j) ? 1.f : 0.f;
+      for (int c = 0; c < CPT; ++c) {
+        const int j = tx + 32 * c;
+        float v = S[a][c];
+        if (i < w && j < w) {
+          if (MODE == 0) Graw[(long long)i * w + j] = v;
+          else v *= GVraw[(long long)i * w + j];
+          if (i == j) diag += v;
+        } else {
+          v = (i == j) ? 1.f : 0.f;
+        }
+        S[a][c] = v;
       }
-      S[a][c] = v;
     }
+    const float dw = warp_sum(diag);
+    if (lane == 0) red[ty] = dw;
   }
-  const float dw = warp_sum(diag);
-  if (lane == 0) red[ty] = dw;
   __syncthreads();
   float tr = 0.f;
 #pragma unroll
   for (int q = 0; q < 16; ++q) tr += red[q];
   const float eps = ((MODE == 0) || (w > 1)) ? (float)kEpsRel * tr / (float)w : 0.f;
-#pragma unroll
-  for (int a = 0; a < RPT; ++a)
-#pragma unroll
-    for (int c = 0; c < CPT; ++c)
-      if (i0 + a < w && i0 + a == tx + 32 * c) S[a][c] += eps;
-
-  for (int k0 = 0; k0 < w; k0 += NB) {
-    // 1. publish rows K
-#pragma unroll
-    for (int a = 0; a < RPT; ++a) {
-      const int i = i0 + a;
-      if (i >= k0 && i < k0 + NB) {
-#pragma unroll
-        for (int c = 0; c < CPT; ++c) Rk[i - k0][tx + 32 * c] = S[a][c];
-      }
-    }
-    __syncthreads();
-    // 2. warp 0: Q = P^-1 (symmetric sweep of the NB x NB block; lane l holds column l, i.e. P[.][l])
-    if (ty == 0) {
-      float col[NB];
-#pragma unroll
-      for (int e = 0; e < NB; ++e) {
-        const bool inside = (lane < NB) && (k0 + e < w) && (k0 + lane < w);
-        col[e] = inside ? Rk[e][k0 + lane] : ((e == lane) ? 1.f : 0.f);
-      }
-#pragma unroll
-      for (int kk = 0; kk < NB; ++kk) {
-        const float pkl = col[kk];                                   // P[kk][l] = P[l][kk]
-        const float p = __shfl_sync(0xffffffffu, pkl, kk);            // P[kk][kk]
-        const float ip = __fdividef(1.f, p);
-#pragma unroll
-        for (int e = 0; e < NB; ++e) {
-          const float pek = __shfl_sync(0xffffffffu, pkl, e);          // P[e][kk] = P[kk][e] (lane e's entry)
-          float v = fmaf(-pek * ip, pkl, col[e]);
-          v = (e == kk) ? pkl * ip : v;                               // row kk
-          v = (lane == kk) ? ((e == kk) ? -ip : pek * ip) : v;        // column kk, pivot
-          col[e] = v;
-        }
-      }
-      if (lane < NB) {
-#pragma unroll
-        for (int e = 0; e < NB; ++e) Qs[e][lane] = -col[e];
-      }
-    }
-    __syncthreads();
-    // 3. T'[i][b] = sum_c S[i][k0 + c] Q[c][b] = sum_c Rk[c][i] Q[c][b] outside K, -Q[i - k0][b] on K
-    for (int idx = tid; idx < W_PAD * (NB / 8); idx += 512) {
-      const int i = idx / (NB / 8), bq = (idx % (NB / 8)) * 8;
-      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      if (i >= k0 && i < k0 + NB) {
-#pragma unroll
-        for (int u = 0; u < 8; ++u) acc[u] = -Qs[i - k0][bq + u];
-      } else {
-#pragma unroll
-        for (int c = 0; c < NB; ++c) {
-          const float rv = Rk[c][i];
-#pragma unroll
-          for (int u = 0; u < 8; ++u) acc[u] = fmaf(rv, Qs[c][bq + u], acc[u]);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) T[i][bq + u] = acc[u];
-    }
-    __syncthreads();
-    // 4. S <- D S - T' Rk, then the columns of K (all in register column cK: NB divides 32) take T'
-    float acc[RPT][CPT];
+  if (tile) {
 #pragma unroll
     for (int a = 0; a < RPT; ++a)
 #pragma unroll
-      for (int c = 0; c < CPT; ++c) acc[a][c] = 0.f;
-#pragma unroll 4
-    for (int b = 0; b < NB; ++b) {
-      float tv[RPT], rv[CPT];
-#pragma unroll
-      for (int a = 0; a < RPT; ++a) tv[a] = T[i0 + a][b];
-#pragma unroll
-      for (int c = 0; c < CPT; ++c) rv[c] = Rk[b][tx + 32 * c];
-#pragma unroll
-      for (int a = 0; a < RPT; ++a)
-#pragma unroll
-        for (int c = 0; c < CPT; ++c) acc[a][c] = fmaf(tv[a], rv[c], acc[a][c]);
-    }
-    const int cK = k0 >> 5;
-    const int jk = tx + 32 * cK - k0;                 // this lane's column within K, when in [0, NB)
-    const bool lane_in = jk >= 0 && jk < NB;
-    const int jb = min(max(jk, 0), NB - 1);
+      for (int c = 0; c < CPT; ++c)
+        if (i0 + a < w && i0 + a == tx + 32 * c) S[a][c] += eps;
+  }
+
+  // rows [kb, kb + NB) of the register tiles into Rk[buf]
+  auto publish_rows = [&](int kb, int buf) {
 #pragma unroll
     for (int a = 0; a < RPT; ++a) {
       const int i = i0 + a;
-      const bool i_in = (i >= k0 && i < k0 + NB);   // uniform across the warp
+      if (i >= kb && i < kb + NB) {
 #pragma unroll
-      for (int c = 0; c < CPT; ++c) {
-        float v = (i_in ? 0.f : S[a][c]) - acc[a][c];
-        if (c == cK) {
-          const float tk = T[i][jb];
-          v = lane_in ? tk : v;
-        }
-        S[a][c] = v;
+        for (int c = 0; c < CPT; ++c) Rk[buf][i - kb][tx + 32 * c] = S[a][c];
       }
     }
-    __syncthreads();   // Rk, Qs, T are rewritten by the next step
+  };
+  // prologue: the first pivot block and its inverse
+  if (tile) publish_rows(0, 0);
+  __syncthreads();
+  if (!tile) {
+    float A[EPL];
+    const int pr_ = lane / LPR, pc = (lane % LPR) * EPL;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) A[e] = Rk[0][pr_][pc + e];
+    warp_sweep<NB>(A, lane);
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) Qs[0][pr_][pc + e] = -A[e];
+  }
+  __syncthreads();
+
+  for (int k0 = 0, step = 0; k0 < w; k0 += NB, ++step) {
+    const int cur = step & 1, nxt = cur ^ 1;
+    const int kn = k0 + NB;
+    const bool has_next = kn < w;
+    // a. T' and the next pivot block as it stands
+    if (tile) {
+      for (int it = tid; it < W_PAD * (NB / 4); it += 512) {
+        const int i = it % W_PAD, bq = (it / W_PAD) * 4;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i >= k0 && i < k0 + NB) {
+          const float4 q = *reinterpret_cast<const float4*>(&Qs[cur][i - k0][bq]);
+          acc = make_float4(-q.x, -q.y, -q.z, -q.w);
+        } else {
+#pragma unroll
+          for (int c = 0; c < NB; ++c) {
+            const float rv = Rk[cur][c][i];
+            const float4 q = *reinterpret_cast<const float4*>(&Qs[cur][c][bq]);
+            acc.x = fmaf(rv, q.x, acc.x);
+            acc.y = fmaf(rv, q.y, acc.y);
+            acc.z = fmaf(rv, q.z, acc.z);
+            acc.w = fmaf(rv, q.w, acc.w);
+          }
+        }
+        *reinterpret_cast<float4*>(&T[i][bq]) = acc;
+      }
+      if (has_next) {
+#pragma unroll
+        for (int a = 0; a < RPT; ++a) {
+          const int i = i0 + a;
+          if (i >= kn && i < kn + NB) {
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) {
+              const int j = tx + 32 * c;
+              if (j >= kn && j < kn + NB) Pn[i - kn][j - kn] = S[a][c];
+            }
+          }
+        }
+      }
+    }
+    __syncthreads();
+    // b. the update (tile warps) beside the next pivot block's inverse (pivot warp)
+    if (tile) {
+#pragma unroll
+      for (int a = 0; a < RPT; ++a)
+        if (i0 + a >= k0 && i0 + a < k0 + NB)
+#pragma unroll
+          for (int c = 0; c < CPT; ++c) S[a][c] = 0.f;
+#pragma unroll
+      for (int b = 0; b < NB; b += 4) {
+        float4 tv[RPT];
+        float rv[4][CPT];
+#pragma unroll
+        for (int a = 0; a < RPT; ++a) tv[a] = *reinterpret_cast<const float4*>(&T[i0 + a][b]);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+#pragma unroll
+          for (int c = 0; c < CPT; ++c) rv[q][c] = Rk[cur][b + q][tx + 32 * c];
+#pragma unroll
+        for (int a = 0; a < RPT; ++a)
+#pragma unroll
+          for (int c = 0; c < CPT; ++c) {
+            S[a][c] = fmaf(-tv[a].x, rv[0][c], S[a][c]);
+            S[a][c] = fmaf(-tv[a].y, rv[1][c], S[a][c]);
+            S[a][c] = fmaf(-tv[a].z, rv[2][c], S[a][c]);
+            S[a][c] = fmaf(-tv[a].w, rv[3][c], S[a][c]);
+          }
+      }
+      const int cK = k0 >> 5;
+      const int jk = tx + 32 * cK - k0;   // this lane's column within K, when in [0, NB)
+      const bool lane_in = jk >= 0 && jk < NB;
+      const int jb = min(max(jk, 0), NB - 1);
+#pragma unroll
+      for (int a = 0; a < RPT; ++a)
+#pragma unroll
+        for (int c = 0; c < CPT; ++c)
+          if (c == cK) {
+            const float tk = T[i0 + a][jb];
+            S[a][c] = lane_in ? tk : S[a][c];
+          }
+      if (has_next) publish_rows(kn, nxt);
+    } else if (has_next) {
+      float A[EPL];
+      const int pr_ = lane / LPR, pc = (lane % LPR) * EPL;
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) {
+        float v = Pn[pr_][pc + e];
+#pragma unroll
+        for (int b = 0; b < NB; b += 4) {
+          const float4 t4 = *reinterpret_cast<const float4*>(&T[kn + pr_][b]);
+          v = fmaf(-t4.x, Rk[cur][b + 0][kn + pc + e], v);
+          v = fmaf(-t4.y, Rk[cur][b + 1][kn + pc + e], v);
+          v = fmaf(-t4.z, Rk[cur][b + 2][kn + pc + e], v);
+          v = fmaf(-t4.w, Rk[cur][b + 3][kn + pc + e], v);
+        }
+        A[e] = v;
+      }
+      warp_sweep<NB>(A, lane);
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) Qs[nxt][pr_][pc + e] = -A[e];
+    }
+    __syncthreads();
   }
 
+  if (!tile) return;
   if (MODE == 0) {
 #pragma unroll
     for (int a = 0; a < RPT; ++a) {
@@ -555,7 +633,8 @@ __global__ void __launch_bounds__(512) sweep32_kernel(const float* __restrict__ 
       acc2 = warp_sum(acc2);
       if (lane == 0 && i < w) out[i] = acc2.hi + acc2.lo;
     }
-  }  if (IN_INT) {   // every thread has read its entries (barrier after the last step): reset the upper triangle
+  }
+  if (IN_INT) {   // every thread has read its entries (barrier after the last step): reset the upper triangle
 #pragma unroll
     for (int a = 0; a < RPT; ++a)
 #pragma unroll
@@ -587,7 +666,7 @@ cudaError_t launch_sweep_int_w(int* Gint, int w, const float* GVraw, const float
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  sweep32_kernel<W_PAD, NB, MODE, true><<<1, 512, smem, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint);
+  sweep32_kernel<W_PAD, NB, MODE, true><<<1, 544, smem, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint);
   return cudaGetLastError();
 }
 
@@ -605,9 +684,9 @@ cudaError_t launch_sweep(const float* Gpart, int splits, int w, const float* GVr
                          float* out, cudaStream_t s) {
   // elements per lane RPW * CPL = W_PAD^2 / (32 * NWARP): 4 / 8 / 32 / 64
   // pivot-block sizes measured fastest on GB300: 8 up to w = 64, 16 at w = 128
-  if (w <= 32) sweep32_kernel<32, 8, MODE, false><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
-  else if (w <= 64) sweep32_kernel<64, 8, MODE, false><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
-  else if (w <= 128) sweep32_kernel<128, 16, MODE, false><<<1, 512, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
+  if (w <= 32) sweep32_kernel<32, 8, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
+  else if (w <= 64) sweep32_kernel<64, 8, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
+  else if (w <= 128) sweep32_kernel<128, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
   else sweep_kernel<256, 32, MODE><<<1, 32 * 32, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
   return cudaGetLastError();
 }
