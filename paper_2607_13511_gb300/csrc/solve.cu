@@ -397,24 +397,28 @@ __global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ 
 #pragma unroll
     for (int c = 0; c < CPT; ++c) S[a][c] = 0.f;
   if (IN_INT) {
-    extern __shared__ float mirror[];   // [W_PAD][W_PAD + 1]: mirror[j][i] = G[i][j] for i < j
-    if (tile) {   // every load issued before the first mirror store
+    // stage the integer Gram in shared memory: warp q copies rows q, q + 17, ... with coalesced loads, all of a
+    // thread's loads issued before its first store; then every tile thread reads its entries by symmetry
+    extern __shared__ int Gs[];   // [W_PAD][W_PAD + 1]
+    constexpr int NR = (W_PAD + 16) / 17, NC = W_PAD / 32, QB = 4;   // rows per warp, batches of QB rows
 #pragma unroll
-      for (int a = 0; a < RPT; ++a) {
-        const int i = i0 + a;
+    for (int q0 = 0; q0 < NR; q0 += QB) {
+      int v[QB][NC];
 #pragma unroll
-        for (int c = 0; c < CPT; ++c) {
-          const int j = tx + 32 * c;
-          S[a][c] = (i <= j && j < w) ? (float)Gint[(long long)i * w + j] : 0.f;
+      for (int q = 0; q < QB; ++q) {
+        const int i = warp + 17 * (q0 + q);
+#pragma unroll
+        for (int c = 0; c < NC; ++c) {
+          const int j = lane + 32 * c;
+          v[q][c] = (q0 + q < NR && i < w && j < w) ? Gint[(long long)i * w + j] : 0;
         }
       }
 #pragma unroll
-      for (int a = 0; a < RPT; ++a) {
-        const int i = i0 + a;
+      for (int q = 0; q < QB; ++q) {
+        const int i = warp + 17 * (q0 + q);
+        if (q0 + q < NR && i < W_PAD) {
 #pragma unroll
-        for (int c = 0; c < CPT; ++c) {
-          const int j = tx + 32 * c;
-          if (i < j && j < w) mirror[j * (W_PAD + 1) + i] = S[a][c];
+          for (int c = 0; c < NC; ++c) Gs[i * (W_PAD + 1) + lane + 32 * c] = v[q][c];
         }
       }
     }
@@ -426,7 +430,7 @@ __global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ 
 #pragma unroll
         for (int c = 0; c < CPT; ++c) {
           const int j = tx + 32 * c;
-          if (j < i && i < w) S[a][c] = mirror[i * (W_PAD + 1) + j];
+          S[a][c] = (float)(i <= j ? Gs[i * (W_PAD + 1) + j] : Gs[j * (W_PAD + 1) + i]);
         }
       }
     }
@@ -634,15 +638,10 @@ __global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ 
       if (lane == 0 && i < w) out[i] = acc2.hi + acc2.lo;
     }
   }
-  if (IN_INT) {   // every thread has read its entries (barrier after the last step): reset the upper triangle
-#pragma unroll
-    for (int a = 0; a < RPT; ++a)
-#pragma unroll
-      for (int c = 0; c < CPT; ++c) {
-        const int i = i0 + a, j = tx + 32 * c;
-        if (i <= j && j < w) Gint[(long long)i * w + j] = 0;
-      }
+  if (IN_INT) {   // every thread has read the Gram (barrier after staging): reset it for the next accumulation
+    for (int idx = tid; idx < w * w; idx += 512) Gint[idx] = 0;   // tile threads (tid < 512) only
   }
+
 }
 
 int gram_chunk(int w, int L, int* splits) {
@@ -658,7 +657,7 @@ int gram_chunk(int w, int L, int* splits) {
 template <int W_PAD, int NB, int MODE>
 cudaError_t launch_sweep_int_w(int* Gint, int w, const float* GVraw, const float* r, float* Graw, float* out,
                                cudaStream_t s) {
-  const size_t smem = (size_t)W_PAD * (W_PAD + 1) * sizeof(float);   // the lower-triangle mirror
+  const size_t smem = (size_t)W_PAD * (W_PAD + 1) * sizeof(int);   // the staged integer Gram
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(sweep32_kernel<W_PAD, NB, MODE, true>,
