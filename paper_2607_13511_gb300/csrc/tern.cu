@@ -68,16 +68,18 @@ __global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X,
                                                     Thresh th, int8_t* __restrict__ T, long long ldt,
                                                     int* __restrict__ gram, int P, __half* __restrict__ T16,
                                                     long long ldt16, __half* __restrict__ Tk, long long ldk) {
-  constexpr int PPT = (VB * VB) / 256 > 0 ? (VB * VB) / 256 : 1;   // Gram pairs per thread
+  // Gram pairs a <= b, folded: row f and row VB-1-f together hold VB+1 pairs; FR = VB/2 folded rows, NPART
+  // threads per folded row, PPT pairs per thread (strided along the folded row)
+  constexpr int FR = VB / 2, NPART = 256 / FR, PPT = (VB + 1 + NPART - 1) / NPART;
   constexpr int IT = VB / 4;                                      // warp passes per 64-position chunk
   constexpr int KLD = VB + 8;                                     // sK row (halves): 16-byte rows, 4-way stores
-  __shared__ unsigned mpos[VB][2], mneg[VB][2];
+  __shared__ unsigned mnz[VB][2], mpos[VB][2];   // per 64-position chunk: nonzero and positive bitplanes
   __shared__ __align__(16) __half sK[64][KLD];                    // the chunk as [position][component]
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int v0 = blockIdx.y * VB;
   const int nvb = min(VB, nv - v0);
   const int xbeg = blockIdx.x * P, xend = min(L, xbeg + P);
-  const int ga = tid % VB, gb0 = (tid / VB) * PPT;
+  const int gf = tid % FR, gpart = tid / FR;
   int acc[PPT];
 #pragma unroll
   for (int k = 0; k < PPT; ++k) acc[k] = 0;
@@ -113,10 +115,10 @@ __global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X,
           if (T16 != nullptr) T16[(long long)v * ldt16 + x] = __short2half_rn((short)t);
         }
         if (GRAM) {
-          const unsigned pm = __ballot_sync(0xffffffffu, t > 0), nm = __ballot_sync(0xffffffffu, t < 0);
+          const unsigned zm = __ballot_sync(0xffffffffu, t != 0), pm = __ballot_sync(0xffffffffu, t > 0);
           if (lane == 0) {
+            mnz[a][half] = zm;
             mpos[a][half] = pm;
-            mneg[a][half] = nm;
           }
         }
         if (Tk != nullptr) sK[32 * half + lane][a] = __short2half_rn((short)t);
@@ -134,15 +136,25 @@ __global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X,
       __syncthreads();
     }
     if (GRAM) {
+      // G_ab += popc(Z_a & Z_b) - 2 popc(Z_a & Z_b & (P_a ^ P_b)): both nonzero, minus twice the opposite signs
       __syncthreads();
-      const unsigned long long pa = mpos[ga][0] | ((unsigned long long)mpos[ga][1] << 32);
-      const unsigned long long na = mneg[ga][0] | ((unsigned long long)mneg[ga][1] << 32);
+      const int a1 = gf, a2 = VB - 1 - gf;
+      const unsigned long long z1 = mnz[a1][0] | ((unsigned long long)mnz[a1][1] << 32);
+      const unsigned long long p1 = mpos[a1][0] | ((unsigned long long)mpos[a1][1] << 32);
+      const unsigned long long z2 = mnz[a2][0] | ((unsigned long long)mnz[a2][1] << 32);
+      const unsigned long long p2 = mpos[a2][0] | ((unsigned long long)mpos[a2][1] << 32);
 #pragma unroll
       for (int k = 0; k < PPT; ++k) {
-        const int b = gb0 + k;
-        const unsigned long long pb = mpos[b][0] | ((unsigned long long)mpos[b][1] << 32);
-        const unsigned long long nb = mneg[b][0] | ((unsigned long long)mneg[b][1] << 32);
-        acc[k] += __popcll(pa & pb) + __popcll(na & nb) - __popcll(pa & nb) - __popcll(na & pb);
+        const int e = gpart + NPART * k;          // position along the folded row
+        const bool first = e < VB - gf;
+        const int b = first ? gf + e : a2 + (e - (VB - gf));
+        if (e <= VB) {
+          const unsigned long long zb = mnz[b][0] | ((unsigned long long)mnz[b][1] << 32);
+          const unsigned long long pb = mpos[b][0] | ((unsigned long long)mpos[b][1] << 32);
+          const unsigned long long zz = (first ? z1 : z2) & zb;
+          const unsigned long long dd = zz & ((first ? p1 : p2) ^ pb);
+          acc[k] += __popcll(zz) - 2 * __popcll(dd);
+        }
       }
       __syncthreads();
     }
@@ -150,8 +162,11 @@ __global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X,
   if (GRAM) {
 #pragma unroll
     for (int k = 0; k < PPT; ++k) {
-      const int b = gb0 + k;
-      if (ga < nvb && b < nvb && ga <= b && acc[k] != 0) atomicAdd(&gram[(long long)ga * nv + b], acc[k]);
+      const int e = gpart + NPART * k;
+      const bool first = e < VB - gf;
+      const int a = first ? gf : VB - 1 - gf;
+      const int b = first ? gf + e : VB - 1 - gf + (e - (VB - gf));
+      if (e <= VB && a < nvb && b < nvb && acc[k] != 0) atomicAdd(&gram[(long long)a * nv + b], acc[k]);
     }
   }
 }
