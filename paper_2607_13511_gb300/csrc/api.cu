@@ -237,6 +237,7 @@ struct Bufs {
   float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE, *maxpart, *maxabs, *theta;
   unsigned *err, *arg, *ticket;
   int *fallback, *GintU, *GintV;
+  GramScratch gram;   // per-CTA partials and group tickets of the fused Gram
   int8_t *Ut, *Vt;
   __half *Ut16, *Vt16;   // fp16 copies of Ut, Vt for the tensor-core products (nullptr when unused)
   __half *Uk16, *Vk16;   // K-major fp16 copies of the final U, V of a block for the tensor-core deflation
@@ -279,6 +280,13 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "ticket", 1, &B->ticket, true));
   TRY(need(ws, "GintU", (size_t)w * w, &B->GintU, true));
   TRY(need(ws, "GintV", (size_t)w * w, &B->GintV, true));
+  {
+    size_t pm, gm, pn, gn;
+    apply_gram_scratch(p.m, &pm, &gm);
+    apply_gram_scratch(p.n, &pn, &gn);
+    TRY(need(ws, "gram.part", std::max(pm, pn), &B->gram.part));
+    TRY(need(ws, "gram.ticket", std::max(gm, gn), &B->gram.ticket, true));
+  }
   TRY(need(ws, "X", (size_t)w * L, &B->X));
   TRY(need(ws, "spart", (size_t)w * std::max(p.nchunk_m, p.nchunk_n), &B->spart));
   TRY(need(ws, "Gpart", (size_t)std::max(p.gm, p.gn) * w * w, &B->Gpart));
@@ -381,7 +389,7 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
     __half* const U16 = use_tc(w) ? B.Ut16 : nullptr;
     __half* const V16 = use_tc(w) ? B.Vt16 : nullptr;
     KL(kApply, 1, launch_apply(B.X, w, m, m, th_m, B.Ut, (int)p.ldm, (fusedU && w > 1) ? B.GintU : nullptr, s, U16,
-                               p.ldm));
+                               p.ldm, nullptr, 0, B.gram));
     for (int it = 0; it < p.iters; ++it) {
       const bool last = it == p.iters - 1;
       // V-step: V <- T([(U^T U + eps I)^-1 U^T R]^T)   (plain R even when weighted, §2.5).
@@ -399,7 +407,7 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
       if (w > 1) JOIN();
       KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, sv, n, B.X, n, st_n, s));
       KL(kApply, 1, launch_apply(B.X, w, n, n, th_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, s, V16, p.ldn,
-                                 (last && use_tc(w)) ? B.Vk16 : nullptr, B.ldk));
+                                 (last && use_tc(w)) ? B.Vk16 : nullptr, B.ldk, B.gram));
       // U-step: U <- T(R H V (V^T H V + eps I)^-1)
       FORK();
       if (fusedV) {
@@ -414,7 +422,8 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
       // the next V-step's inverse (w > 1) or, after the last iteration, Eq. 4 consumes U's Gram
       // (the fp16 copy of U is not needed after the last iteration)
       KL(kApply, 1, launch_apply(B.X, w, m, m, th_m, B.Ut, (int)p.ldm, (fusedU && (w > 1 || last)) ? B.GintU : nullptr,
-                                 s, last ? nullptr : U16, p.ldm, (last && use_tc(w)) ? B.Uk16 : nullptr, B.ldk));
+                                 s, last ? nullptr : U16, p.ldm, (last && use_tc(w)) ? B.Uk16 : nullptr, B.ldk,
+                                 B.gram));
     }
     // Eq. 4: [(U^T U) .* (V^T H V)] d = diag(U^T R H V), with R H V the last U-step product
     KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, su, B.r, s));

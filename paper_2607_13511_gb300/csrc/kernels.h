@@ -178,9 +178,17 @@ cudaError_t launch_stats(const float* X, int nv, int L, int ldx, Stats st, cudaS
 // must hold zeros or a running sum).
 // T16 (optional): the same ternary values as fp16 rows with leading dimension ldt16. Tk (optional): as fp16 in
 // K-major layout, Tk[x * ldk + a] for a < nv (ldk a multiple of 8, >= round_up(nv, 8); 16-byte aligned).
+// With gram (nv <= 128) the exact integer Gram is added into its upper triangle; gs then holds the per-CTA
+// partials and the zero-initialized group tickets, sized by apply_gram_scratch for the vectors' length L.
+constexpr int kGramGroup = 8;   // CTAs whose partials one CTA sums before the atomics
+struct GramScratch {
+  int* part = nullptr;
+  unsigned* ticket = nullptr;
+};
+void apply_gram_scratch(int L, size_t* part_ints, size_t* groups);
 cudaError_t launch_apply(const float* X, int nv, int L, int ldx, const Thresh& th, int8_t* T, int ldt, int* gram,
                          cudaStream_t s, __half* T16 = nullptr, long long ldt16 = 0, __half* Tk = nullptr,
-                         long long ldk = 0);
+                         long long ldk = 0, GramScratch gs = GramScratch{});
 cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, float* Y, int ldy, Stats st,
                           cudaStream_t s);
 // J = the w columns of largest h_c * sum_t colpart[t][c] (ties to the lower c), ascending; e (n floats) is scratch.

@@ -67,7 +67,8 @@ template <int VB, bool GRAM>
 __global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X, int nv, int L, long long ldx,
                                                     Thresh th, int8_t* __restrict__ T, long long ldt,
                                                     int* __restrict__ gram, int P, __half* __restrict__ T16,
-                                                    long long ldt16, __half* __restrict__ Tk, long long ldk) {
+                                                    long long ldt16, __half* __restrict__ Tk, long long ldk,
+                                                    GramScratch gs) {
   // Gram pairs a <= b, folded: row f and row VB-1-f together hold VB+1 pairs; FR = VB/2 folded rows, NPART
   // threads per folded row, PPT pairs per thread (strided along the folded row)
   constexpr int FR = VB / 2, NPART = 256 / FR, PPT = (VB + 1 + NPART - 1) / NPART;
@@ -160,13 +161,60 @@ __global__ void __launch_bounds__(256) apply_kernel(const float* __restrict__ X,
     }
   }
   if (GRAM) {
-#pragma unroll
-    for (int k = 0; k < PPT; ++k) {
+    // Few CTAs: every CTA adds its partials atomically. Many CTAs (gs.part given): each CTA stores its partials
+    // (slot-major, coalesced) and the last CTA of every group of kGramGroup consecutive CTAs (acquire-release
+    // ticket, as for the statistics) sums the group's partials, four slots of loads in flight at a time, and adds
+    // them, so one atomic per slot and group reaches L2.
+    auto pair_of = [&](int k, int& a, int& b) {
       const int e = gpart + NPART * k;
       const bool first = e < VB - gf;
-      const int a = first ? gf : VB - 1 - gf;
-      const int b = first ? gf + e : VB - 1 - gf + (e - (VB - gf));
-      if (e <= VB && a < nvb && b < nvb && acc[k] != 0) atomicAdd(&gram[(long long)a * nv + b], acc[k]);
+      a = first ? gf : VB - 1 - gf;
+      b = first ? gf + e : VB - 1 - gf + (e - (VB - gf));
+      return e <= VB;
+    };
+    if (gs.part == nullptr) {
+#pragma unroll
+      for (int k = 0; k < PPT; ++k) {
+        int a, b;
+        if (pair_of(k, a, b) && a < nvb && b < nvb && acc[k] != 0) atomicAdd(&gram[(long long)a * nv + b], acc[k]);
+      }
+    } else {
+      __shared__ int s_last_g;
+      int* mine = gs.part + (long long)blockIdx.x * PPT * 256;
+#pragma unroll
+      for (int k = 0; k < PPT; ++k) mine[k * 256 + tid] = acc[k];
+      __syncthreads();
+      const int grp = blockIdx.x / kGramGroup, g0 = grp * kGramGroup;
+      const int gn = min(kGramGroup, (int)gridDim.x - g0);
+      if (tid == 0) {
+        unsigned old;
+        asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(gs.ticket + grp) : "memory");
+        s_last_g = (old == (unsigned)gn - 1u);
+      }
+      __syncthreads();
+      if (s_last_g) {
+        constexpr int KB = PPT < 4 ? PPT : 4;
+        const int* base = gs.part + (long long)g0 * PPT * 256;
+#pragma unroll 1
+        for (int k0 = 0; k0 < PPT; k0 += KB) {
+          int v[KB][kGramGroup];
+#pragma unroll
+          for (int q = 0; q < KB; ++q)
+#pragma unroll
+            for (int c = 0; c < kGramGroup; ++c)
+              v[q][c] = (k0 + q < PPT && c < gn) ? base[((long long)c * PPT + k0 + q) * 256 + tid] : 0;
+#pragma unroll
+          for (int q = 0; q < KB; ++q) {
+            int sum = 0;
+#pragma unroll
+            for (int c = 0; c < kGramGroup; ++c) sum += v[q][c];
+            int a, b;
+            if (k0 + q < PPT && pair_of(k0 + q, a, b) && a < nvb && b < nvb && sum != 0)
+              atomicAdd(&gram[(long long)a * nv + b], sum);
+          }
+        }
+        if (tid == 0) gs.ticket[grp] = 0u;
+      }
     }
   }
 }
@@ -389,20 +437,40 @@ cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, flo
   return cudaGetLastError();
 }
 
-cudaError_t launch_apply(const float* X, int nv, int L, int ldx, const Thresh& th, int8_t* T, int ldt, int* gram,
-                         cudaStream_t s, __half* T16, long long ldt16, __half* Tk, long long ldk) {
-  if (Tk != nullptr && (ldk < round_up(nv, 8) || (ldk & 7) != 0)) return cudaErrorInvalidValue;
-  // one 64-position chunk per CTA up to one CTA per SM, whole chunks per CTA beyond
+namespace {
+// the apply grid: P positions per CTA, gx CTAs
+void apply_grid(int L, int* P, int* gx) {
   int sms = 152, dev = 0;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int P = 64 * (int)std::max<long long>(1, cdiv(L, 64LL * sms));
-  const int gx = (int)cdiv(L, P);
+  *P = 64 * (int)std::max<long long>(1, cdiv(L, 64LL * sms));
+  *gx = (int)cdiv(L, *P);
+}
+}  // namespace
+
+void apply_gram_scratch(int L, size_t* part_ints, size_t* groups) {
+  int P, gx;
+  apply_grid(L, &P, &gx);
+  *part_ints = (size_t)gx * 256 * 33;   // PPT <= 33 (128 vectors)
+  *groups = (size_t)cdiv(gx, kGramGroup);
+}
+
+cudaError_t launch_apply(const float* X, int nv, int L, int ldx, const Thresh& th, int8_t* T, int ldt, int* gram,
+                         cudaStream_t s, __half* T16, long long ldt16, __half* Tk, long long ldk, GramScratch gs) {
+  if (Tk != nullptr && (ldk < round_up(nv, 8) || (ldk & 7) != 0)) return cudaErrorInvalidValue;
+  // one 64-position chunk per CTA up to one CTA per SM, whole chunks per CTA beyond
+  int P, gx;
+  apply_grid(L, &P, &gx);
   const bool g = gram != nullptr && nv <= 128;   // 256 vectors would need 256 accumulators per thread
+  if (g && (gs.part == nullptr || gs.ticket == nullptr)) return cudaErrorInvalidValue;
+  // the grouped reduction pays off once the direct atomics (one per pair and CTA) would number ~400K or more
+  if ((long long)gx * nv * (nv + 1) / 2 < 400000) gs = GramScratch{};
 #define APPLY_LAUNCH(VB)                                                                                 \
   do {                                                                                                   \
     dim3 grid((unsigned)gx, (unsigned)cdiv(nv, VB));                                                     \
-    if (g) apply_kernel<VB, true><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, gram, P, T16, ldt16, Tk, ldk);  \
-    else apply_kernel<VB, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16, Tk, ldk); \
+    if (g) apply_kernel<VB, true><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, gram, P, T16, ldt16, Tk, ldk,   \
+                                                         gs);                                                \
+    else apply_kernel<VB, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16, Tk, ldk, \
+                                                      GramScratch{});                                        \
   } while (0)
   if (nv <= 16) APPLY_LAUNCH(16);
   else if (nv <= 32) APPLY_LAUNCH(32);
@@ -410,7 +478,8 @@ cudaError_t launch_apply(const float* X, int nv, int L, int ldx, const Thresh& t
   else if (nv <= 128) APPLY_LAUNCH(128);
   else {
     dim3 grid((unsigned)gx, (unsigned)cdiv(nv, 256));
-    apply_kernel<256, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16, Tk, ldk);
+    apply_kernel<256, false><<<grid, 256, 0, s>>>(X, nv, L, ldx, th, T, ldt, nullptr, P, T16, ldt16, Tk, ldk,
+                                                  GramScratch{});
   }
 #undef APPLY_LAUNCH
   return cudaGetLastError();
