@@ -332,7 +332,7 @@ Plan make_plan(long long m, long long n, long long k, int block, int iters, doub
 // A kernel launch of class `kind` that launches `nk` kernels: counted, and bracketed by events when profiled.
 #define KLS(kind_, nk, st_, call)                           \
   do {                                                      \
-    const bool prof_ = g_prof.kind == (kind_);              \
+    const bool prof_ = g_prof.kind != 0 && g_prof.kind == (kind_); \
     if (prof_) LK(prof_mark(st_));                          \
     LK(call);                                               \
     if (prof_) LK(prof_mark(st_));                          \
@@ -388,6 +388,7 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
     KL(kStart, 1, launch_gather(B.R, m, n, B.J, w, B.X, m, st_g, s));
     __half* const U16 = use_tc(w) ? B.Ut16 : nullptr;
     __half* const V16 = use_tc(w) ? B.Vt16 : nullptr;
+    if (blk > 0) JOIN();   // the previous block's outputs (side branch) have read Ut, Vt and d
     KL(kApply, 1, launch_apply(B.X, w, m, m, th_m, B.Ut, (int)p.ldm, (fusedU && w > 1) ? B.GintU : nullptr, s, U16,
                                p.ldm, nullptr, 0, B.gram));
     for (int it = 0; it < p.iters; ++it) {
@@ -425,6 +426,12 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
                                  s, last ? nullptr : U16, p.ldm, (last && use_tc(w)) ? B.Uk16 : nullptr, B.ldk,
                                  B.gram));
     }
+    // The block's outputs leave on the side branch: B from the final U and C from the final V now, D after the
+    // scales; the next block joins before it overwrites Ut.
+    FORK();
+    KLS(0, 1, side, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, side));
+    LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
+                         cudaMemcpyDeviceToDevice, side));
     // Eq. 4: [(U^T U) .* (V^T H V)] d = diag(U^T R H V), with R H V the last U-step product
     KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, su, B.r, s));
     if (fusedU) {
@@ -433,6 +440,8 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
       KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
       KL(kSolve, 1, launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s));
     }
+    FORK();
+    LK(cudaMemcpyAsync(Dout + j0, B.d, sizeof(float) * w, cudaMemcpyDeviceToDevice, side));
     // R <- R - U diag(d) V^T
     if (use_tc(w)) {
       KL(kDeflate, 1, launch_deflate_tc(B.R, m, n, B.Uk16, B.Vk16, B.ldk, B.d, w, h, B.colpart, B.normpart, B.maxpart,
@@ -442,11 +451,8 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
                                      B.normpart, s, B.maxpart));
     }
     KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_r, B.norm_a, B.trace + blk, s, B.maxpart, B.maxabs));
-    KL(0, 1, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, s));
-    LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
-                         cudaMemcpyDeviceToDevice, s));
-    LK(cudaMemcpyAsync(Dout + j0, B.d, sizeof(float) * w, cudaMemcpyDeviceToDevice, s));
   }
+  if (p.nblocks > 0) JOIN();
   return EXTERND_OK;
 }
 
