@@ -673,7 +673,7 @@ template <int MODE>
 cudaError_t launch_sweep_int(int* Gint, int w, const float* GVraw, const float* r, float* Graw, float* out,
                              cudaStream_t s) {
   if (w <= 32) return launch_sweep_int_w<32, 8, MODE>(Gint, w, GVraw, r, Graw, out, s);
-  if (w <= 64) return launch_sweep_int_w<64, 8, MODE>(Gint, w, GVraw, r, Graw, out, s);
+  if (w <= 64) return launch_sweep_int_w<64, 16, MODE>(Gint, w, GVraw, r, Graw, out, s);
   if (w <= 128) return launch_sweep_int_w<128, 16, MODE>(Gint, w, GVraw, r, Graw, out, s);
   return cudaErrorInvalidValue;   // callers use the float-partial Gram above 128 components
 }
@@ -684,7 +684,7 @@ cudaError_t launch_sweep(const float* Gpart, int splits, int w, const float* GVr
   // elements per lane RPW * CPL = W_PAD^2 / (32 * NWARP): 4 / 8 / 32 / 64
   // pivot-block sizes measured fastest on GB300: 8 up to w = 64, 16 at w = 128
   if (w <= 32) sweep32_kernel<32, 8, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
-  else if (w <= 64) sweep32_kernel<64, 8, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
+  else if (w <= 64) sweep32_kernel<64, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
   else if (w <= 128) sweep32_kernel<128, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
   else sweep_kernel<256, 32, MODE><<<1, 32 * 32, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
   return cudaGetLastError();
