@@ -148,6 +148,26 @@ int externd_block_scales(const float *R, int64_t m, int64_t n, const int8_t *U, 
 int externd_deflate(float *R, int64_t m, int64_t n, const int8_t *U, const float *d, const int8_t *Cb, int64_t w,
                     const float *weights, double *norm2);
 
+/* ---- Inference with the factors (§2.6, Eq. 5) ----------------------------------------------------------- */
+
+/* Packs a ternary matrix for externd_ternary_apply. T: rows x cols int8 in {-1, 0, 1}, row-major with leading
+ * dimension ldt >= cols (device). Each entry becomes a 2-bit code (bit 0: nonzero, bit 1: negative), i.e. the
+ * mask and sign bits of §2.6 at a fixed position, laid out for the tensor-core product: words (device,
+ * caller-allocated) holds ceil(rows / 16) * ceil(cols / 128) * 128 uint32 words; word
+ * ((rt * ceil(cols / 128) + grp) * 32 + lane) * 4 + q, lane = 4 g + t, carries at bits 14 - 2p (low element)
+ * and 30 - 2p (high element), p = 0..7, the codes of row 16 rt + g + 8 (p & 1) and columns
+ * 128 grp + 16 (2 q + p / 4) + 8 ((p & 3) >> 1) + 2 t and + 1; entries past rows or cols are zero. If nnz != NULL
+ * it receives (host) the number of nonzeros, from which Eq. 5's storage of the sparse mask+sign form follows:
+ * rows * cols mask bits plus nnz sign bits. Synchronous only when nnz != NULL. */
+int externd_pack_ternary(const int8_t *T, int64_t rows, int64_t cols, int64_t ldt, uint32_t *words, int64_t *nnz);
+
+/* §2.6: y = B diag(D) (C x) with B (m x k) and C (k x n) packed by externd_pack_ternary; D (k), x (n) and
+ * y (m) float32, all device pointers; the intermediate D (C x) stays in the library's workspace. Each product
+ * runs on the tensor cores with the vector split exactly into three bf16 parts, so the result is the exact one up
+ * to fp32 accumulation. Asynchronous on the library stream. */
+int externd_ternary_apply(const uint32_t *Bp, const float *D, const uint32_t *Cp, int64_t m, int64_t k, int64_t n,
+                          const float *x, float *y);
+
 #ifdef __cplusplus
 }
 #endif

@@ -16,7 +16,8 @@ from typing import Optional
 __all__ = [
     "ExterndError", "Decomposition", "library_path", "load", "rank", "block_width", "decompose", "decompose_host",
     "energy", "ternarize", "vstep_product", "ustep_product", "vstep_target", "ustep_target", "block_scales",
-    "deflate", "profile", "profile_read", "kernel_launches", "PROFILE_KINDS",
+    "deflate", "profile", "profile_read", "kernel_launches", "PROFILE_KINDS", "Packed", "pack_ternary",
+    "ternary_apply",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -50,6 +51,8 @@ _SIGNATURES = {
     "externd_ustep_target": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_i64, _c_void, _c_void]),
     "externd_block_scales": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_i64, _c_void, _c_void]),
     "externd_deflate": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_void, _c_i64, _c_void, _c_dptr]),
+    "externd_pack_ternary": (_c_int, [_c_void, _c_i64, _c_i64, _c_i64, _c_void, ctypes.POINTER(_c_i64)]),
+    "externd_ternary_apply": (_c_int, [_c_void, _c_void, _c_void, _c_i64, _c_i64, _c_i64, _c_void, _c_void]),
 }
 
 
@@ -300,3 +303,45 @@ def deflate(R, U, d, Cb, weights=None) -> float:
         _check(lib.externd_deflate(_ptr(R), m, n, _ptr(U), _ptr(d), _ptr(Cb), U.shape[1], _ptr(h),
                                    ctypes.byref(out)))
     return out.value
+
+
+@dataclass
+class Packed:
+    """A ternary matrix in the library's packed form (§2.6): ``words`` is a (ceil(rows/16), ceil(cols/128), 32, 4)
+    int32 tensor of 2-bit codes (bit 0 nonzero, bit 1 negative) in tensor-core fragment order (layout in
+    include/externd.h); ``nnz`` is the number of nonzeros."""
+    words: object
+    rows: int
+    cols: int
+    nnz: int
+
+
+def pack_ternary(T) -> Packed:
+    """Packs a CUDA int8 ternary matrix; ``nnz`` gives Eq. 5's storage (rows*cols mask bits + nnz sign bits)."""
+    torch = _torch()
+    lib = load()
+    T = _prep(T, torch.int8, "T")
+    rows, cols = T.shape
+    words = torch.empty(((rows + 15) // 16, (cols + 127) // 128, 32, 4), dtype=torch.int32, device=T.device)
+    nnz = _c_i64()
+    with torch.cuda.device(T.device):
+        _stream(lib, T.device)
+        _check(lib.externd_pack_ternary(_ptr(T), rows, cols, cols, _ptr(words), ctypes.byref(nnz)))
+    return Packed(words, rows, cols, nnz.value)
+
+
+def ternary_apply(Bp: Packed, D, Cp: Packed, x):
+    """§2.6: y = B diag(D) (C x) from the packed factors; x is a CUDA float32 vector of length n."""
+    torch = _torch()
+    lib = load()
+    m, k, n = Bp.rows, Bp.cols, Cp.cols
+    if Cp.rows != k:
+        raise ExterndError(f"inner ranks differ: B has {k} columns, C has {Cp.rows} rows")
+    D, x = _prep(D, torch.float32, "D"), _prep(x, torch.float32, "x")
+    if D.numel() != k or x.numel() != n:
+        raise ExterndError("D must have k entries and x n entries")
+    y = torch.empty((m,), dtype=torch.float32, device=x.device)
+    with torch.cuda.device(x.device):
+        _stream(lib, x.device)
+        _check(lib.externd_ternary_apply(_ptr(Bp.words), _ptr(D), _ptr(Cp.words), m, k, n, _ptr(x), _ptr(y)))
+    return y

@@ -986,6 +986,53 @@ int externd_deflate(float* R, int64_t m, int64_t n, const int8_t* U, const float
   return EXTERND_OK;
 }
 
+int externd_pack_ternary(const int8_t* T, int64_t rows, int64_t cols, int64_t ldt, uint32_t* words, int64_t* nnz) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (rows < 1 || cols < 1 || ldt < cols || rows > (1LL << 31) || cols > (1LL << 31) ||
+      packed_words(rows, cols) > (1LL << 36))
+    return EXTERND_EINVAL;
+  TRY(check_dev(T));
+  TRY(check_dev(words));
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  unsigned long long* cnt;
+  TRY(need(*ws, "pack.nnz", 1, &cnt));
+  LK(cudaMemsetAsync(cnt, 0, sizeof(unsigned long long), g_stream));
+  LK(launch_pack_ternary(T, rows, cols, ldt, words, cnt, g_stream));
+  if (nnz != nullptr) {
+    void* hb;
+    TRY(need_host(*ws, sizeof(unsigned long long), &hb));
+    CK(cudaMemcpyAsync(hb, cnt, sizeof(unsigned long long), cudaMemcpyDeviceToHost, g_stream));
+    CK(cudaStreamSynchronize(g_stream));
+    *nnz = (int64_t)(*static_cast<unsigned long long*>(hb));
+  }
+  return EXTERND_OK;
+}
+
+int externd_ternary_apply(const uint32_t* Bp, const float* D, const uint32_t* Cp, int64_t m, int64_t k, int64_t n,
+                          const float* x, float* y) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (m < 1 || k < 1 || n < 1 || m > (1LL << 31) || k > (1LL << 31) || n > (1LL << 31)) return EXTERND_EINVAL;
+  TRY(check_dev(Bp));
+  TRY(check_dev(D));
+  TRY(check_dev(Cp));
+  TRY(check_dev(x));
+  TRY(check_dev(y));
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  float *z, *part = nullptr;
+  unsigned* ticket = nullptr;
+  TRY(need(*ws, "apply.z", (size_t)k, &z));
+  const long long np = std::max(gemv_partial_floats(k, n), gemv_partial_floats(m, k));
+  if (np > 0) {
+    TRY(need(*ws, "apply.part", (size_t)np, &part));
+    TRY(need(*ws, "apply.ticket", (size_t)std::max(gemv_tickets(k), gemv_tickets(m)), &ticket, true));
+  }
+  LK(launch_ternary_gemv(Cp, k, n, x, D, z, part, ticket, g_stream));         // z = D (.) (C x)
+  LK(launch_ternary_gemv(Bp, m, k, z, nullptr, y, part, ticket, g_stream));   // y = B z
+  return EXTERND_OK;
+}
+
 }  // extern "C"
 
 // Accessors for other translation units of the library (the stream, lock and error text above).
