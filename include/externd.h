@@ -148,6 +148,55 @@ int externd_block_scales(const float *R, int64_t m, int64_t n, const int8_t *U, 
 int externd_deflate(float *R, int64_t m, int64_t n, const int8_t *U, const float *d, const int8_t *Cb, int64_t w,
                     const float *weights, double *norm2);
 
+/* ---- Extensions of the block loop ------------------------------------------------------------------------- */
+
+/* externd_decompose with the convergence safeguard of Prop. 2 (appendix): before each block is deflated, what it
+ * removes from the weighted squared residual, 2 r^T d - d^T K d (r_a = u_a^T R H v_a, K = (U^T U) .* (V^T H V)), is
+ * compared with what the best single-entry pair removes, max_ij h_j R_ij^2 (ties to the lower row-major index);
+ * when the pair removes more, the block becomes u = e_i, v = sgn(R_ij) e_j, d = |R_ij| followed by w - 1 zero
+ * components (zero columns of B, rows of C, entries of D). With b = 1 this is Prop. 2 as stated, and
+ * ||R_k||^2 <= (1 - 1/(mn))^k ||A||^2 after every component. *activations (host, required) receives the number of
+ * blocks replaced. Arguments and errors otherwise as externd_decompose. */
+int externd_decompose_safeguarded(const float *A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
+                                  const float *weights, int8_t *B, float *D, int8_t *C, double *energy, double *trace,
+                                  int64_t *activations);
+
+/* Refinement sweeps (§2.4) of factors B (m x k), D (k), C (k x n) -- device memory, updated in place -- laid out
+ * in blocks of b = min(block, floor(min(m, n) / 8)) components as externd_decompose writes them. Each sweep visits
+ * the blocks in order: the block is added back to the residual R = A - B D C, refitted by `iters` ALS iterations
+ * warm-started from its own U (no column selection), and replaced by the refit only if the refit removes at least
+ * as much from the added-back residual as the block did; then the kept block is deflated. The energy therefore
+ * never decreases. energy (host, or NULL): the final energy; trace (host, sweeps doubles, or NULL): the energy
+ * after each sweep; replaced (host, sweeps entries, or NULL): blocks replaced per sweep. EXTERND_EINVAL for
+ * k < 1, sweeps < 1 or the parameter errors of externd_decompose. Synchronous. */
+int externd_refine(const float *A, int64_t m, int64_t n, double tau, int block, int iters, int sweeps,
+                   const float *weights, int8_t *B, float *D, int8_t *C, int64_t k, double *energy, double *trace,
+                   int64_t *replaced);
+
+/* ---- Rank and storage budgets from the energy trace (host only; no device work) ------------------------- */
+
+/* The inner ranks at which a run at (m, n, mu, block) finishes a block (§2.4): b, 2b, ..., k (the last one
+ * capped at k), i.e. the ranks the entries of the decompose call's energy trace belong to. With ranks == NULL only
+ * *count is written (the number of blocks); otherwise *count must hold the capacity of ranks and receives the
+ * number written. Errors as externd_rank / externd_block_width, or EXTERND_EINVAL if the capacity is short. */
+int externd_block_boundaries(int64_t m, int64_t n, double mu, int block, int64_t *ranks, int64_t *count);
+
+/* Smallest block-boundary rank whose energy reaches target, from the trace of one run at (m, n, mu, block):
+ * greedy deflation (§2.3, §2.4) makes a run at a smaller rank the prefix of this one, so the trace gives E(k) for
+ * every smaller run (the equal-energy comparisons of §3 then use mu = k / min(m, n)). ntrace must equal the
+ * number of blocks. *k = 0 when the run never reaches target. */
+int externd_rank_for_energy(int64_t m, int64_t n, double mu, int block, const double *trace, int64_t ntrace,
+                            double target, int64_t *k);
+
+/* Per-matrix rank allocation under a storage budget (§5): matrix j has npts[j] points (k, E_j(k)) at its block
+ * boundaries, stored consecutively in ks (strictly increasing per matrix) and energies; taking matrix j to rank
+ * k costs costs[j] * k (> 0, e.g. (m + n) bits of mask per component); weights (or NULL for 1) scale each
+ * matrix's energy. Greedy: repeatedly the next block of the matrix with the largest weighted energy gain per
+ * unit cost that still fits (ties to the lower index; optimal when every curve is concave). chosen[j] receives
+ * the rank of matrix j (0 for none). EXTERND_EINVAL on bad sizes, non-increasing ks or non-finite values. */
+int externd_allocate_ranks(int64_t nmat, const int64_t *npts, const int64_t *ks, const double *energies,
+                           const double *costs, const double *weights, double budget, int64_t *chosen);
+
 /* ---- Inference with the factors (§2.6, Eq. 5) ----------------------------------------------------------- */
 
 /* Packs a ternary matrix for externd_ternary_apply. T: rows x cols int8 in {-1, 0, 1}, row-major with leading

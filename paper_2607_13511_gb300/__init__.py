@@ -17,7 +17,7 @@ __all__ = [
     "ExterndError", "Decomposition", "library_path", "load", "rank", "block_width", "decompose", "decompose_host",
     "energy", "ternarize", "vstep_product", "ustep_product", "vstep_target", "ustep_target", "block_scales",
     "deflate", "profile", "profile_read", "kernel_launches", "PROFILE_KINDS", "Packed", "pack_ternary",
-    "ternary_apply",
+    "ternary_apply", "block_boundaries", "rank_for_energy", "allocate_ranks", "decompose_safeguarded", "refine",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -51,6 +51,17 @@ _SIGNATURES = {
     "externd_ustep_target": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_i64, _c_void, _c_void]),
     "externd_block_scales": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_i64, _c_void, _c_void]),
     "externd_deflate": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_void, _c_i64, _c_void, _c_dptr]),
+    "externd_decompose_safeguarded": (_c_int, [_c_void, _c_i64, _c_i64, _c_double, _c_double, _c_int, _c_int,
+                                               _c_void, _c_void, _c_void, _c_void, _c_dptr, _c_dptr,
+                                               ctypes.POINTER(_c_i64)]),
+    "externd_refine": (_c_int, [_c_void, _c_i64, _c_i64, _c_double, _c_int, _c_int, _c_int, _c_void, _c_void,
+                                _c_void, _c_void, _c_i64, _c_dptr, _c_dptr, ctypes.POINTER(_c_i64)]),
+    "externd_block_boundaries": (_c_int, [_c_i64, _c_i64, _c_double, _c_int, ctypes.POINTER(_c_i64),
+                                          ctypes.POINTER(_c_i64)]),
+    "externd_rank_for_energy": (_c_int, [_c_i64, _c_i64, _c_double, _c_int, _c_dptr, _c_i64, _c_double,
+                                         ctypes.POINTER(_c_i64)]),
+    "externd_allocate_ranks": (_c_int, [_c_i64, ctypes.POINTER(_c_i64), ctypes.POINTER(_c_i64), _c_dptr, _c_dptr,
+                                        _c_dptr, _c_double, ctypes.POINTER(_c_i64)]),
     "externd_pack_ternary": (_c_int, [_c_void, _c_i64, _c_i64, _c_i64, _c_void, ctypes.POINTER(_c_i64)]),
     "externd_ternary_apply": (_c_int, [_c_void, _c_void, _c_void, _c_i64, _c_i64, _c_i64, _c_void, _c_void]),
 }
@@ -181,6 +192,48 @@ def decompose(A, mu: float, tau: float, block: int, iters: int, weights=None, ou
         _check(lib.externd_decompose(_ptr(A), m, n, mu, tau, block, iters, _ptr(h), _ptr(B), _ptr(D), _ptr(C),
                                      ctypes.byref(e), tr))
     return Decomposition(B, D, C, e.value, list(tr))
+
+
+def decompose_safeguarded(A, mu: float, tau: float, block: int, iters: int, weights=None):
+    """``decompose`` with Prop. 2's safeguard; returns (Decomposition, blocks replaced by a single-entry pair)."""
+    torch = _torch()
+    lib = load()
+    A = _prep(A, torch.float32, "A")
+    m, n = A.shape
+    k = rank(m, n, mu)
+    nblocks = -(-k // block_width(m, n, block))
+    h = None if weights is None else _prep(weights, torch.float32, "weights")
+    B = torch.empty((m, k), dtype=torch.int8, device=A.device)
+    D = torch.empty((k,), dtype=torch.float32, device=A.device)
+    C = torch.empty((k, n), dtype=torch.int8, device=A.device)
+    e = _c_double()
+    tr = (_c_double * nblocks)()
+    act = _c_i64()
+    with torch.cuda.device(A.device):
+        _stream(lib, A.device)
+        _check(lib.externd_decompose_safeguarded(_ptr(A), m, n, mu, tau, block, iters, _ptr(h), _ptr(B), _ptr(D),
+                                                 _ptr(C), ctypes.byref(e), tr, ctypes.byref(act)))
+    return Decomposition(B, D, C, e.value, list(tr)), act.value
+
+
+def refine(A, dec: Decomposition, tau: float, block: int, iters: int, sweeps: int, weights=None):
+    """§2.4 refinement sweeps of ``dec``'s factors (same block layout as the run that made them). Returns
+    (Decomposition with new factors, blocks replaced per sweep); ``dec``'s tensors are left untouched."""
+    torch = _torch()
+    lib = load()
+    A = _prep(A, torch.float32, "A")
+    m, n = A.shape
+    B, D, C = dec.B.clone(), dec.D.clone(), dec.C.clone()
+    k = B.shape[1]
+    h = None if weights is None else _prep(weights, torch.float32, "weights")
+    e = _c_double()
+    tr = (_c_double * sweeps)()
+    rep = (_c_i64 * sweeps)()
+    with torch.cuda.device(A.device):
+        _stream(lib, A.device)
+        _check(lib.externd_refine(_ptr(A), m, n, tau, block, iters, sweeps, _ptr(h), _ptr(B), _ptr(D), _ptr(C), k,
+                                  ctypes.byref(e), tr, rep))
+    return Decomposition(B, D, C, e.value, list(tr)), list(rep)
 
 
 def decompose_host(A, mu: float, tau: float, block: int, iters: int, weights=None, out=None) -> Decomposition:
@@ -345,3 +398,38 @@ def ternary_apply(Bp: Packed, D, Cp: Packed, x):
         _stream(lib, x.device)
         _check(lib.externd_ternary_apply(_ptr(Bp.words), _ptr(D), _ptr(Cp.words), m, k, n, _ptr(x), _ptr(y)))
     return y
+
+
+def block_boundaries(m: int, n: int, mu: float, block: int) -> list[int]:
+    """The inner ranks b, 2b, ..., k at which a run finishes a block: the ranks of the decompose trace."""
+    lib = load()
+    cnt = _c_i64()
+    _check(lib.externd_block_boundaries(m, n, mu, block, None, ctypes.byref(cnt)))
+    arr = (_c_i64 * cnt.value)()
+    _check(lib.externd_block_boundaries(m, n, mu, block, arr, ctypes.byref(cnt)))
+    return list(arr)
+
+
+def rank_for_energy(trace, m: int, n: int, mu: float, block: int, target: float) -> Optional[int]:
+    """Smallest block-boundary rank reaching ``target`` from one run's trace (None if never); mu = k / min(m, n)."""
+    lib = load()
+    tr = (_c_double * len(trace))(*trace)
+    k = _c_i64()
+    _check(lib.externd_rank_for_energy(m, n, mu, block, tr, len(trace), target, ctypes.byref(k)))
+    return None if k.value == 0 else k.value
+
+
+def allocate_ranks(curves, costs, budget: float, weights=None) -> list[int]:
+    """Ranks per matrix under a storage budget: ``curves[j]`` lists (k, E_j(k)) at block boundaries, choosing
+    rank k of matrix j costs ``costs[j] * k``."""
+    lib = load()
+    nm = len(curves)
+    npts = (_c_i64 * nm)(*[len(c) for c in curves])
+    flat = [p for c in curves for p in c]
+    ks = (_c_i64 * max(1, len(flat)))(*[int(k) for k, _ in flat])
+    es = (_c_double * max(1, len(flat)))(*[float(e) for _, e in flat])
+    cs = (_c_double * nm)(*[float(c) for c in costs])
+    ws = None if weights is None else (_c_double * nm)(*[float(w) for w in weights])
+    out = (_c_i64 * nm)()
+    _check(lib.externd_allocate_ranks(nm, npts, ks, es, cs, ws, budget, out))
+    return list(out)

@@ -224,10 +224,14 @@ int check_device_error(Workspace& ws, unsigned* err, cudaStream_t s);
 // ------------------------------------------------------------------------------------------------------------
 // Decomposition
 // ------------------------------------------------------------------------------------------------------------
+enum Mode { kPlain = 0, kSafeguard = 1, kRefine = 2 };
+
 struct Plan {
   int m, n, b, iters, nblocks;
   long long k;
   double tau;
+  int mode = kPlain;           // Prop. 2 safeguard in the block loop, or refinement sweeps of given factors
+  int sweeps = 0;
   int gm, gn;                  // Gram split counts over m and n
   int nchunk_m, nchunk_n;
   long long ldm, ldn;
@@ -245,8 +249,13 @@ struct Bufs {
   StatPart* spart;
   F2* normpart;
   float* r;
-  double *norm_a, *norm_r, *trace;
+  double *norm_a, *norm_r, *norm_add, *trace;
   int* J;
+  float* K;               // Eq. 4's G_U .* G_V of the block (safeguard and refinement decisions)
+  EntryBest* best;        // per-CTA best single entries (safeguard)
+  int nbest;
+  BlockChoice* choice;
+  long long* counts;      // activations (safeguard) or replaced blocks per sweep (refinement)
 };
 
 int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
@@ -301,7 +310,22 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "normpart", (size_t)deflate_tiles(p.m, p.n), &B->normpart));
   TRY(need(ws, "scalars", 4, &B->norm_a));
   B->norm_r = B->norm_a + 1;
-  TRY(need(ws, "trace", (size_t)p.nblocks, &B->trace));
+  B->norm_add = B->norm_a + 2;
+  TRY(need(ws, "trace", (size_t)std::max(p.nblocks, p.sweeps), &B->trace));
+  B->K = nullptr;
+  B->best = nullptr;
+  B->nbest = 0;
+  B->choice = nullptr;
+  B->counts = nullptr;
+  if (p.mode != kPlain) {
+    TRY(need(ws, "K", (size_t)w * w, &B->K));
+    TRY(need(ws, "choice", 1, &B->choice, true));
+    TRY(need(ws, "counts", (size_t)std::max(1, p.sweeps), &B->counts));
+    if (p.mode == kSafeguard) {
+      B->nbest = entry_argmax_parts(p.m);
+      TRY(need(ws, "best", (size_t)B->nbest, &B->best));
+    }
+  }
   return get_one(ws, &B->one);
 }
 
@@ -355,104 +379,216 @@ Plan make_plan(long long m, long long n, long long k, int block, int iters, doub
 
 enum Kind { kVstep = 1, kUstep = 2, kDeflate = 3, kDecor = 4, kApply = 5, kGram = 6, kSolve = 7, kStart = 8 };
 
-// Enqueues the whole decomposition on stream s.
+// Thresholds and statistics of the Eq. 2 producers (per-block chunk counts set by fit_block).
+struct Eq2 {
+  Thresh th_m, th_n;
+  Stats st_g, st_m, st_n;
+};
+
+Eq2 make_eq2(const Plan& p, const Bufs& B) {
+  Eq2 e{Thresh{B.theta, B.fallback, B.arg, B.ticket, p.tau, p.m}, Thresh{B.theta, B.fallback, B.arg, B.ticket, p.tau, p.n},
+        Stats{}, Stats{}, Stats{}};
+  e.st_g = Stats{B.spart, (int)cdiv(p.m, kStatChunk), e.th_m};   // gather (block start)
+  e.st_m = Stats{B.spart, 0, e.th_m};                              // U-step decorrelation
+  e.st_n = Stats{B.spart, 0, e.th_n};                              // V-step decorrelation
+  return e;
+}
+
+// The ALS fit of one block of w components (§2.3 for w = 1, §2.4): `iters` V-step / U-step pairs, ending with U
+// in Ut (and its exact Gram where fused), V in Vt, the K-major fp16 copies for the tensor-core deflation, and the
+// last U-step product in B.part. With `staged` the caller has put the starting U in Ut (and Ut16) -- a refinement
+// revisit -- otherwise the block starts from the selected columns of R (§2.4, initial columns).
+int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* h, int blk, int w, bool staged,
+              cudaStream_t s) {
+  cudaStream_t side = ws.side;
+  const int m = p.m, n = p.n;
+  const int nrt = deflate_row_tiles(m);
+  const int sv = splits_v(w, m, n), su = splits_u(w, m, n);
+  q.st_m.nchunk = decorrelate_chunks(m, w);
+  q.st_n.nchunk = decorrelate_chunks(n, w);
+  // Exact Gram matrices of unweighted ternary factors are accumulated by the apply that writes the factor
+  // (integer atomics) up to 128 components; wider blocks and the weighted V^T H V use the Gram kernel.
+  const bool fusedU = w <= 128, fusedV = w <= 128 && h == nullptr;
+  __half* const U16 = use_tc(w) ? B.Ut16 : nullptr;
+  __half* const V16 = use_tc(w) ? B.Vt16 : nullptr;
+  if (!staged) {
+    KL(kStart, 2, launch_select_with(B.colpart, nrt, n, h, w, B.J, B.colE, s));
+    KL(kStart, 1, launch_gather(B.R, m, n, B.J, w, B.X, m, q.st_g, s));
+    if (blk > 0) JOIN();   // the previous block's outputs (side branch) have read Ut, Vt and d
+    KL(kApply, 1, launch_apply(B.X, w, m, m, q.th_m, B.Ut, (int)p.ldm, (fusedU && w > 1) ? B.GintU : nullptr, s, U16,
+                               p.ldm, nullptr, 0, B.gram));
+  }
+  for (int it = 0; it < p.iters; ++it) {
+    const bool last = it == p.iters - 1;
+    // V-step: V <- T([(U^T U + eps I)^-1 U^T R]^T)   (plain R even when weighted, §2.5).
+    // The Gram inverse depends only on U: it runs on the side branch while the product streams R. A staged U has
+    // no integer Gram yet, so its first inverse takes the Gram kernel.
+    if (w > 1) {
+      FORK();
+      if (fusedU && !(staged && it == 0)) {
+        KLS(kSolve, 1, side, launch_inverse_int(B.GintU, w, B.GrawU, B.Ginv, side));
+      } else {
+        KLS(kGram, 1, side, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, side));
+        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side));
+      }
+    }
+    KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
+    if (w > 1) JOIN();
+    KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, sv, n, B.X, n, q.st_n, s));
+    KL(kApply, 1, launch_apply(B.X, w, n, n, q.th_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, s, V16, p.ldn,
+                               (last && use_tc(w)) ? B.Vk16 : nullptr, B.ldk, B.gram));
+    // U-step: U <- T(R H V (V^T H V + eps I)^-1)
+    FORK();
+    if (fusedV) {
+      KLS(kSolve, 1, side, launch_inverse_int(B.GintV, w, B.GrawV, B.Ginv, side));
+    } else {
+      KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
+      KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side));
+    }
+    KL(kUstep, 1, product_u(B.R, m, n, B.Vt, V16, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s));
+    JOIN();
+    KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, su, m, B.X, m, q.st_m, s));
+    // the next V-step's inverse (w > 1) or, after the last iteration, Eq. 4 consumes U's Gram
+    // (the fp16 copy of U is not needed after the last iteration)
+    KL(kApply, 1, launch_apply(B.X, w, m, m, q.th_m, B.Ut, (int)p.ldm, (fusedU && (w > 1 || last)) ? B.GintU : nullptr,
+                               s, last ? nullptr : U16, p.ldm, (last && use_tc(w)) ? B.Uk16 : nullptr, B.ldk,
+                               B.gram));
+  }
+  return EXTERND_OK;
+}
+
+// Eq. 4: [(U^T U) .* (V^T H V)] d = diag(U^T R H V), with R H V the last U-step product; K (if given) receives
+// the matrix without the ridge.
+int block_scales_step(const Plan& p, const Bufs& B, int w, float* K, cudaStream_t s) {
+  const int m = p.m, n = p.n;
+  const int su = splits_u(w, m, n);
+  KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, su, B.r, s));
+  if (w <= 128) {
+    KL(kSolve, 1, launch_scales_int(B.GintU, B.GrawV, B.r, w, B.d, s, K));
+  } else {
+    KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
+    KL(kSolve, 1, launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s, K));
+  }
+  return EXTERND_OK;
+}
+
+// R <- R - U diag(d) V^T with the block in (Ut, Vt, d) / (Uk16, Vk16, d), statistics for the next selection, and
+// the squared norm into *norm (and the energy into *trace if given).
+int deflate_step(const Plan& p, const Bufs& B, const float* h, int w, double* norm, double* trace, cudaStream_t s) {
+  const int m = p.m, n = p.n;
+  if (use_tc(w)) {
+    KL(kDeflate, 1, launch_deflate_tc(B.R, m, n, B.Uk16, B.Vk16, B.ldk, B.d, w, h, B.colpart, B.normpart, B.maxpart,
+                                      B.err, s));
+  } else {
+    KL(kDeflate, 1, launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart, B.normpart,
+                                   s, B.maxpart));
+  }
+  KL(0, 1, launch_norm(B.normpart, deflate_tiles(m, n), norm, trace != nullptr ? B.norm_a : nullptr, trace, s,
+                       B.maxpart, B.maxabs));
+  return EXTERND_OK;
+}
+
+// R = A with column energies, ||A||_H^2 and the fp16 scaling scalars.
+int start_residual(const Plan& p, const Bufs& B, const float* A, const float* h, cudaStream_t s) {
+  const int m = p.m, n = p.n;
+  KL(kDeflate, 1, launch_deflate(A, B.R, m, n, nullptr, 0, false, nullptr, nullptr, 0, 0, h, B.colpart, B.normpart, s,
+                                 B.maxpart));
+  KL(0, 1, launch_norm(B.normpart, deflate_tiles(m, n), B.norm_a, nullptr, nullptr, s, B.maxpart, B.maxabs));
+  if (h != nullptr) KL(0, 1, launch_absmax(h, n, B.maxabs + 1, s));
+  return EXTERND_OK;
+}
+
+// Enqueues the whole decomposition on stream s (with Prop. 2's safeguard when p.mode == kSafeguard).
 int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* A, const float* h, int8_t* Bout,
                       float* Dout, int8_t* Cout, cudaStream_t s) {
   cudaStream_t side = ws.side;
   const int m = p.m, n = p.n;
-  // each producer of Eq. 2 statistics and its apply agree on the chunk count; the producer's last CTA writes the
-  // thresholds the apply reads
-  const Thresh th_m{B.theta, B.fallback, B.arg, B.ticket, p.tau, m};
-  const Thresh th_n{B.theta, B.fallback, B.arg, B.ticket, p.tau, n};
-  const Stats st_g{B.spart, (int)cdiv(m, kStatChunk), th_m};   // gather (block start)
-  Stats st_m{B.spart, 0, th_m};       // U-step decorrelation (chunk count set per block width)
-  Stats st_n{B.spart, 0, th_n};       // V-step decorrelation
-  const int nrt = deflate_row_tiles(m), ntiles = deflate_tiles(m, n);
+  Eq2 q = make_eq2(p, B);
   g_prof.used = 0;
   g_prof.launches = 0;
-  // R = A, column energies, ||A||_H^2
-  KL(kDeflate, 1, launch_deflate(A, B.R, m, n, nullptr, 0, false, nullptr, nullptr, 0, 0, h, B.colpart, B.normpart, s,
-                                 B.maxpart));
-  KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_a, nullptr, nullptr, s, B.maxpart, B.maxabs));
-  if (h != nullptr) KL(0, 1, launch_absmax(h, n, B.maxabs + 1, s));
+  TRY(start_residual(p, B, A, h, s));
+  const bool guard = p.mode == kSafeguard;
   for (int blk = 0; blk < p.nblocks; ++blk) {
     const long long j0 = (long long)blk * p.b;
     const int w = (int)std::min<long long>(p.b, p.k - j0);
-    const int sv = splits_v(w, m, n), su = splits_u(w, m, n);
-    st_m.nchunk = decorrelate_chunks(m, w);
-    st_n.nchunk = decorrelate_chunks(n, w);
-    // Exact Gram matrices of unweighted ternary factors are accumulated by the apply that writes the factor
-    // (integer atomics) up to 128 components; wider blocks and the weighted V^T H V use the Gram kernel.
-    const bool fusedU = w <= 128, fusedV = w <= 128 && h == nullptr;
-    KL(kStart, 2, launch_select_with(B.colpart, nrt, n, h, w, B.J, B.colE, s));
-    KL(kStart, 1, launch_gather(B.R, m, n, B.J, w, B.X, m, st_g, s));
-    __half* const U16 = use_tc(w) ? B.Ut16 : nullptr;
-    __half* const V16 = use_tc(w) ? B.Vt16 : nullptr;
-    if (blk > 0) JOIN();   // the previous block's outputs (side branch) have read Ut, Vt and d
-    KL(kApply, 1, launch_apply(B.X, w, m, m, th_m, B.Ut, (int)p.ldm, (fusedU && w > 1) ? B.GintU : nullptr, s, U16,
-                               p.ldm, nullptr, 0, B.gram));
-    for (int it = 0; it < p.iters; ++it) {
-      const bool last = it == p.iters - 1;
-      // V-step: V <- T([(U^T U + eps I)^-1 U^T R]^T)   (plain R even when weighted, §2.5).
-      // The Gram inverse depends only on U: it runs on the side branch while the product streams R.
-      if (w > 1) {
-        FORK();
-        if (fusedU) {
-          KLS(kSolve, 1, side, launch_inverse_int(B.GintU, w, B.GrawU, B.Ginv, side));
-        } else {
-          KLS(kGram, 1, side, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, side));
-          KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side));
-        }
-      }
-      KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
-      if (w > 1) JOIN();
-      KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, sv, n, B.X, n, st_n, s));
-      KL(kApply, 1, launch_apply(B.X, w, n, n, th_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, s, V16, p.ldn,
-                                 (last && use_tc(w)) ? B.Vk16 : nullptr, B.ldk, B.gram));
-      // U-step: U <- T(R H V (V^T H V + eps I)^-1)
+    // Prop. 2: the best single entry of the residual this block is fitted to
+    if (guard) KL(0, 1, launch_entry_argmax(B.R, m, n, h, B.best, s));
+    TRY(fit_block(ws, p, B, q, h, blk, w, false, s));
+    if (!guard) {
+      // The block's outputs leave on the side branch: B from the final U and C from the final V now, D after the
+      // scales; the next block joins before it overwrites Ut.
       FORK();
-      if (fusedV) {
-        KLS(kSolve, 1, side, launch_inverse_int(B.GintV, w, B.GrawV, B.Ginv, side));
-      } else {
-        KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
-        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side));
-      }
-      KL(kUstep, 1, product_u(B.R, m, n, B.Vt, V16, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s));
-      JOIN();
-      KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, su, m, B.X, m, st_m, s));
-      // the next V-step's inverse (w > 1) or, after the last iteration, Eq. 4 consumes U's Gram
-      // (the fp16 copy of U is not needed after the last iteration)
-      KL(kApply, 1, launch_apply(B.X, w, m, m, th_m, B.Ut, (int)p.ldm, (fusedU && (w > 1 || last)) ? B.GintU : nullptr,
-                                 s, last ? nullptr : U16, p.ldm, (last && use_tc(w)) ? B.Uk16 : nullptr, B.ldk,
-                                 B.gram));
+      KLS(0, 1, side, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, side));
+      LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
+                           cudaMemcpyDeviceToDevice, side));
     }
-    // The block's outputs leave on the side branch: B from the final U and C from the final V now, D after the
-    // scales; the next block joins before it overwrites Ut.
-    FORK();
-    KLS(0, 1, side, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, side));
-    LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
-                         cudaMemcpyDeviceToDevice, side));
-    // Eq. 4: [(U^T U) .* (V^T H V)] d = diag(U^T R H V), with R H V the last U-step product
-    KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, su, B.r, s));
-    if (fusedU) {
-      KL(kSolve, 1, launch_scales_int(B.GintU, B.GrawV, B.r, w, B.d, s));
+    TRY(block_scales_step(p, B, w, guard ? B.K : nullptr, s));
+    if (guard) {
+      KL(0, 1, launch_safeguard_decide(B.best, B.nbest, n, h, B.r, B.d, B.K, w, B.choice, s));
+      KL(0, 1, launch_safeguard_replace(B.choice, w, m, n, B.Ut, p.ldm, B.Vt, p.ldn, use_tc(w) ? B.Uk16 : nullptr,
+                                        use_tc(w) ? B.Vk16 : nullptr, B.ldk, s));
+      FORK();
+      KLS(0, 1, side, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, side));
+      LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
+                           cudaMemcpyDeviceToDevice, side));
     } else {
-      KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
-      KL(kSolve, 1, launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s));
+      FORK();
     }
-    FORK();
     LK(cudaMemcpyAsync(Dout + j0, B.d, sizeof(float) * w, cudaMemcpyDeviceToDevice, side));
-    // R <- R - U diag(d) V^T
-    if (use_tc(w)) {
-      KL(kDeflate, 1, launch_deflate_tc(B.R, m, n, B.Uk16, B.Vk16, B.ldk, B.d, w, h, B.colpart, B.normpart, B.maxpart,
-                                        B.err, s));
-    } else {
-      KL(kDeflate, 1, launch_deflate(B.R, B.R, m, n, B.Ut, p.ldm, false, B.d, B.Vt, p.ldn, w, h, B.colpart,
-                                     B.normpart, s, B.maxpart));
-    }
-    KL(0, 1, launch_norm(B.normpart, ntiles, B.norm_r, B.norm_a, B.trace + blk, s, B.maxpart, B.maxabs));
+    TRY(deflate_step(p, B, h, w, B.norm_r, B.trace + blk, s));
   }
   if (p.nblocks > 0) JOIN();
+  if (guard) KL(0, 1, launch_count_reset(B.choice, B.counts, s));
+  return EXTERND_OK;
+}
+
+// Block j0 .. j0 + w - 1 of the factors (B m x k, C k x n, D) into the internal layouts: Ut (and its fp16 copy
+// when `u16`), Vt, the K-major fp16 copies for the tensor-core deflation, and sign * D into B.d.
+int stage_block(const Plan& p, const Bufs& B, const int8_t* Bf, const float* Df, const int8_t* Cf, long long j0, int w,
+                float sign, bool u16, cudaStream_t s) {
+  const int m = p.m, n = p.n;
+  KL(0, 1, launch_transpose_i8(Bf + j0, p.k, m, w, B.Ut, p.ldm, s));
+  LK(cudaMemcpy2DAsync(B.Vt, (size_t)p.ldn, Cf + j0 * n, (size_t)n, (size_t)n, (size_t)w, cudaMemcpyDeviceToDevice, s));
+  if (use_tc(w)) {
+    if (u16) KL(0, 1, launch_i8_to_f16(B.Ut, p.ldm, w, m, B.Ut16, p.ldm, s));
+    KL(0, 1, launch_kmajor(B.Ut, p.ldm, 1, w, m, B.Uk16, B.ldk, s));
+    KL(0, 1, launch_kmajor(B.Vt, p.ldn, 1, w, n, B.Vk16, B.ldk, s));
+  }
+  KL(0, 1, launch_scale_copy(Df + j0, sign, w, B.d, s));
+  return EXTERND_OK;
+}
+
+// Enqueues p.sweeps refinement sweeps (§2.4) of the factors in (Bf, Df, Cf), updated in place: R = A - B D C,
+// then for every block in order: add it back, refit it from its own U, keep the refit if it removes at least as
+// much, deflate the kept block. trace[s] = energy after sweep s; counts[s] = blocks replaced in sweep s.
+int enqueue_refine(Workspace& ws, const Plan& p, const Bufs& B, const float* A, const float* h, int8_t* Bf, float* Df,
+                   int8_t* Cf, cudaStream_t s) {
+  const int m = p.m, n = p.n;
+  Eq2 q = make_eq2(p, B);
+  g_prof.used = 0;
+  g_prof.launches = 0;
+  TRY(start_residual(p, B, A, h, s));
+  for (int blk = 0; blk < p.nblocks; ++blk) {
+    const long long j0 = (long long)blk * p.b;
+    const int w = (int)std::min<long long>(p.b, p.k - j0);
+    TRY(stage_block(p, B, Bf, Df, Cf, j0, w, 1.f, false, s));
+    TRY(deflate_step(p, B, h, w, B.norm_r, nullptr, s));
+  }
+  for (int sw = 0; sw < p.sweeps; ++sw) {
+    for (int blk = 0; blk < p.nblocks; ++blk) {
+      const long long j0 = (long long)blk * p.b;
+      const int w = (int)std::min<long long>(p.b, p.k - j0);
+      TRY(stage_block(p, B, Bf, Df, Cf, j0, w, -1.f, true, s));
+      TRY(deflate_step(p, B, h, w, B.norm_add, nullptr, s));              // add back: R_add = R + U D V^T
+      TRY(fit_block(ws, p, B, q, h, blk, w, true, s));
+      TRY(block_scales_step(p, B, w, B.K, s));
+      KL(0, 1, launch_refine_decide(B.norm_add, B.norm_r, B.r, B.d, B.K, w, B.choice, s));
+      KL(0, 1, launch_commit(B.choice, B.Ut, p.ldm, B.Vt, p.ldn, B.d, w, m, n, Bf, Df, Cf, p.k, j0, s));
+      TRY(stage_block(p, B, Bf, Df, Cf, j0, w, 1.f, false, s));           // the kept block
+      TRY(deflate_step(p, B, h, w, B.norm_r, blk == p.nblocks - 1 ? B.trace + sw : nullptr, s));
+    }
+    KL(0, 1, launch_count_reset(B.choice, B.counts + sw, s));
+  }
   return EXTERND_OK;
 }
 
@@ -462,10 +598,10 @@ struct GraphKey {
   int b, iters;
   double tau;
   unsigned gen;
-  int prof;
+  int prof, mode, sweeps;
   bool operator<(const GraphKey& o) const {
-    return std::tie(A, h, B, D, C, m, n, k, b, iters, tau, gen, prof) <
-           std::tie(o.A, o.h, o.B, o.D, o.C, o.m, o.n, o.k, o.b, o.iters, o.tau, o.gen, o.prof);
+    return std::tie(A, h, B, D, C, m, n, k, b, iters, tau, gen, prof, mode, sweeps) <
+           std::tie(o.A, o.h, o.B, o.D, o.C, o.m, o.n, o.k, o.b, o.iters, o.tau, o.gen, o.prof, o.mode, o.sweeps);
   }
 };
 
@@ -482,20 +618,25 @@ bool graphs_enabled() {
   return !(e && std::strcmp(e, "0") == 0);
 }
 
-int run_decompose(const float* A, long long m, long long n, double mu, double tau, int block, int iters,
-                  const float* h, int8_t* Bout, float* Dout, int8_t* Cout, double* energy, double* trace) {
+// Runs the block loop of plan p on the library stream: captured once per configuration into a CUDA graph and
+// replayed (EXTERND_GRAPHS=0 enqueues it directly). Then reads `ntrace` trace entries and, in the safeguard and
+// refinement modes, `ncounts` counts back to the host.
+int run_plan(const Plan& p, const float* A, const float* h, int8_t* Bout, float* Dout, int8_t* Cout, double* energy,
+             double* trace, int ntrace, long long* counts, int ncounts) {
   Workspace* ws;
   TRY(current_ws(&ws));
-  int64_t k;
-  TRY(externd_rank(m, n, mu, &k));
-  Plan p = make_plan(m, n, k, block, iters, tau);
   Bufs B;
   TRY(plan_buffers(*ws, p, &B));
   int dev;
   CK(cudaGetDevice(&dev));
   cudaStream_t s = g_stream;
+  auto enqueue = [&](cudaStream_t st) {
+    return p.mode == kRefine ? enqueue_refine(*ws, p, B, A, h, Bout, Dout, Cout, st)
+                             : enqueue_decompose(*ws, p, B, A, h, Bout, Dout, Cout, st);
+  };
   if (graphs_enabled()) {
-    GraphKey key{A, h, Bout, Dout, Cout, m, n, k, p.b, iters, tau, ws->generation, g_prof.kind};
+    GraphKey key{A, h, Bout, Dout, Cout, p.m, p.n, p.k, p.b, p.iters, p.tau, ws->generation, g_prof.kind, p.mode,
+                 p.sweeps};
     auto& cache = g_graphs[dev];
     auto it = cache.find(key);
     if (it == cache.end()) {
@@ -505,7 +646,7 @@ int run_decompose(const float* A, long long m, long long n, double mu, double ta
       }
       cudaGraph_t graph;
       CK(cudaStreamBeginCapture(ws->cap_stream, cudaStreamCaptureModeThreadLocal));
-      int rc = enqueue_decompose(*ws, p, B, A, h, Bout, Dout, Cout, ws->cap_stream);
+      int rc = enqueue(ws->cap_stream);
       cudaError_t ec = cudaStreamEndCapture(ws->cap_stream, &graph);
       if (rc != EXTERND_OK) return rc;
       if (ec != cudaSuccess) return cuda_fail(ec, "cudaStreamEndCapture");
@@ -519,22 +660,35 @@ int run_decompose(const float* A, long long m, long long n, double mu, double ta
     g_prof.last_used = it->second.events;
     g_prof.last_launches = it->second.launches;
   } else {
-    TRY(enqueue_decompose(*ws, p, B, A, h, Bout, Dout, Cout, s));
+    TRY(enqueue(s));
     g_prof.last_used = g_prof.used;
     g_prof.last_launches = g_prof.launches;
   }
-  if (energy != nullptr || trace != nullptr) {
+  if (energy != nullptr || trace != nullptr || counts != nullptr) {
+    const size_t tb = sizeof(double) * (size_t)ntrace, cb = sizeof(long long) * (size_t)ncounts;
     void* hbuf;
-    TRY(need_host(*ws, sizeof(double) * (size_t)p.nblocks, &hbuf));
-    CK(cudaMemcpyAsync(hbuf, B.trace, sizeof(double) * p.nblocks, cudaMemcpyDeviceToHost, s));
+    TRY(need_host(*ws, tb + cb + 16, &hbuf));
+    if (ntrace > 0) CK(cudaMemcpyAsync(hbuf, B.trace, tb, cudaMemcpyDeviceToHost, s));
+    if (ncounts > 0) CK(cudaMemcpyAsync(static_cast<char*>(hbuf) + tb, B.counts, cb, cudaMemcpyDeviceToHost, s));
     CK(cudaStreamSynchronize(s));
     const double* tr = static_cast<const double*>(hbuf);
-    if (energy) *energy = tr[p.nblocks - 1];
-    if (trace) std::memcpy(trace, tr, sizeof(double) * p.nblocks);
+    if (energy && ntrace > 0) *energy = tr[ntrace - 1];
+    if (trace && ntrace > 0) std::memcpy(trace, tr, tb);
+    if (counts && ncounts > 0) std::memcpy(counts, static_cast<char*>(hbuf) + tb, cb);
     TRY(check_device_error(*ws, B.err, s));
   }
   CK(cudaGetLastError());
   return EXTERND_OK;
+}
+
+int run_decompose(const float* A, long long m, long long n, double mu, double tau, int block, int iters,
+                  const float* h, int8_t* Bout, float* Dout, int8_t* Cout, double* energy, double* trace,
+                  long long* activations = nullptr) {
+  int64_t k;
+  TRY(externd_rank(m, n, mu, &k));
+  Plan p = make_plan(m, n, k, block, iters, tau);
+  p.mode = activations != nullptr ? kSafeguard : kPlain;
+  return run_plan(p, A, h, Bout, Dout, Cout, energy, trace, p.nblocks, activations, activations ? 1 : 0);
 }
 
 int check_device_error(Workspace& ws, unsigned* err, cudaStream_t s) {
@@ -700,6 +854,46 @@ int externd_decompose(const float* A, int64_t m, int64_t n, double mu, double ta
   TRY(check_dev(C));
   if (weights != nullptr) TRY(check_dev(weights));
   return run_decompose(A, m, n, mu, tau, block, iters, weights, B, D, C, energy, trace);
+}
+
+int externd_decompose_safeguarded(const float* A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
+                                  const float* weights, int8_t* B, float* D, int8_t* C, double* energy, double* trace,
+                                  int64_t* activations) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  TRY(check_common(m, n));
+  TRY(check_params(mu, tau, block, iters));
+  if (activations == nullptr) return EXTERND_EINVAL;
+  TRY(check_dev(A));
+  TRY(check_dev(B));
+  TRY(check_dev(D));
+  TRY(check_dev(C));
+  if (weights != nullptr) TRY(check_dev(weights));
+  long long act = 0;
+  TRY(run_decompose(A, m, n, mu, tau, block, iters, weights, B, D, C, energy, trace, &act));
+  *activations = act;
+  return EXTERND_OK;
+}
+
+int externd_refine(const float* A, int64_t m, int64_t n, double tau, int block, int iters, int sweeps,
+                   const float* weights, int8_t* B, float* D, int8_t* C, int64_t k, double* energy, double* trace,
+                   int64_t* replaced) {
+  std::lock_guard<std::mutex> lock(g_mutex);
+  TRY(check_common(m, n));
+  if (k < 1 || k > (1LL << 31) || sweeps < 1 || sweeps > 1000000) return EXTERND_EINVAL;
+  TRY(check_params(1.0, tau, block, iters));
+  TRY(check_dev(A));
+  TRY(check_dev(B));
+  TRY(check_dev(D));
+  TRY(check_dev(C));
+  if (weights != nullptr) TRY(check_dev(weights));
+  Plan p = make_plan(m, n, k, block, iters, tau);
+  p.mode = kRefine;
+  p.sweeps = sweeps;
+  std::vector<long long> counts((size_t)sweeps);
+  TRY(run_plan(p, A, weights, B, D, C, energy, trace, sweeps, counts.data(), sweeps));
+  if (replaced != nullptr)
+    for (int i = 0; i < sweeps; ++i) replaced[i] = counts[(size_t)i];
+  return EXTERND_OK;
 }
 
 int externd_decompose_host(const float* A, int64_t m, int64_t n, double mu, double tau, int block, int iters,

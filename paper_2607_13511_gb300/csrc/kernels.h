@@ -234,10 +234,44 @@ cudaError_t launch_inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaS
 // r[a] = sum_y Ut[a][y] * sum_s part[s][a][y]
 cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, float* r,
                         cudaStream_t s);
-// d solves [(sum_s GUpart[s]) .* GVraw + eps I] d = r (eps = 0 when w == 1).
+// d solves [(sum_s GUpart[s]) .* GVraw + eps I] d = r (eps = 0 when w == 1); K (optional, w x w) receives the
+// matrix without the ridge, K = G_U .* G_V of Eq. 4.
 cudaError_t launch_scales(const float* GUpart, int splits, const float* GVraw, const float* r, int w, float* d,
-                          cudaStream_t s);
+                          cudaStream_t s, float* K = nullptr);
 // Same with G_U from an integer upper-triangle Gram, reset to zero after reading.
-cudaError_t launch_scales_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s);
+cudaError_t launch_scales_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s,
+                              float* K = nullptr);
+
+
+// ---- extensions of the block loop (extend.cu): Prop. 2 safeguard and §2.4 refinement sweeps
+struct __align__(16) EntryBest {   // a CTA's best single entry: score (|R_ij| or h_j R_ij^2), R_ij, row-major index
+  float score, rij;
+  unsigned long long idx;
+};
+struct BlockChoice {                 // the device-side decision of one block, and a running count of positive ones
+  int flag, sign;
+  long long row, col, count;
+};
+int entry_argmax_parts(int m);
+cudaError_t launch_entry_argmax(const float* R, int m, int n, const float* h, EntryBest* part, cudaStream_t s);
+// flag = (h_j R_ij^2 > 2 r^T d - d^T K d) for the best entry; with the flag d becomes (|R_ij|, 0, ..., 0).
+cudaError_t launch_safeguard_decide(const EntryBest* part, int nparts, int n, const float* h, const float* r, float* d,
+                                    const float* K, int w, BlockChoice* choice, cudaStream_t s);
+// With the flag: U = e_i, V = sgn e_j as component 0 and zero components after it, in Ut / Vt and (if given) the
+// K-major fp16 copies Uk / Vk.
+cudaError_t launch_safeguard_replace(const BlockChoice* choice, int w, int m, int n, int8_t* Ut, long long ldm,
+                                     int8_t* Vt, long long ldn, __half* Uk, __half* Vk, long long ldk,
+                                     cudaStream_t s);
+// flag = (2 r^T d - d^T K d >= norm_add - norm_prev).
+cudaError_t launch_refine_decide(const double* norm_add, const double* norm_prev, const float* r, const float* d,
+                                 const float* K, int w, BlockChoice* choice, cudaStream_t s);
+// With the flag: the block (Ut, Vt, d) becomes columns / rows j0 .. j0 + w - 1 of B (m x k), C (k x n) and D.
+cudaError_t launch_commit(const BlockChoice* choice, const int8_t* Ut, long long ldm, const int8_t* Vt, long long ldn,
+                          const float* d, int w, int m, int n, int8_t* B, float* D, int8_t* C, long long k,
+                          long long j0, cudaStream_t s);
+// dst[a] = alpha * src[a]
+cudaError_t launch_scale_copy(const float* src, float alpha, int w, float* dst, cudaStream_t s);
+// *out = count (if out), count = 0
+cudaError_t launch_count_reset(BlockChoice* choice, long long* out, cudaStream_t s);
 
 }  // namespace externd

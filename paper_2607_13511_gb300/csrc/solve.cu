@@ -136,8 +136,12 @@ __global__ void __launch_bounds__(NWARP * 32) sweep_kernel(const float* __restri
       const int j = lane + 32 * c;
       float v = S[a][c];
       if (i < w && j < w) {
-        if (MODE == 0) Graw[(long long)i * w + j] = v;
-        else v *= GVraw[(long long)i * w + j];
+        if (MODE == 0) {
+          Graw[(long long)i * w + j] = v;
+        } else {
+          v *= GVraw[(long long)i * w + j];
+          if (Graw != nullptr) Graw[(long long)i * w + j] = v;
+        }
         if (i == j) diag += v;
       } else {
         v = (i == j) ? 1.f : 0.f;     // identity on the padding
@@ -459,8 +463,12 @@ __global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ 
         const int j = tx + 32 * c;
         float v = S[a][c];
         if (i < w && j < w) {
-          if (MODE == 0) Graw[(long long)i * w + j] = v;
-          else v *= GVraw[(long long)i * w + j];
+          if (MODE == 0) {
+            Graw[(long long)i * w + j] = v;
+          } else {
+            v *= GVraw[(long long)i * w + j];
+            if (Graw != nullptr) Graw[(long long)i * w + j] = v;
+          }
           if (i == j) diag += v;
         } else {
           v = (i == j) ? 1.f : 0.f;
@@ -714,8 +722,9 @@ cudaError_t launch_inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaS
   return launch_sweep_int<0>(Gint, w, nullptr, nullptr, Graw, Ginv, s);
 }
 
-cudaError_t launch_scales_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s) {
-  return launch_sweep_int<1>(GUint, w, GVraw, r, nullptr, d, s);
+cudaError_t launch_scales_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s,
+                              float* K) {
+  return launch_sweep_int<1>(GUint, w, GVraw, r, K, d, s);
 }
 
 cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, float* r,
@@ -725,8 +734,8 @@ cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* pa
 }
 
 cudaError_t launch_scales(const float* GUpart, int splits, const float* GVraw, const float* r, int w, float* d,
-                          cudaStream_t s) {
-  return launch_sweep<1>(GUpart, splits, w, GVraw, r, nullptr, d, s);
+                          cudaStream_t s, float* K) {
+  return launch_sweep<1>(GUpart, splits, w, GVraw, r, K, d, s);
 }
 
 }  // namespace externd
