@@ -1214,16 +1214,22 @@ int externd_ternary_apply(const uint32_t* Bp, const float* D, const uint32_t* Cp
   TRY(check_dev(y));
   Workspace* ws;
   TRY(current_ws(&ws));
-  float *z, *part = nullptr;
-  unsigned* ticket = nullptr;
+  // z = D (.) (C x) goes straight into the fragments of the second product's vector
+  float *z, *part;
+  uint32_t *xf, *zf;
+  unsigned* ticket;
+  long long pc, tc, pb, tb;
+  gemv_scratch(k, n, &pc, &tc);
+  gemv_scratch(m, k, &pb, &tb);
   TRY(need(*ws, "apply.z", (size_t)k, &z));
-  const long long np = std::max(gemv_partial_floats(k, n), gemv_partial_floats(m, k));
-  if (np > 0) {
-    TRY(need(*ws, "apply.part", (size_t)np, &part));
-    TRY(need(*ws, "apply.ticket", (size_t)std::max(gemv_tickets(k), gemv_tickets(m)), &ticket, true));
-  }
-  LK(launch_ternary_gemv(Cp, k, n, x, D, z, part, ticket, g_stream));         // z = D (.) (C x)
-  LK(launch_ternary_gemv(Bp, m, k, z, nullptr, y, part, ticket, g_stream));   // y = B z
+  TRY(need(*ws, "apply.xf", (size_t)fragment_words(n), &xf));
+  TRY(need(*ws, "apply.zf", (size_t)fragment_words(k), &zf, true));
+  TRY(need(*ws, "apply.part", (size_t)std::max(pc, pb), &part));
+  TRY(need(*ws, "apply.ticket", (size_t)std::max(tc, tb), &ticket, true));
+  // x's fragments; the first product writes z's up to 32 * ceil(k / 32) columns, the rest of the last group is zeroed
+  LK(launch_fragments(x, n, xf, zf, k, g_stream));
+  LK(launch_ternary_gemv(Cp, k, n, xf, D, z, zf, part, ticket, g_stream));
+  LK(launch_ternary_gemv(Bp, m, k, zf, nullptr, y, nullptr, part, ticket, g_stream));
   return EXTERND_OK;
 }
 

@@ -168,17 +168,20 @@ cudaError_t launch_product_v_tma(const float* R, int m, int n, const __half* Ut,
 cudaError_t launch_product_u_tma(const float* R, int m, int n, const __half* Vt, int ldv, int w, const float* h,
                                  float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s);
 // ---- packed inference (packed.cu, §2.6): 2-bit codes in tensor-core fragment order (packed_words(rows, cols)
-// 32-bit words; layout in packed.cu) and the row product out[r] = scale[r] * sum_j T[r][j] v[j] (scale optional).
-// Over more than 1024 columns the product splits the columns into slices whose partial rows go to `partial`
-// (gemv_partial_floats(rows, cols) floats) and are summed in order by the last CTA of each block of 128 rows, counted
-// in `ticket` (gemv_tickets(rows) zeroed words, left zeroed); both may be NULL when gemv_partial_floats returns 0.
+// 32-bit words; layout in packed.cu) and the row product out[r] = scale[r] * sum_j T[r][j] v[j] (scale optional)
+// with the vector given as B fragments (fragment_words(cols) words, from launch_fragments). With zf the product also
+// writes the fragments of out (as the next product's vector of length rows; zf's words past 32 * ceil(rows / 32)
+// must be zero). partial / ticket: gemv_scratch(rows, cols) floats / zeroed words (left zeroed).
 long long packed_words(long long rows, long long cols);
 cudaError_t launch_pack_ternary(const int8_t* T, long long rows, long long cols, long long ldt, uint32_t* words,
                                 unsigned long long* nnz, cudaStream_t s);
-long long gemv_partial_floats(long long rows, long long cols);
-long long gemv_tickets(long long rows);
-cudaError_t launch_ternary_gemv(const uint32_t* words, long long rows, long long cols, const float* v,
-                                const float* scale, float* out, float* partial, unsigned* ticket, cudaStream_t s);
+long long fragment_words(long long L);
+// zf (optional): zeroes the words of zf's last group past 32 * ceil(Lz / 32) columns (see launch_ternary_gemv).
+cudaError_t launch_fragments(const float* v, long long L, uint32_t* xf, uint32_t* zf, long long Lz, cudaStream_t s);
+void gemv_scratch(long long rows, long long cols, long long* partial_floats, long long* tickets);
+cudaError_t launch_ternary_gemv(const uint32_t* words, long long rows, long long cols, const uint32_t* xf,
+                                const float* scale, float* out, uint32_t* zf, float* partial, unsigned* ticket,
+                                cudaStream_t s);
 // dst[r][c] = (half) src[r][c] for an rows x cols int8 matrix
 cudaError_t launch_i8_to_f16(const int8_t* src, long long lds, int rows, int cols, __half* dst, long long ldd,
                              cudaStream_t s);
