@@ -12,6 +12,10 @@ With N > 1 (torchrun, one rank per GPU) every rank decomposes its own matrix (in
 collective on the data path): value = all ranks' components / the slowest rank's time ("scaling": "weak").
 ``--impl reference`` times the CPU oracle (the plain fp64 restatement of the method) on a bounded sample of the
 same workload: the first blocks of the same matrix, which by the greedy prefix property are the same work.
+
+``--row safeguard|refine|packed`` measures an extension instead (one GPU, its own JSON line): the decomposition
+with Prop. 2's safeguard, one refinement sweep (§2.4) of the workload's decomposition, or the packed inference
+product y = B diag(D) (C x) (§2.6) on factors of the workload's shape.
 """
 from __future__ import annotations
 
@@ -343,6 +347,136 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
+# ----------------------------------------------------------------------------------------------- extension rows
+def time_steps(torch, stream, steps, fn, flush=None):
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    out = None
+    for i in range(steps):
+        if flush is not None:
+            flush.fill_(float(i))
+        out = fn()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    return ev0.elapsed_time(ev1) / steps, out
+
+
+def run_row(args):
+    """One JSON line for an extension row, on cuda:0."""
+    import numpy as np
+    import torch
+
+    import paper_2607_13511_gb300 as X
+    from oracle import externd_next as N
+    from oracle import externd_oracle as O
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    X.load()
+    wl = workload(args.workload)
+    stream = torch.cuda.current_stream(dev)
+    k = X.rank(wl.m, wl.n, wl.mu)
+    peak, peak_src = peaks()
+    line = {"row": args.row, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "vs_baseline": None,
+            "data": "synthetic (seeded numpy PCG64; see workloads.py)", "config": config_of(wl)}
+    if args.row in ("safeguard", "refine"):
+        A_np = wl.matrix()
+        A = torch.from_numpy(A_np).to(dev)
+        h_np = wl.weights()
+        h = None if h_np is None else torch.from_numpy(h_np).to(dev)
+        flush = torch.empty(128 * 1024 * 1024, dtype=torch.float32, device=dev)   # 512 MB > L2
+        bufs = lambda: (torch.empty((wl.m, k), dtype=torch.int8, device=dev),
+                        torch.empty((k,), dtype=torch.float32, device=dev),
+                        torch.empty((k, wl.n), dtype=torch.int8, device=dev))
+        out_plain, out_ext = bufs(), bufs()
+        plain = lambda: X.decompose(A, wl.mu, wl.tau, wl.block, wl.iters, h, out=out_plain)
+        for _ in range(args.warmup):
+            dec = plain()
+        ms_plain, dec = time_steps(torch, stream, args.steps, plain, flush)
+        b = block_width(wl)
+        if args.row == "safeguard":
+            fn = lambda: X.decompose_safeguarded(A, wl.mu, wl.tau, wl.block, wl.iters, h, out=out_ext)
+            for _ in range(args.warmup):
+                fn()
+            ms, (res, act) = time_steps(torch, stream, args.steps, fn, flush)
+            kk = min(k, args.cpu_blocks * b)
+            t0 = time.perf_counter()
+            N.decompose_safeguarded(A_np, kk / min(wl.m, wl.n), wl.tau, wl.block, wl.iters, h_np)
+            dt = time.perf_counter() - t0
+            line.update({"metric": "ternary components fitted/sec per matrix, Prop. 2 safeguard on", "unit": UNIT,
+                         "value": k / (ms / 1e3), "ms_per_step": ms, "higher_is_better": True, "dtype": "f32",
+                         "energy": res.energy, "activations": act, "plain_ms_per_step": ms_plain,
+                         "overhead_vs_plain": ms / ms_plain - 1.0,
+                         "cpu_baseline": {"value": kk / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                                          "sample": f"first {kk} components of {wl.name} with the safeguard, "
+                                                    f"{dt:.1f} s"}})
+        else:
+            fn = lambda: X.refine(A, dec, wl.tau, wl.block, wl.iters, 1, h, out=out_ext)
+            for _ in range(args.warmup):
+                fn()
+            ms, (ref, rep) = time_steps(torch, stream, args.steps, fn, flush)
+            # oracle: one sweep over the first blocks' factorization (a prefix of the same run)
+            kk = min(k, max(1, args.cpu_blocks // 4) * b)
+            res_o = O.decompose(A_np, kk / min(wl.m, wl.n), wl.tau, wl.block, wl.iters, h_np)
+            t0 = time.perf_counter()
+            N.refine(A_np, res_o, wl.tau, wl.block, wl.iters, 1, h_np)
+            dt = time.perf_counter() - t0
+            line.update({"metric": "components refitted/sec (one refinement sweep, §2.4)", "unit": UNIT,
+                         "value": k / (ms / 1e3), "ms_per_step": ms, "higher_is_better": True, "dtype": "f32",
+                         "energy_before": dec.energy, "energy_after": ref.energy, "blocks_replaced": rep[0],
+                         "decompose_ms_per_step": ms_plain,
+                         "cpu_baseline": {"value": kk / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                                          "sample": f"one sweep over the first {kk} components of {wl.name}, "
+                                                    f"{dt:.1f} s"}})
+    else:   # packed inference product
+        m, n = wl.m, wl.n
+        layer_bytes = (m * k + k * n) / 4.0                    # 2 bits per ternary entry
+        copies = max(2, math.ceil(2 * 129e6 / layer_bytes))   # rotate through more than twice the L2
+        g = torch.Generator(device=dev).manual_seed(wl.seed)
+        layers = []
+        for _ in range(copies):
+            Bt = torch.randint(-1, 2, (m, k), dtype=torch.int8, device=dev, generator=g)
+            Ct = torch.randint(-1, 2, (k, n), dtype=torch.int8, device=dev, generator=g)
+            D = torch.rand(k, device=dev, generator=g) + 0.1
+            layers.append((X.pack_ternary(Bt), D, X.pack_ternary(Ct)))
+            del Bt, Ct
+        x = torch.randn(n, device=dev, generator=g)
+        for _ in range(args.warmup):
+            for L in layers:
+                X.ternary_apply(L[0], L[1], L[2], x)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for L in layers:
+                X.ternary_apply(L[0], L[1], L[2], x)
+        graph.replay()
+        ms, _ = time_steps(torch, stream, args.steps, graph.replay)
+        per_apply = ms / copies
+        bytes_apply = layer_bytes + 4 * (n + 2 * k + m)
+        achieved = bytes_apply / (per_apply / 1e3) / 1e9
+        # oracle: the float64 product on the host, a few applies of one layer
+        rng = np.random.default_rng(wl.seed)
+        Bn = rng.integers(-1, 2, (m, k)).astype(np.int8)
+        Cn = rng.integers(-1, 2, (k, n)).astype(np.int8)
+        Dn, xn = rng.random(k) + 0.1, rng.standard_normal(n)
+        reps, t0 = 0, time.perf_counter()
+        while reps < 3 or time.perf_counter() - t0 < 2.0:
+            N.ternary_apply(Bn, Dn, Cn, xn)
+            reps += 1
+        dt = (time.perf_counter() - t0) / reps
+        line.update({"metric": "packed ternary products y = B diag(D) (C x) per second", "unit": "products/s",
+                     "value": 1e3 / per_apply, "ms_per_step": ms, "higher_is_better": True, "dtype": "bf16x3 (exact f32 split)",
+                     "us_per_product": per_apply * 1e3, "layers_rotated": copies,
+                     "roofline": {"bound": "hbm", "kernel": "apply (fragments + 2 packed products)",
+                                  "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                                  "traffic": None, "peak_source": peak_src, "bytes_per_launch": bytes_apply},
+                     "gpu_launches": 3 * copies * args.steps,
+                     "cpu_baseline": {"value": 1.0 / dt, "unit": "products/s", "cores": cpu_cores(),
+                                      "kind": "oracle", "sample": f"{reps} float64 products of one {m}x{k}x{n} "
+                                                                  f"layer, {dt * reps:.1f} s"}})
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -354,8 +488,12 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-blocks", type=int, default=48, help="blocks of the workload the CPU baseline times")
     ap.add_argument("--reference-blocks", type=int, default=2, help="blocks per step of the reference arm")
+    ap.add_argument("--row", default="decompose", choices=["decompose", "safeguard", "refine", "packed"],
+                    help="an extension row instead of the headline decomposition (one GPU)")
     args = ap.parse_args()
-    if args.impl == "reference":
+    if args.row != "decompose":
+        run_row(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_gpu(args)

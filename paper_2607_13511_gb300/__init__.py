@@ -194,8 +194,9 @@ def decompose(A, mu: float, tau: float, block: int, iters: int, weights=None, ou
     return Decomposition(B, D, C, e.value, list(tr))
 
 
-def decompose_safeguarded(A, mu: float, tau: float, block: int, iters: int, weights=None):
-    """``decompose`` with Prop. 2's safeguard; returns (Decomposition, blocks replaced by a single-entry pair)."""
+def decompose_safeguarded(A, mu: float, tau: float, block: int, iters: int, weights=None, out=None):
+    """``decompose`` with Prop. 2's safeguard; returns (Decomposition, blocks replaced by a single-entry pair).
+    ``out`` may pass preallocated (B, D, C) tensors to reuse."""
     torch = _torch()
     lib = load()
     A = _prep(A, torch.float32, "A")
@@ -203,9 +204,12 @@ def decompose_safeguarded(A, mu: float, tau: float, block: int, iters: int, weig
     k = rank(m, n, mu)
     nblocks = -(-k // block_width(m, n, block))
     h = None if weights is None else _prep(weights, torch.float32, "weights")
-    B = torch.empty((m, k), dtype=torch.int8, device=A.device)
-    D = torch.empty((k,), dtype=torch.float32, device=A.device)
-    C = torch.empty((k, n), dtype=torch.int8, device=A.device)
+    if out is None:
+        B = torch.empty((m, k), dtype=torch.int8, device=A.device)
+        D = torch.empty((k,), dtype=torch.float32, device=A.device)
+        C = torch.empty((k, n), dtype=torch.int8, device=A.device)
+    else:
+        B, D, C = out
     e = _c_double()
     tr = (_c_double * nblocks)()
     act = _c_i64()
@@ -216,14 +220,21 @@ def decompose_safeguarded(A, mu: float, tau: float, block: int, iters: int, weig
     return Decomposition(B, D, C, e.value, list(tr)), act.value
 
 
-def refine(A, dec: Decomposition, tau: float, block: int, iters: int, sweeps: int, weights=None):
+def refine(A, dec: Decomposition, tau: float, block: int, iters: int, sweeps: int, weights=None, out=None):
     """§2.4 refinement sweeps of ``dec``'s factors (same block layout as the run that made them). Returns
-    (Decomposition with new factors, blocks replaced per sweep); ``dec``'s tensors are left untouched."""
+    (Decomposition with new factors, blocks replaced per sweep); ``dec``'s tensors are left untouched. ``out`` may
+    pass preallocated (B, D, C) tensors that receive the factors (they are copied from ``dec`` first)."""
     torch = _torch()
     lib = load()
     A = _prep(A, torch.float32, "A")
     m, n = A.shape
-    B, D, C = dec.B.clone(), dec.D.clone(), dec.C.clone()
+    if out is None:
+        B, D, C = dec.B.clone(), dec.D.clone(), dec.C.clone()
+    else:
+        B, D, C = out
+        B.copy_(dec.B)
+        D.copy_(dec.D)
+        C.copy_(dec.C)
     k = B.shape[1]
     h = None if weights is None else _prep(weights, torch.float32, "weights")
     e = _c_double()

@@ -89,11 +89,24 @@ __global__ void __launch_bounds__(256) safeguard_decide_kernel(const EntryBest* 
                                                                const float* __restrict__ r, float* __restrict__ d,
                                                                const float* __restrict__ K, int w,
                                                                BlockChoice* __restrict__ choice) {
-  const double dec = block_decrease(r, d, K, w);
+  // the best of the per-CTA entries: strided over the threads, then a warp and a CTA reduction (same order rule)
+  EntryBest b{-1.f, 0.f, ~0ull};
+  for (int k = threadIdx.x; k < nparts; k += blockDim.x) {
+    const EntryBest c = part[k];
+    if (better(c.score, c.idx, b.score, b.idx)) b = c;
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    const float s2 = __shfl_xor_sync(0xffffffffu, b.score, o), r2 = __shfl_xor_sync(0xffffffffu, b.rij, o);
+    const unsigned long long i2 = __shfl_xor_sync(0xffffffffu, b.idx, o);
+    if (better(s2, i2, b.score, b.idx)) b = EntryBest{s2, r2, i2};
+  }
+  __shared__ EntryBest wb[8];
+  if ((threadIdx.x & 31) == 0) wb[threadIdx.x >> 5] = b;
+  const double dec = block_decrease(r, d, K, w);   // contains a CTA barrier, after which wb is complete
   if (threadIdx.x != 0) return;
-  EntryBest b = part[0];
-  for (int k = 1; k < nparts; ++k)
-    if (better(part[k].score, part[k].idx, b.score, b.idx)) b = part[k];
+  b = wb[0];
+  for (int k = 1; k < (int)(blockDim.x >> 5); ++k)
+    if (better(wb[k].score, wb[k].idx, b.score, b.idx)) b = wb[k];
   const long long i = (long long)(b.idx / (unsigned long long)n), j = (long long)(b.idx % (unsigned long long)n);
   const double single = (h != nullptr ? (double)h[j] : 1.0) * (double)b.rij * (double)b.rij;
   const int take = single > dec ? 1 : 0;
