@@ -239,7 +239,7 @@ struct Plan {
 
 struct Bufs {
   float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE, *maxpart, *maxabs, *theta;
-  unsigned *err, *arg, *ticket;
+  unsigned *err, *arg, *ticket, *bar;
   int *fallback, *GintU, *GintV;
   GramScratch gram;   // per-CTA partials and group tickets of the fused Gram
   int8_t *Ut, *Vt;
@@ -287,6 +287,7 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "fallback", (size_t)w, &B->fallback));
   TRY(need(ws, "arg", (size_t)w, &B->arg));
   TRY(need(ws, "ticket", 1, &B->ticket, true));
+  TRY(need(ws, "bar", 3, &B->bar, true));
   TRY(need(ws, "GintU", (size_t)w * w, &B->GintU, true));
   TRY(need(ws, "GintV", (size_t)w * w, &B->GintV, true));
   {
@@ -394,6 +395,31 @@ Eq2 make_eq2(const Plan& p, const Bufs& B) {
   return e;
 }
 
+// The fused decorrelation + ternarization (one cooperative grid) where it applies; EXTERND_FUSED=0 keeps the
+// two kernels everywhere, for comparisons.
+bool fused_enabled() {
+  static const bool enabled = [] {
+    const char* e = std::getenv("EXTERND_FUSED");
+    return !(e && std::strcmp(e, "0") == 0);
+  }();
+  return enabled;
+}
+
+// Eq. 3 targets of the product partials and Eq. 2 on them: T (and its fp16 / K-major copies, its integer Gram).
+int targets_step(const Bufs& B, const float* Ginv, int w, int splits, int L, const Stats& st, int8_t* T, int ldt,
+                 int* gram, __half* T16, long long ldt16, __half* Tk, cudaStream_t s) {
+  if (fused_enabled() && decorrelate_apply_fits(w, L)) {
+    bool used = false;
+    KL(kDecor, 1, launch_decorrelate_apply(Ginv, w, B.part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, B.ldk, B.bar,
+                                           B.err, s, &used));
+    if (used) return EXTERND_OK;
+    return cuda_fail(cudaErrorInvalidValue, "launch_decorrelate_apply");
+  }
+  KL(kDecor, 1, launch_decorrelate(Ginv, w, B.part, splits, L, B.X, L, st, s));
+  KL(kApply, 1, launch_apply(B.X, w, L, L, st.th, T, ldt, gram, s, T16, ldt16, Tk, B.ldk, B.gram));
+  return EXTERND_OK;
+}
+
 // The ALS fit of one block of w components (§2.3 for w = 1, §2.4): `iters` V-step / U-step pairs, ending with U
 // in Ut (and its exact Gram where fused), V in Vt, the K-major fp16 copies for the tensor-core deflation, and the
 // last U-step product in B.part. With `staged` the caller has put the starting U in Ut (and Ut16) -- a refinement
@@ -434,9 +460,8 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
     }
     KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
     if (w > 1) JOIN();
-    KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, sv, n, B.X, n, q.st_n, s));
-    KL(kApply, 1, launch_apply(B.X, w, n, n, q.th_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, s, V16, p.ldn,
-                               (last && use_tc(w)) ? B.Vk16 : nullptr, B.ldk, B.gram));
+    TRY(targets_step(B, w > 1 ? B.Ginv : B.one, w, sv, n, q.st_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, V16,
+                     p.ldn, (last && use_tc(w)) ? B.Vk16 : nullptr, s));
     // U-step: U <- T(R H V (V^T H V + eps I)^-1)
     FORK();
     if (fusedV) {
@@ -447,12 +472,11 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
     }
     KL(kUstep, 1, product_u(B.R, m, n, B.Vt, V16, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s));
     JOIN();
-    KL(kDecor, 1, launch_decorrelate(w > 1 ? B.Ginv : B.one, w, B.part, su, m, B.X, m, q.st_m, s));
     // the next V-step's inverse (w > 1) or, after the last iteration, Eq. 4 consumes U's Gram
     // (the fp16 copy of U is not needed after the last iteration)
-    KL(kApply, 1, launch_apply(B.X, w, m, m, q.th_m, B.Ut, (int)p.ldm, (fusedU && (w > 1 || last)) ? B.GintU : nullptr,
-                               s, last ? nullptr : U16, p.ldm, (last && use_tc(w)) ? B.Uk16 : nullptr, B.ldk,
-                               B.gram));
+    TRY(targets_step(B, w > 1 ? B.Ginv : B.one, w, su, m, q.st_m, B.Ut, (int)p.ldm,
+                     (fusedU && (w > 1 || last)) ? B.GintU : nullptr, last ? nullptr : U16, p.ldm,
+                     (last && use_tc(w)) ? B.Uk16 : nullptr, s));
   }
   return EXTERND_OK;
 }
@@ -698,6 +722,8 @@ int check_device_error(Workspace& ws, unsigned* err, cudaStream_t s) {
   CK(cudaStreamSynchronize(s));
   if (*static_cast<unsigned*>(hb) != 0u) {
     CK(cudaMemsetAsync(err, 0, sizeof(unsigned), s));
+    auto bar = ws.bufs.find("bar");   // a grid that gave up may have left its barrier counters set
+    if (bar != ws.bufs.end() && bar->second.p != nullptr) CK(cudaMemsetAsync(bar->second.p, 0, bar->second.cap, s));
     CK(cudaStreamSynchronize(s));
     return EXTERND_ETIMEOUT;
   }

@@ -302,6 +302,337 @@ cudaError_t launch_decorrelate_dx(const float* Ginv, int w, const float* part, i
   return cudaGetLastError();
 }
 
+// ---- Decorrelation and ternarization in one cooperative grid (w <= 64 components) ------------------------------
+//
+// The same X tile as decorrelate_kernel (thread (ty, tx): components 4ty .. 4ty + 3, positions tx * PX ..), kept in
+// registers; then
+//   barrier 1 -- every CTA has written its Eq. 2 statistics chunk;
+//   each CTA finalizes the thresholds of vectors blockIdx.x, blockIdx.x + grid, ... from all chunks;
+//   barrier 2 -- every threshold is written;
+//   each CTA ternarizes its tile (int8 rows, optional fp16 rows and K-major fp16) and adds its positions' exact
+//   Gram entries (bitplanes in shared memory, popcounts, integer atomics into the upper triangle).
+// This replaces two launches, the serial tail of the last-CTA finalize and the round trip of X through memory.
+// The grid is launched cooperatively (all CTAs resident); each barrier is a device-scope counter that thread 0
+// of every CTA increments with release semantics and polls with acquire loads, giving up after kWaitNs (error
+// word set, the CTA skips the rest). Counter 0 is reset by CTA 0 after barrier 2 (everyone has left barrier 1),
+// counters 1 and 2 by the last CTA to finish (an exit ticket), so the next launch finds them at zero.
+constexpr unsigned long long kGridWaitNs = 2000000000ull;   // 2 s
+
+__device__ __forceinline__ unsigned long long grid_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Grid barrier on ctr (see above); false after a timeout (then err holds 1).
+__device__ __forceinline__ bool grid_barrier(unsigned* ctr, unsigned target, unsigned* err) {
+  __shared__ int s_ok;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
+    int ok = 1;
+    const unsigned long long t0 = grid_ns();
+    for (unsigned it = 0;; ++it) {
+      unsigned v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+      if (v >= target) break;
+      if ((it & 63u) == 63u && grid_ns() - t0 > kGridWaitNs) {
+        atomicOr(err, 1u);
+        ok = 0;
+        break;
+      }
+    }
+    __threadfence();
+    s_ok = ok;
+  }
+  __syncthreads();
+  return s_ok != 0;
+}
+
+template <int DXT>
+__global__ void __launch_bounds__(256, 2) decorrelate_apply_kernel(const float* __restrict__ Ginv, int w,
+                                                                const float* __restrict__ part, int splits, int L,
+                                                                Stats st, int8_t* __restrict__ T, long long ldt,
+                                                                int* __restrict__ gram, __half* __restrict__ T16,
+                                                                long long ldt16, __half* __restrict__ Tk,
+                                                                long long ldk, unsigned* __restrict__ bar,
+                                                                unsigned* __restrict__ err) {
+  constexpr int PX = DXT / 16, NW = (DXT + 31) / 32;
+  extern __shared__ __align__(16) float dsm[];
+  float* const Ps = dsm;                 // [w][DXT]
+  float* const Gs = dsm + w * DXT;       // [w][kGsLd]
+  __shared__ unsigned mz[TM][NW], mp[TM][NW];   // nonzero / positive bitplanes of the tile
+  const int x0 = blockIdx.x * DXT;
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const unsigned G = gridDim.x;
+
+  // ---- X tile = Ginv (sum_s part[s])[:, x0 .. x0 + DXT) (as decorrelate_kernel, a0 = 0)
+  {
+    constexpr int Q = DXT / 4, NB = 8;
+    const bool pvec = (L & 3) == 0, gvec = (w & 3) == 0;
+    const long long sstride = (long long)w * L;
+    const int nps = w * Q, pper = (nps + 255) / 256, nld = pper * splits;
+    const int ngs = w * 16, gper = (ngs + 255) / 256;
+    constexpr int GB = 4;
+    float4 g[GB];
+#pragma unroll
+    for (int q = 0; q < GB; ++q) {
+      const int i = q * 256 + tid;
+      g[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (q < gper && i < ngs) g[q] = load4(Ginv + (long long)(i >> 4) * w, (i & 15) * 4, w, gvec);
+    }
+    for (int f0 = 0; f0 < nld; f0 += NB) {
+      float4 v[NB];
+      int e = f0 / splits, sp = f0 - e * splits;
+#pragma unroll
+      for (int k = 0; k < NB; ++k) {
+        const int i = e * 256 + tid;
+        v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (f0 + k < nld && i < nps)
+          v[k] = load4(part + sp * sstride + (long long)(i / Q) * L, x0 + (i % Q) * 4, L, pvec);
+        if (++sp == splits) {
+          sp = 0;
+          ++e;
+        }
+      }
+      e = f0 / splits;
+      sp = f0 - e * splits;
+#pragma unroll
+      for (int k = 0; k < NB; ++k) {
+        const int i = e * 256 + tid;
+        if (f0 + k < nld && i < nps) {
+          float4* dst = reinterpret_cast<float4*>(&Ps[(i / Q) * DXT + (i % Q) * 4]);
+          if (sp == 0) {
+            *dst = v[k];
+          } else {
+            float4 t = *dst;
+            t.x += v[k].x;
+            t.y += v[k].y;
+            t.z += v[k].z;
+            t.w += v[k].w;
+            *dst = t;
+          }
+        }
+        if (++sp == splits) {
+          sp = 0;
+          ++e;
+        }
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < GB; ++q) {
+      const int i = q * 256 + tid;
+      if (q < gper && i < ngs) *reinterpret_cast<float4*>(&Gs[(i >> 4) * kGsLd + (i & 15) * 4]) = g[q];
+    }
+    for (int i = tid; i < TM * NW; i += 256) {
+      (&mz[0][0])[i] = 0u;
+      (&mp[0][0])[i] = 0u;
+    }
+  }
+  __syncthreads();
+
+  float acc[4][PX];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < PX; ++j) acc[i][j] = 0.f;
+#pragma unroll 4
+  for (int b = 0; b < w; ++b) {
+    const float4 g = *reinterpret_cast<const float4*>(&Gs[b * kGsLd + ty * 4]);
+    float p[PX];
+#pragma unroll
+    for (int j = 0; j < PX; ++j) p[j] = Ps[b * DXT + tx * PX + j];
+    const float gv[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < PX; ++j) acc[i][j] = fmaf(gv[i], p[j], acc[i][j]);
+  }
+
+  // ---- Eq. 2 statistics of this chunk (one per CTA)
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int a = ty * 4 + i;
+    AbsSum sum;
+    u64 key = 0;
+    if (a < w) {
+#pragma unroll
+      for (int j = 0; j < PX; ++j) {
+        const int x = x0 + tx * PX + j;
+        if (x < L) {
+          sum.add(acc[i][j]);
+          const u64 kk = mag_key(acc[i][j], (uint32_t)x);
+          key = kk > key ? kk : key;
+        }
+      }
+    }
+    F2 sv = sum.acc;
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) {
+      sv = f2_add(sv, f2_shfl_xor(sv, o));
+      const u64 t = __shfl_xor_sync(0xffffffffu, key, o);
+      key = t > key ? t : key;
+    }
+    if (tx == 0 && a < w) put_stat(st, a, blockIdx.x, sv, key);
+  }
+  if (!grid_barrier(bar + 0, G, err)) return;
+
+  // ---- thresholds of vectors blockIdx.x, blockIdx.x + G, ...: all chunks, fixed-order CTA reduction
+  {
+    __shared__ F2 rs[8];
+    __shared__ u64 rk[8];
+    for (int a = blockIdx.x; a < w; a += G) {
+      F2 sv;
+      u64 key = 0;
+      const uint4* pp = reinterpret_cast<const uint4*>(st.part + (long long)a * st.nchunk);
+      for (int c = tid; c < st.nchunk; c += 256) {
+        const uint4 r = __ldcg(pp + c);
+        F2 t;
+        t.hi = __uint_as_float(r.x);
+        t.lo = __uint_as_float(r.y);
+        sv = f2_add(sv, t);
+        const u64 kk = ((u64)r.w << 32) | r.z;
+        key = kk > key ? kk : key;
+      }
+      for (int o = 16; o > 0; o >>= 1) {
+        sv = f2_add(sv, f2_shfl_xor(sv, o));
+        const u64 t = __shfl_xor_sync(0xffffffffu, key, o);
+        key = t > key ? t : key;
+      }
+      if ((tid & 31) == 0) {
+        rs[tid >> 5] = sv;
+        rk[tid >> 5] = key;
+      }
+      __syncthreads();
+      if (tid == 0) {
+        F2 tot = rs[0];
+        u64 kmax = rk[0];
+        for (int q = 1; q < 8; ++q) {
+          tot = f2_add(tot, rs[q]);
+          kmax = rk[q] > kmax ? rk[q] : kmax;
+        }
+        const float th = __double2float_rd(st.th.tau * (f2_value(tot) / (double)st.th.L));
+        st.th.theta[a] = th;
+        st.th.fallback[a] = !(key_mag(kmax) > th);
+        st.th.arg[a] = key_index(kmax);
+      }
+      __syncthreads();
+    }
+  }
+  if (!grid_barrier(bar + 1, G, err)) return;
+  if (blockIdx.x == 0 && tid == 0) bar[0] = 0u;   // everyone has left barrier 1
+
+  // ---- ternarize the tile, write the factor layouts, bitplanes for the Gram
+  {
+    float thv[4];
+    int fbv[4];
+    unsigned argv[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int a = ty * 4 + i;
+      thv[i] = a < w ? __ldcg(st.th.theta + a) : 0.f;
+      fbv[i] = a < w ? __ldcg(st.th.fallback + a) : 0;
+      argv[i] = a < w ? __ldcg(st.th.arg + a) : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < PX; ++j) {
+      const int xl = tx * PX + j, x = x0 + xl;
+      if (x >= L) continue;
+      short tk[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int a = ty * 4 + i;
+        int8_t t = 0;
+        if (a < w) {
+          t = ternary_of(acc[i][j], thv[i]);
+          if (fbv[i] && (uint32_t)x == argv[i]) t = acc[i][j] < 0.f ? (int8_t)-1 : (int8_t)1;
+          T[(long long)a * ldt + x] = t;
+          if (T16 != nullptr) T16[(long long)a * ldt16 + x] = __short2half_rn((short)t);
+          if (gram != nullptr && t != 0) {
+            atomicOr(&mz[a][xl >> 5], 1u << (xl & 31));
+            if (t > 0) atomicOr(&mp[a][xl >> 5], 1u << (xl & 31));
+          }
+        }
+        tk[i] = t;
+      }
+      if (Tk != nullptr) {   // components 4ty .. 4ty + 3 of position x: 8 bytes (ldk is a multiple of 8)
+        __half* dst = Tk + (long long)x * ldk + ty * 4;
+        if (ty * 4 + 3 < w) {
+          const __half2 h01 = __halves2half2(__short2half_rn(tk[0]), __short2half_rn(tk[1]));
+          const __half2 h23 = __halves2half2(__short2half_rn(tk[2]), __short2half_rn(tk[3]));
+          uint2 u;
+          u.x = *reinterpret_cast<const unsigned*>(&h01);
+          u.y = *reinterpret_cast<const unsigned*>(&h23);
+          *reinterpret_cast<uint2*>(dst) = u;
+        } else {
+          for (int i = 0; i < 4 && ty * 4 + i < w; ++i) dst[i] = __short2half_rn(tk[i]);
+        }
+      }
+    }
+  }
+  if (gram != nullptr) {
+    __syncthreads();
+    // G_ab += popc(Z_a & Z_b) - 2 popc(Z_a & Z_b & (P_a ^ P_b)) over this tile's positions, a <= b
+    for (int idx = tid; idx < w * w; idx += 256) {
+      const int a = idx / w, b = idx - a * w;
+      if (b < a) continue;
+      int v = 0;
+#pragma unroll
+      for (int q = 0; q < NW; ++q) {
+        const unsigned zz = mz[a][q] & mz[b][q];
+        v += __popc(zz) - 2 * __popc(zz & (mp[a][q] ^ mp[b][q]));
+      }
+      if (v != 0) atomicAdd(&gram[(long long)a * w + b], v);
+    }
+  }
+  // ---- exit ticket: the last CTA resets barrier 2 and the ticket
+  __syncthreads();
+  if (tid == 0) {
+    unsigned old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(bar + 2) : "memory");
+    if (old == G - 1u) {
+      bar[1] = 0u;
+      bar[2] = 0u;
+    }
+  }
+}
+
+template <int DXT>
+cudaError_t launch_decorrelate_apply_dx(const float* Ginv, int w, const float* part, int splits, int L, Stats st,
+                                        int8_t* T, long long ldt, int* gram, __half* T16, long long ldt16, __half* Tk,
+                                        long long ldk, unsigned* bar, unsigned* err, cudaStream_t s, bool* used) {
+  static int max_grid = -1;
+  if (max_grid < 0) {
+    cudaError_t e = cudaFuncSetAttribute(decorrelate_apply_kernel<DXT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)decorrelate_smem(TM, DXT));
+    if (e != cudaSuccess) return e;
+    int per_sm = 0, sms = 0, dev = 0;
+    e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e == cudaSuccess)
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decorrelate_apply_kernel<DXT>, 256,
+                                                        decorrelate_smem(TM, DXT));
+    if (e != cudaSuccess) return e;
+    max_grid = per_sm * sms;
+  }
+  const int grid = (int)cdiv(L, DXT);
+  *used = grid <= max_grid;
+  if (!*used) return cudaSuccess;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(256);
+  cfg.dynamicSmemBytes = decorrelate_smem(w, DXT);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decorrelate_apply_kernel<DXT>, Ginv, w, part, splits, L, st, T, ldt, gram, T16,
+                            ldt16, Tk, ldk, bar, err);
+}
+
 template <bool UROW>
 __global__ void __launch_bounds__(256) deflate_kernel(const float* Rin, float* Rout, int m, int n,
                                                       const int8_t* __restrict__ U, long long ldu,
@@ -481,6 +812,43 @@ cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int 
     case 32: return launch_decorrelate_dx<32>(Ginv, w, part, splits, L, X, ldx, st, s);
     case 64: return launch_decorrelate_dx<64>(Ginv, w, part, splits, L, X, ldx, st, s);
     default: return launch_decorrelate_dx<128>(Ginv, w, part, splits, L, X, ldx, st, s);
+  }
+}
+
+bool decorrelate_apply_fits(int w, int L) {
+  if (w > TM) return false;
+  int dx = decorrelate_dx(L, w), per_sm = 0, sms = 0, dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return false;
+  cudaError_t e = cudaSuccess;
+  switch (dx) {
+    case 16: e = cudaFuncSetAttribute(decorrelate_apply_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)decorrelate_smem(TM, 16));
+             if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decorrelate_apply_kernel<16>, 256, decorrelate_smem(TM, 16)); break;
+    case 32: e = cudaFuncSetAttribute(decorrelate_apply_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)decorrelate_smem(TM, 32));
+             if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decorrelate_apply_kernel<32>, 256, decorrelate_smem(TM, 32)); break;
+    case 64: e = cudaFuncSetAttribute(decorrelate_apply_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)decorrelate_smem(TM, 64));
+             if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decorrelate_apply_kernel<64>, 256, decorrelate_smem(TM, 64)); break;
+    default: e = cudaFuncSetAttribute(decorrelate_apply_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)decorrelate_smem(TM, 128));
+             if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decorrelate_apply_kernel<128>, 256, decorrelate_smem(TM, 128)); break;
+  }
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return cdiv(L, dx) <= (long long)per_sm * sms;
+}
+
+cudaError_t launch_decorrelate_apply(const float* Ginv, int w, const float* part, int splits, int L, Stats st,
+                                     int8_t* T, long long ldt, int* gram, __half* T16, long long ldt16, __half* Tk,
+                                     long long ldk, unsigned* bar, unsigned* err, cudaStream_t s, bool* used) {
+  *used = false;
+  if (w > TM || st.nchunk != decorrelate_chunks(L, w)) return cudaSuccess;
+  if (Tk != nullptr && (ldk < round_up(w, 8) || (ldk & 7) != 0)) return cudaErrorInvalidValue;
+  switch (decorrelate_dx(L, w)) {
+    case 16: return launch_decorrelate_apply_dx<16>(Ginv, w, part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, ldk, bar, err, s, used);
+    case 32: return launch_decorrelate_apply_dx<32>(Ginv, w, part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, ldk, bar, err, s, used);
+    case 64: return launch_decorrelate_apply_dx<64>(Ginv, w, part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, ldk, bar, err, s, used);
+    default: return launch_decorrelate_apply_dx<128>(Ginv, w, part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, ldk, bar, err, s, used);
   }
 }
 

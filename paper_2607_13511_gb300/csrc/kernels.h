@@ -132,6 +132,15 @@ cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int
 int decorrelate_chunks(int L, int w);
 cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
                                Stats st, cudaStream_t s);
+// The decorrelation followed by the ternarization of its output (launch_decorrelate + launch_apply, with X kept
+// on chip) in one cooperative grid, for w <= 64 and grids that fit the GPU at once; *used tells whether it ran
+// (if not, nothing was launched and the caller runs the two kernels). T16 / Tk / gram as launch_apply's (gram:
+// the integer upper triangle, added to). bar: 3 words, zero, left zero; err: the device error word (a barrier
+// that waited 2 s sets it, and the rest of the grid's work is skipped).
+bool decorrelate_apply_fits(int w, int L);
+cudaError_t launch_decorrelate_apply(const float* Ginv, int w, const float* part, int splits, int L, Stats st,
+                                     int8_t* T, long long ldt, int* gram, __half* T16, long long ldt16, __half* Tk,
+                                     long long ldk, unsigned* bar, unsigned* err, cudaStream_t s, bool* used);
 // Rout = Rin - U diag(d) V (Rout may alias Rin or be NULL); U is Ut (component-major, ldu) or, when
 // u_rowmajor, an m x ldu row-major block of B. colpart: [cdiv(m,64)][n] per-tile column sums of Rout^2 (or NULL);
 // normpart: [cdiv(m,64) * cdiv(n,128)] per-tile sums of h_j Rout_ij^2.
