@@ -194,8 +194,19 @@ bool use_tma() {
   }();
   return enabled;
 }
-int splits_v(int w, int m, int n) { return use_tc(w) ? tc_product_splits(w, n, m) : product_splits(w, n, m); }
-int splits_u(int w, int m, int n) { return use_tc(w) ? tc_product_splits(w, m, n) : product_splits(w, m, n); }
+// Partial slots of a product: the kernel that will run decides (product_v / product_u make the same choice).
+int splits_of(int w, int Lx, int Ly, bool tma) {
+  if (!use_tc(w)) return product_splits(w, Lx, Ly);
+  return tma ? tma_product_slots(w, Lx, Ly) : tc_product_splits(w, Lx, Ly);
+}
+int splits_v(int w, int m, int n, const float* R, const __half* T16, int ld) {
+  return splits_of(w, n, m, use_tma() && T16 != nullptr && tma_product_ok(R, n, T16, ld));
+}
+int splits_u(int w, int m, int n, const float* R, const __half* T16, int ld) {
+  return splits_of(w, m, n, use_tma() && T16 != nullptr && tma_product_ok(R, n, T16, ld));
+}
+// The most slots either kernel can use (workspace sizing).
+int splits_max(int w, int Lx, int Ly) { return std::max(splits_of(w, Lx, Ly, false), splits_of(w, Lx, Ly, true)); }
 
 // The factor comes as int8 rows (FMA tiles) and as the same values in fp16 rows (tensor cores), both with
 // leading dimension ld elements.
@@ -276,8 +287,8 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   size_t part = 0;
   for (long long wi : {(long long)p.b, p.k % p.b}) {
     if (wi < 1) continue;
-    part = std::max(part, (size_t)std::max((long long)splits_v((int)wi, p.m, p.n) * wi * p.n,
-                                           (long long)splits_u((int)wi, p.m, p.n) * wi * p.m));
+    part = std::max(part, (size_t)std::max((long long)splits_max((int)wi, p.n, p.m) * wi * p.n,
+                                           (long long)splits_max((int)wi, p.m, p.n) * wi * p.m));
   }
   TRY(need(ws, "part", part, &B->part));
   TRY(need(ws, "maxpart", (size_t)deflate_tiles(p.m, p.n), &B->maxpart));
@@ -429,7 +440,8 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
   cudaStream_t side = ws.side;
   const int m = p.m, n = p.n;
   const int nrt = deflate_row_tiles(m);
-  const int sv = splits_v(w, m, n), su = splits_u(w, m, n);
+  const int sv = splits_v(w, m, n, B.R, use_tc(w) ? B.Ut16 : nullptr, (int)p.ldm);
+  const int su = splits_u(w, m, n, B.R, use_tc(w) ? B.Vt16 : nullptr, (int)p.ldn);
   q.st_m.nchunk = decorrelate_chunks(m, w);
   q.st_n.nchunk = decorrelate_chunks(n, w);
   // Exact Gram matrices of unweighted ternary factors are accumulated by the apply that writes the factor
@@ -485,7 +497,7 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
 // the matrix without the ridge.
 int block_scales_step(const Plan& p, const Bufs& B, int w, float* K, cudaStream_t s) {
   const int m = p.m, n = p.n;
-  const int su = splits_u(w, m, n);
+  const int su = splits_u(w, m, n, B.R, use_tc(w) ? B.Vt16 : nullptr, (int)p.ldn);
   KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, su, B.r, s));
   if (w <= 128) {
     KL(kSolve, 1, launch_scales_int(B.GintU, B.GrawV, B.r, w, B.d, s, K));
@@ -1032,7 +1044,7 @@ int externd_vstep_product(const float* R, int64_t m, int64_t n, const int8_t* U,
   unsigned* err;
   TRY(stage_u(*ws, U, m, (int)w, &Ut, &U16));
   TRY(step_scalars(*ws, R, m * n, nullptr, 0, &mx, &err));
-  const int sv = splits_v((int)w, (int)m, (int)n);
+  const int sv = splits_v((int)w, (int)m, (int)n, R, U16, (int)ld16(m));
   TRY(need(*ws, "part", (size_t)sv * w * n, &part));
   LK(product_v(R, (int)m, (int)n, Ut, U16, (int)ld16(m), (int)w, part, sv, mx, err, g_stream));
   LK(launch_sum_splits(part, sv, (int)w, (int)n, PV, n, g_stream));
@@ -1054,7 +1066,7 @@ int externd_ustep_product(const float* R, int64_t m, int64_t n, const int8_t* Cb
   unsigned* err;
   TRY(stage_v(*ws, Cb, n, (int)w, &Vt, &V16));
   TRY(step_scalars(*ws, R, m * n, weights, n, &mx, &err));
-  const int su = splits_u((int)w, (int)m, (int)n);
+  const int su = splits_u((int)w, (int)m, (int)n, R, V16, (int)ld16(n));
   TRY(need(*ws, "part", (size_t)su * w * m, &part));
   TRY(need(*ws, "X", (size_t)w * m, &X));
   LK(product_u(R, (int)m, (int)n, Vt, V16, (int)ld16(n), (int)w, weights, part, su, mx, err, g_stream));
@@ -1081,7 +1093,7 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   float* mx;
   unsigned* err;
   TRY(step_scalars(*ws, R, m * n, vstep ? nullptr : h, n, &mx, &err));
-  const int splits = vstep ? splits_v(w, (int)m, (int)n) : splits_u(w, (int)m, (int)n);
+  const int splits = vstep ? splits_v(w, (int)m, (int)n, R, T16, (int)ldt) : splits_u(w, (int)m, (int)n, R, T16, (int)ldt);
   const int gs = gram_splits(w, (int)Lred);
   TRY(need(*ws, "part", (size_t)splits * w * L, &part));
   TRY(need(*ws, "X", (size_t)w * L, &X));
@@ -1150,7 +1162,7 @@ int externd_block_scales(const float* R, int64_t m, int64_t n, const int8_t* U, 
   TRY(stage_u(*ws, U, m, (int)w, &Ut));
   TRY(stage_v(*ws, Cb, n, (int)w, &Vt, &V16));
   TRY(step_scalars(*ws, R, m * n, weights, n, &mx, &err));
-  const int su = splits_u((int)w, (int)m, (int)n);
+  const int su = splits_u((int)w, (int)m, (int)n, R, V16, (int)ld16(n));
   const int gm = gram_splits((int)w, (int)m), gn = gram_splits((int)w, (int)n);
   TRY(need(*ws, "part", (size_t)su * w * m, &part));
   TRY(need(*ws, "Gpart", (size_t)std::max(gm, gn) * w * w, &Gpart));

@@ -172,6 +172,8 @@ void tc_split(int w, int Lx, int Ly, int* splits, int* chunk);
 // TMA-fed products (product_tma.cu): same contract as the launch_product_*_tc above; usable when
 // tma_product_ok (R and the factor 16-byte aligned, n % 4 == 0, factor ld a multiple of 8).
 bool tma_product_ok(const float* R, int n, const __half* T, int ldt);
+// Partial slots the TMA-fed product writes (its classic split count, or more under its stream plan).
+int tma_product_slots(int w, int Lx, int Ly);
 cudaError_t launch_product_v_tma(const float* R, int m, int n, const __half* Ut, int ldu, int w, float* part,
                                  int splits, const float* maxabs, unsigned* err, cudaStream_t s);
 cudaError_t launch_product_u_tma(const float* R, int m, int n, const __half* Vt, int ldv, int w, const float* h,

@@ -16,6 +16,15 @@
 //                          free the A and B slots
 // R never passes through registers on its way into shared memory, so the loads of several stages are in flight
 // per SM without any register cost.
+//
+// Work is a sequence of units (128 positions x 64 reduction rows), tile-major. Classic plan: CTA (tile, split)
+// takes one tile's units of its split, and writes partial slot `split`. Stream plan, used when tiles x splits
+// would fill every SM (the w x w inverse runs beside the product on one SM, so one CTA of such a grid would wait
+// for it): a 1-D grid of SMs - 1 CTAs splits all units evenly into contiguous runs; a run that crosses a tile
+// boundary accumulates each tile in its own TMEM buffer (two, alternating) and writes each to the slot numbered
+// by its place among the runs meeting that tile; slots a tile has no run for are written with zeros by the run
+// that ends the tile. The converter warps store a finished tile's partials as soon as they have converted the
+// next tile's last unit, so the MMAs keep going.
 #include <cuda.h>
 
 #include "kernels.h"
@@ -37,11 +46,14 @@ struct TmaArgs {
   int m, n, w, wpad;
   const float* h;
   float* part;
-  int ychunk;
   const float* maxabs;
   unsigned* err;
   int s32, sb, s16;
   uint32_t tmem_cols;
+  int nkt;             // units per tile: cdiv(Ly, 64)
+  int cu;              // classic: units per split
+  long long U;         // stream: all units (tiles x nkt)
+  int slots;           // partial slots (classic: splits)
 };
 
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
@@ -69,7 +81,11 @@ __device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uin
   lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
-template <bool USTEP>
+__device__ __forceinline__ long long unit_owner(long long u, long long U, long long G) {
+  return ((u + 1) * G + U - 1) / U - 1;   // the CTA whose run holds unit u (stream plan)
+}
+
+template <bool USTEP, bool STREAM>
 __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_constant__ CUtensorMap mapR,
                                                                   const __grid_constant__ CUtensorMap mapT,
                                                                   const TmaArgs p) {
@@ -85,16 +101,22 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
   const uint32_t full32 = bars, empty32 = full32 + 8u * p.s32;
   const uint32_t fullB = empty32 + 8u * p.s32, emptyB = fullB + 8u * p.sb;
   const uint32_t full16 = emptyB + 8u * p.sb, empty16 = full16 + 8u * p.s16;
-  const uint32_t done_bar = empty16 + 8u * p.s16;
-  const uint32_t tmem_slot = done_bar + 8u;
+  const uint32_t accfull = empty16 + 8u * p.s16, accempty = accfull + 16u;   // two TMEM accumulators
+  const uint32_t tmem_slot = accempty + 16u;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int Lx = USTEP ? p.m : p.n;
   const int Ly = USTEP ? p.n : p.m;
-  const int x0 = blockIdx.x * 128;
-  const int ybeg = blockIdx.z * p.ychunk;
-  const int yend = min(Ly, ybeg + p.ychunk);
-  const int nk = ybeg < yend ? (int)cdiv(yend - ybeg, kStageK) : 0;
+  // this CTA's run of units [u0, u1)
+  long long u0, u1;
+  if (STREAM) {
+    u0 = (long long)blockIdx.x * p.U / gridDim.x;
+    u1 = ((long long)blockIdx.x + 1) * p.U / gridDim.x;
+  } else {
+    u0 = (long long)blockIdx.x * p.nkt + (long long)blockIdx.z * p.cu;
+    u1 = min(u0 + p.cu, ((long long)blockIdx.x + 1) * p.nkt);
+  }
+  const int nk = (int)(u1 > u0 ? u1 - u0 : 0);
 
   float mx = __ldg(p.maxabs);
   if (USTEP && p.h != nullptr) mx *= __ldg(p.maxabs + 1);
@@ -116,7 +138,10 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
       mbar_init(full16 + 8u * s, kConvWarps);
       mbar_init(empty16 + 8u * s, 1);
     }
-    mbar_init(done_bar, 1);
+    for (int j = 0; j < 2; ++j) {
+      mbar_init(accfull + 8u * j, 1);
+      mbar_init(accempty + 8u * j, kConvWarps);
+    }
     fence_barrier_init();
   }
   if (warp == kMmaWarp) {
@@ -129,14 +154,67 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(gbase + (tmem_slot - sbase));
 
   bool ok = true;
+  int seg = -1, seg_tile = -1;   // converters: the segment in progress and its tile
+  // converter warps: partials of segment `sg` (tile `ts`) from TMEM buffer sg & 1 into its slot; false after a
+  // timeout
+  const int quad = warp & 3, group = warp >> 2;   // 2 warps per TMEM lane quadrant
+  auto epilogue = [&](int sg, int ts) -> bool {
+    const bool waited = mbar_wait(accfull + 8u * (sg & 1), (uint32_t)(sg / 2) & 1u, p.err);
+    const bool have = __all_sync(0xffffffffu, waited) != 0;
+    tc_fence_after();
+    const int xi = ts * 128 + quad * 32 + lane;
+    const long long tu0 = (long long)ts * p.nkt;
+    int slot, zero_from = p.slots;
+    if (STREAM) {
+      const long long wf = unit_owner(tu0, p.U, gridDim.x);
+      slot = (int)((long long)blockIdx.x - wf);
+      if (u1 >= tu0 + p.nkt) zero_from = (int)(unit_owner(tu0 + p.nkt - 1, p.U, gridDim.x) - wf + 1);
+    } else {
+      slot = (int)blockIdx.z;
+    }
+    float* out = p.part + (long long)slot * p.w * Lx;
+    for (int ch = group; ch < p.wpad / 16; ch += kConvWarps / 4) {
+      uint32_t v[16];
+      if (have) {
+        tmem_ld16(tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)((sg & 1) * p.wpad + ch * 16), v);
+        tmem_wait_ld();
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = 0u;
+      }
+      if (xi < Lx) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int a = ch * 16 + i;
+          if (a < p.w) out[(long long)a * Lx + xi] = __uint_as_float(v[i]) * inv_scale;
+        }
+        for (int z = zero_from; STREAM && z < p.slots; ++z) {   // slots no run fills for this tile
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int a = ch * 16 + i;
+            if (a < p.w) p.part[((long long)z * p.w + a) * Lx + xi] = 0.f;
+          }
+        }
+      }
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(accempty + 8u * (sg & 1));
+    return have;
+  };
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------------ TMA producer
     if (lane == 0) {
       int k = 0, kb = 0;   // stages whose R copies / B copies were issued
+      int t = (int)(u0 / p.nkt), kc = (int)(u0 - (long long)t * p.nkt);   // advanced without divisions
       for (; k < nk; ++k) {
+        if (STREAM && k > 0 && ++kc == p.nkt) {
+          kc = 0;
+          ++t;
+        }
+        const int x0 = t * 128, y0 = (STREAM ? kc : kc + k) * kStageK;   // a classic run stays in its tile
         const int s = k % p.s32, sb = k % p.sb;
         if (k >= p.s32 && !mbar_wait(empty32 + 8u * s, (uint32_t)(k / p.s32 - 1) & 1u, p.err)) break;
-        const int y0 = ybeg + k * kStageK;
         mbar_expect_tx(full32 + 8u * s, kStage32);
         if (!USTEP) {
 #pragma unroll
@@ -161,7 +239,20 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idesc = f16_idesc(128, (uint32_t)p.wpad);
+      int seg = -1;
+      int kc = STREAM ? (int)(u0 % p.nkt) - 1 : 0;
       for (int k = 0; k < nk; ++k) {
+        if (STREAM && ++kc == p.nkt) kc = 0;
+        const bool first = k == 0 || (STREAM && kc == 0);
+        const bool last = k == nk - 1 || (STREAM && kc == p.nkt - 1);
+        if (first) {
+          ++seg;
+          // a run holds at most two segments in flight: the third waits for the first one's partials
+          if (seg >= 2 && !mbar_wait(accempty + 8u * (seg & 1), (uint32_t)(seg / 2 - 1) & 1u, p.err)) {
+            ok = false;
+            break;
+          }
+        }
         const int s = k % p.s16, sb = k % p.sb;
         if (!mbar_wait(full16 + 8u * s, (uint32_t)(k / p.s16) & 1u, p.err) ||
             !mbar_wait(fullB + 8u * sb, (uint32_t)(k / p.sb) & 1u, p.err)) {
@@ -169,22 +260,34 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
           break;
         }
         tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)((seg & 1) * p.wpad);
         const uint32_t a_hi = ra + (uint32_t)s * 2u * kTileA, a_lo = a_hi + kTileA, bt = rb + (uint32_t)sb * tileB;
 #pragma unroll
         for (int kk = 0; kk < kStageK / 16; ++kk) {
           const uint64_t bd = sw128_desc(bt + 32u * kk);
-          mma_f16(tmem, sw128_desc(a_hi + 32u * kk), bd, idesc, (k > 0 || kk > 0) ? 1u : 0u);
-          mma_f16(tmem, sw128_desc(a_lo + 32u * kk), bd, idesc, 1u);
+          mma_f16(d, sw128_desc(a_hi + 32u * kk), bd, idesc, (!first || kk > 0) ? 1u : 0u);
+          mma_f16(d, sw128_desc(a_lo + 32u * kk), bd, idesc, 1u);
         }
         mma_commit(empty16 + 8u * s);
         mma_commit(emptyB + 8u * sb);
+        if (last) mma_commit(accfull + 8u * (seg & 1));
       }
-      mma_commit(done_bar);
     }
   } else {
-    // ------------------------------------------------------------------ converters
+    // ------------------------------------------------------------------ converters (and the epilogues)
     // item i = tid + 256 q (q < 4): A row x = i % 128 (lanes on consecutive rows), K chunk o = i / 128
+    int prev_tile = -1;
+    int t = (int)(u0 / p.nkt), kc = (int)(u0 - (long long)t * p.nkt);   // advanced without divisions
     for (int k = 0; k < nk && ok; ++k) {
+      if (STREAM && k > 0 && ++kc == p.nkt) {
+        kc = 0;
+        ++t;
+      }
+      if (k == 0 || (STREAM && kc == 0)) {
+        ++seg;
+        prev_tile = seg_tile;
+        seg_tile = t;
+      }
       const int s = k % p.s32, s16 = k % p.s16;
       const bool got = mbar_wait(full32 + 8u * s, (uint32_t)(k / p.s32) & 1u, p.err) &&
                        (k < p.s16 || mbar_wait(empty16 + 8u * s16, (uint32_t)(k / p.s16 - 1) & 1u, p.err));
@@ -193,12 +296,12 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
       const uint8_t* st = gbase + (r32 - sbase) + (size_t)s * kStage32;
       uint8_t* a_hi = gbase + (ra - sbase) + (size_t)s16 * 2u * kTileA;
       uint8_t* a_lo = a_hi + kTileA;
-      const int y0 = ybeg + k * kStageK;
+      const int y0 = (STREAM ? kc : kc + k) * kStageK;
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int i = tid + kConv * q;
         const int x = i & 127, o = i >> 7;
-        const int valid = yend - (y0 + 8 * o);   // elements of this chunk inside the split
+        const int valid = Ly - (y0 + 8 * o);   // elements of this chunk inside R
         float v[8];
         if (!USTEP) {
           // R[y0 + 8o + j][x0 + x]: box x / 32, row 8o + j, float x % 32
@@ -235,37 +338,15 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
         mbar_arrive(full16 + 8u * s16);
         mbar_arrive(empty32 + 8u * s);
       }
+      // the previous segment's partials, once this segment is fully converted (its MMAs are then queued)
+      const bool seg_end = k == nk - 1 || kc == p.nkt - 1;
+      if (STREAM && seg_end && seg >= 1) ok = epilogue(seg - 1, prev_tile);
     }
   }
+  // the last segment (or zeros after a failure, so every partial slot is written), once every role is done
+  __syncthreads();
+  if (warp < kConvWarps && nk > 0 && seg >= 0) epilogue(seg, seg_tile);
 
-  // ------------------------------------------------------------------ epilogue (converter warps)
-  const int all_ok = __syncthreads_and(ok ? 1 : 0);
-  if (warp < kConvWarps) {
-    bool have = nk > 0 && all_ok;
-    const bool waited = mbar_wait(done_bar, 0u, p.err);
-    have = __all_sync(0xffffffffu, have && waited);
-    tc_fence_after();
-    const int quad = warp & 3, group = warp >> 2;   // 2 warps per TMEM lane quadrant
-    const int xi = x0 + quad * 32 + lane;
-    float* out = p.part + (long long)blockIdx.z * p.w * Lx;
-    for (int ch = group; ch < p.wpad / 16; ch += kConvWarps / 4) {
-      uint32_t v[16];
-      if (have) {
-        tmem_ld16(tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(ch * 16), v);
-        tmem_wait_ld();
-      } else {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] = 0u;
-      }
-      if (xi < Lx) {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int a = ch * 16 + i;
-          if (a < p.w) out[(long long)a * Lx + xi] = __uint_as_float(v[i]) * inv_scale;
-        }
-      }
-    }
-  }
   tc_fence_before();
   __syncthreads();
   if (warp == kMmaWarp) {
@@ -311,15 +392,46 @@ TmaPlan tma_plan(int w) {
   return t;
 }
 
+// Which plan the TMA product runs (see the header) and its partial slot count.
+struct TmaWork {
+  int stream, nkt, cu, slots, grid_x, grid_z;
+  long long U;
+};
+
+TmaWork tma_work(int w, int Lx, int Ly) {
+  int sms = 152, dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int sp, chunk;
+  tc_split(w, Lx, Ly, &sp, &chunk);
+  const int tiles = (int)cdiv(Lx, 128), nkt = (int)cdiv(Ly, kStageK);
+  TmaWork t{0, nkt, chunk / kStageK, sp, tiles, sp, (long long)tiles * nkt};
+  const long long G = sms - 1;
+  if ((long long)tiles * sp >= sms && G >= 1 && t.U >= G) {
+    int S = 0;
+    for (long long tt = 0; tt < tiles; ++tt) {
+      const long long a = tt * nkt, b = a + nkt - 1;
+      const long long oa = ((a + 1) * G + t.U - 1) / t.U - 1, ob = ((b + 1) * G + t.U - 1) / t.U - 1;
+      S = std::max<int>(S, (int)(ob - oa + 1));
+    }
+    if (S <= sp + 2) {   // only where the extra partial slots stay few
+      t.stream = 1;
+      t.cu = 0;
+      t.slots = S;
+      t.grid_x = (int)G;
+      t.grid_z = 1;
+    }
+  }
+  return t;
+}
+
 template <bool USTEP>
 cudaError_t launch_tma(const float* R, int m, int n, const __half* T, int ldt, int w, const float* h, float* part,
                        int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
   EncodeTiled enc = encoder();
   if (enc == nullptr) return cudaErrorNotSupported;
   const int Lx = USTEP ? m : n, Ly = USTEP ? n : m;
-  int chunk, sp;
-  tc_split(w, Lx, Ly, &sp, &chunk);
-  if (splits != sp) return cudaErrorInvalidValue;
+  const TmaWork wk = tma_work(w, Lx, Ly);
+  if (splits != wk.slots) return cudaErrorInvalidValue;
   const TmaPlan t = tma_plan(w);
   CUtensorMap mapR, mapT;
   {
@@ -344,16 +456,21 @@ cudaError_t launch_tma(const float* R, int m, int n, const __half* T, int ldt, i
   }
   static bool configured[2] = {false, false};
   if (!configured[USTEP]) {
-    cudaError_t e = cudaFuncSetAttribute(product_tma_kernel<USTEP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(product_tma_kernel<USTEP, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          227 * 1024);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(product_tma_kernel<USTEP, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     if (e != cudaSuccess) return e;
     configured[USTEP] = true;
   }
   uint32_t cols = 32;
-  while ((int)cols < t.wpad) cols <<= 1;
-  TmaArgs a{m, n, w, t.wpad, h, part, chunk, maxabs, err, t.s32, t.sb, t.s16, cols};
-  dim3 grid((unsigned)cdiv(Lx, 128), 1, (unsigned)splits);
-  product_tma_kernel<USTEP><<<grid, kThreads, t.smem, s>>>(mapR, mapT, a);
+  while ((int)cols < (wk.stream ? 2 : 1) * t.wpad) cols <<= 1;   // the stream plan alternates two accumulators
+  TmaArgs a{m, n, w, t.wpad, h, part, maxabs, err, t.s32, t.sb, t.s16, cols, wk.nkt, wk.cu, wk.U, wk.slots};
+  dim3 grid((unsigned)wk.grid_x, 1, (unsigned)wk.grid_z);
+  if (wk.stream)
+    product_tma_kernel<USTEP, true><<<grid, kThreads, t.smem, s>>>(mapR, mapT, a);
+  else
+    product_tma_kernel<USTEP, false><<<grid, kThreads, t.smem, s>>>(mapR, mapT, a);
   return cudaGetLastError();
 }
 
@@ -363,6 +480,8 @@ bool tma_product_ok(const float* R, int n, const __half* T, int ldt) {
   return encoder() != nullptr && (n % 4) == 0 && ((uintptr_t)R & 15u) == 0 && ((uintptr_t)T & 15u) == 0 &&
          (ldt % 8) == 0;
 }
+
+int tma_product_slots(int w, int Lx, int Ly) { return tma_work(w, Lx, Ly).slots; }
 
 cudaError_t launch_product_v_tma(const float* R, int m, int n, const __half* Ut, int ldu, int w, float* part,
                                  int splits, const float* maxabs, unsigned* err, cudaStream_t s) {

@@ -25,6 +25,8 @@ SHAPES = [  # (m, n, w): several 64x128 tiles with ragged tails, a GEMV, a tiny 
     (1000, 777, 1),
     (129, 1031, 128),
     (640, 300, 256),
+    (300, 9728, 32),    # V-step grid of 76 tiles x 2 splits = every SM: the stream plan over SMs - 1 CTAs
+    (9728, 300, 32),    # the same for the U-step
 ]
 
 
