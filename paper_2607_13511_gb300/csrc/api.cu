@@ -416,6 +416,15 @@ bool fused_enabled() {
   return enabled;
 }
 
+// The cooperative decorrelation (parallel threshold finalize); EXTERND_COOP=0 keeps the last-CTA finalize.
+bool coop_enabled() {
+  static const bool enabled = [] {
+    const char* e = std::getenv("EXTERND_COOP");
+    return !(e && std::strcmp(e, "0") == 0);
+  }();
+  return enabled;
+}
+
 // Eq. 3 targets of the product partials and Eq. 2 on them: T (and its fp16 / K-major copies, its integer Gram).
 int targets_step(const Bufs& B, const float* Ginv, int w, int splits, int L, const Stats& st, int8_t* T, int ldt,
                  int* gram, __half* T16, long long ldt16, __half* Tk, cudaStream_t s) {
@@ -426,7 +435,7 @@ int targets_step(const Bufs& B, const float* Ginv, int w, int splits, int L, con
     if (used) return EXTERND_OK;
     return cuda_fail(cudaErrorInvalidValue, "launch_decorrelate_apply");
   }
-  KL(kDecor, 1, launch_decorrelate(Ginv, w, B.part, splits, L, B.X, L, st, s));
+  KL(kDecor, 1, launch_decorrelate(Ginv, w, B.part, splits, L, B.X, L, st, s, coop_enabled() ? B.bar : nullptr, B.err));
   KL(kApply, 1, launch_apply(B.X, w, L, L, st.th, T, ldt, gram, s, T16, ldt16, Tk, B.ldk, B.gram));
   return EXTERND_OK;
 }

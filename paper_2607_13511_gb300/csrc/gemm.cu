@@ -148,10 +148,93 @@ int decorrelate_dx(int L, int w) {
   return dx;
 }
 
-template <int DXT>
+// ---- Device-scope grid barriers (cooperative launches) -------------------------------------------------------
+constexpr unsigned long long kGridWaitNs = 2000000000ull;   // 2 s
+
+__device__ __forceinline__ unsigned long long grid_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Grid barrier on ctr (see above); false after a timeout (then err holds 1).
+__device__ __forceinline__ bool grid_barrier(unsigned* ctr, unsigned target, unsigned* err) {
+  __shared__ int s_ok;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
+    int ok = 1;
+    const unsigned long long t0 = grid_ns();
+    for (unsigned it = 0;; ++it) {
+      unsigned v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+      if (v >= target) break;
+      if ((it & 63u) == 63u && grid_ns() - t0 > kGridWaitNs) {
+        atomicOr(err, 1u);
+        ok = 0;
+        break;
+      }
+    }
+    __threadfence();
+    s_ok = ok;
+  }
+  __syncthreads();
+  return s_ok != 0;
+}
+
+// Eq. 2 thresholds of vectors c0, c0 + step, ... < nv from all chunks of the statistics, one CTA per vector at a
+// time: the threads take chunks tid, tid + 256, ... and the CTA combines them in a fixed order.
+__device__ void finalize_range(const Stats& st, int nv, int c0, int step) {
+  __shared__ F2 rs[8];
+  __shared__ u64 rk[8];
+  const int tid = threadIdx.x;
+  for (int a = c0; a < nv; a += step) {
+    F2 sv;
+    u64 key = 0;
+    const uint4* pp = reinterpret_cast<const uint4*>(st.part + (long long)a * st.nchunk);
+    for (int c = tid; c < st.nchunk; c += 256) {
+      const uint4 r = __ldcg(pp + c);
+      F2 t;
+      t.hi = __uint_as_float(r.x);
+      t.lo = __uint_as_float(r.y);
+      sv = f2_add(sv, t);
+      const u64 kk = ((u64)r.w << 32) | r.z;
+      key = kk > key ? kk : key;
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+      sv = f2_add(sv, f2_shfl_xor(sv, o));
+      const u64 t = __shfl_xor_sync(0xffffffffu, key, o);
+      key = t > key ? t : key;
+    }
+    if ((tid & 31) == 0) {
+      rs[tid >> 5] = sv;
+      rk[tid >> 5] = key;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      F2 tot = rs[0];
+      u64 kmax = rk[0];
+      for (int q = 1; q < 8; ++q) {
+        tot = f2_add(tot, rs[q]);
+        kmax = rk[q] > kmax ? rk[q] : kmax;
+      }
+      const float th = __double2float_rd(st.th.tau * (f2_value(tot) / (double)st.th.L));
+      st.th.theta[a] = th;
+      st.th.fallback[a] = !(key_mag(kmax) > th);
+      st.th.arg[a] = key_index(kmax);
+    }
+    __syncthreads();
+  }
+}
+
+// COOP: launched cooperatively; the thresholds are finalized after a grid barrier by every CTA for its share of
+// the vectors (bar: 2 zero words, left zero) instead of by the last CTA for all of them.
+template <int DXT, bool COOP>
 __global__ void __launch_bounds__(256, 2) decorrelate_kernel(const float* __restrict__ Ginv, int w,
                                                           const float* __restrict__ part, int splits, int L,
-                                                          float* __restrict__ X, int ldx, Stats st) {
+                                                          float* __restrict__ X, int ldx, Stats st,
+                                                          unsigned* __restrict__ bar, unsigned* __restrict__ err) {
   constexpr int PX = DXT / 16;
   extern __shared__ __align__(16) float dsm[];
   float* const Ps = dsm;                 // [w][DXT]
@@ -284,21 +367,61 @@ __global__ void __launch_bounds__(256, 2) decorrelate_kernel(const float* __rest
     }
     if (tx == 0 && a < w) put_stat(st, a, blockIdx.x, s, key);
   }
-  stats_done(st, w);
+  if (!COOP) {
+    stats_done(st, w);
+    return;
+  }
+  const unsigned G = gridDim.x * gridDim.y, c = blockIdx.y * gridDim.x + blockIdx.x;
+  if (!grid_barrier(bar, G, err)) return;
+  finalize_range(st, w, (int)c, (int)G);
+  __syncthreads();
+  if (threadIdx.x == 0) {   // exit ticket: the last CTA resets both words
+    unsigned old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(bar + 1) : "memory");
+    if (old == G - 1u) {
+      bar[0] = 0u;
+      bar[1] = 0u;
+    }
+  }
 }
 
 template <int DXT>
 cudaError_t launch_decorrelate_dx(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
-                                  Stats st, cudaStream_t s) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(decorrelate_kernel<DXT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  Stats st, unsigned* bar, unsigned* err, cudaStream_t s) {
+  static int max_coop = -1;
+  if (max_coop < 0) {
+    cudaError_t e = cudaFuncSetAttribute(decorrelate_kernel<DXT, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)decorrelate_smem(kMaxBlock, DXT));
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(decorrelate_kernel<DXT, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)decorrelate_smem(kMaxBlock, DXT));
     if (e != cudaSuccess) return e;
-    configured = true;
+    int per_sm = 0, sms = 0, dev = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decorrelate_kernel<DXT, true>, 256,
+                                                      decorrelate_smem(kMaxBlock, DXT)) == cudaSuccess)
+      max_coop = per_sm * sms;
+    else
+      max_coop = 0;
+    cudaGetLastError();
   }
   dim3 grid((unsigned)cdiv(L, DXT), (unsigned)cdiv(w, TM));
-  decorrelate_kernel<DXT><<<grid, 256, decorrelate_smem(w, DXT), s>>>(Ginv, w, part, splits, L, X, ldx, st);
+  const size_t smem = decorrelate_smem(w, DXT);
+  if (bar != nullptr && err != nullptr && (long long)grid.x * grid.y <= max_coop) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, decorrelate_kernel<DXT, true>, Ginv, w, part, splits, L, X, ldx, st, bar, err);
+  }
+  decorrelate_kernel<DXT, false><<<grid, 256, smem, s>>>(Ginv, w, part, splits, L, X, ldx, st, nullptr, nullptr);
   return cudaGetLastError();
 }
 
@@ -316,40 +439,6 @@ cudaError_t launch_decorrelate_dx(const float* Ginv, int w, const float* part, i
 // of every CTA increments with release semantics and polls with acquire loads, giving up after kWaitNs (error
 // word set, the CTA skips the rest). Counter 0 is reset by CTA 0 after barrier 2 (everyone has left barrier 1),
 // counters 1 and 2 by the last CTA to finish (an exit ticket), so the next launch finds them at zero.
-constexpr unsigned long long kGridWaitNs = 2000000000ull;   // 2 s
-
-__device__ __forceinline__ unsigned long long grid_ns() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
-// Grid barrier on ctr (see above); false after a timeout (then err holds 1).
-__device__ __forceinline__ bool grid_barrier(unsigned* ctr, unsigned target, unsigned* err) {
-  __shared__ int s_ok;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
-    int ok = 1;
-    const unsigned long long t0 = grid_ns();
-    for (unsigned it = 0;; ++it) {
-      unsigned v;
-      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
-      if (v >= target) break;
-      if ((it & 63u) == 63u && grid_ns() - t0 > kGridWaitNs) {
-        atomicOr(err, 1u);
-        ok = 0;
-        break;
-      }
-    }
-    __threadfence();
-    s_ok = ok;
-  }
-  __syncthreads();
-  return s_ok != 0;
-}
-
 template <int DXT>
 __global__ void __launch_bounds__(256, 2) decorrelate_apply_kernel(const float* __restrict__ Ginv, int w,
                                                                 const float* __restrict__ part, int splits, int L,
@@ -479,47 +568,7 @@ __global__ void __launch_bounds__(256, 2) decorrelate_apply_kernel(const float* 
   if (!grid_barrier(bar + 0, G, err)) return;
 
   // ---- thresholds of vectors blockIdx.x, blockIdx.x + G, ...: all chunks, fixed-order CTA reduction
-  {
-    __shared__ F2 rs[8];
-    __shared__ u64 rk[8];
-    for (int a = blockIdx.x; a < w; a += G) {
-      F2 sv;
-      u64 key = 0;
-      const uint4* pp = reinterpret_cast<const uint4*>(st.part + (long long)a * st.nchunk);
-      for (int c = tid; c < st.nchunk; c += 256) {
-        const uint4 r = __ldcg(pp + c);
-        F2 t;
-        t.hi = __uint_as_float(r.x);
-        t.lo = __uint_as_float(r.y);
-        sv = f2_add(sv, t);
-        const u64 kk = ((u64)r.w << 32) | r.z;
-        key = kk > key ? kk : key;
-      }
-      for (int o = 16; o > 0; o >>= 1) {
-        sv = f2_add(sv, f2_shfl_xor(sv, o));
-        const u64 t = __shfl_xor_sync(0xffffffffu, key, o);
-        key = t > key ? t : key;
-      }
-      if ((tid & 31) == 0) {
-        rs[tid >> 5] = sv;
-        rk[tid >> 5] = key;
-      }
-      __syncthreads();
-      if (tid == 0) {
-        F2 tot = rs[0];
-        u64 kmax = rk[0];
-        for (int q = 1; q < 8; ++q) {
-          tot = f2_add(tot, rs[q]);
-          kmax = rk[q] > kmax ? rk[q] : kmax;
-        }
-        const float th = __double2float_rd(st.th.tau * (f2_value(tot) / (double)st.th.L));
-        st.th.theta[a] = th;
-        st.th.fallback[a] = !(key_mag(kmax) > th);
-        st.th.arg[a] = key_index(kmax);
-      }
-      __syncthreads();
-    }
-  }
+  finalize_range(st, w, blockIdx.x, G);
   if (!grid_barrier(bar + 1, G, err)) return;
   if (blockIdx.x == 0 && tid == 0) bar[0] = 0u;   // everyone has left barrier 1
 
@@ -806,12 +855,12 @@ cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int
 int decorrelate_chunks(int L, int w) { return (int)cdiv(L, decorrelate_dx(L, w)); }
 
 cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
-                               Stats st, cudaStream_t s) {
+                               Stats st, cudaStream_t s, unsigned* bar, unsigned* err) {
   switch (decorrelate_dx(L, w)) {
-    case 16: return launch_decorrelate_dx<16>(Ginv, w, part, splits, L, X, ldx, st, s);
-    case 32: return launch_decorrelate_dx<32>(Ginv, w, part, splits, L, X, ldx, st, s);
-    case 64: return launch_decorrelate_dx<64>(Ginv, w, part, splits, L, X, ldx, st, s);
-    default: return launch_decorrelate_dx<128>(Ginv, w, part, splits, L, X, ldx, st, s);
+    case 16: return launch_decorrelate_dx<16>(Ginv, w, part, splits, L, X, ldx, st, bar, err, s);
+    case 32: return launch_decorrelate_dx<32>(Ginv, w, part, splits, L, X, ldx, st, bar, err, s);
+    case 64: return launch_decorrelate_dx<64>(Ginv, w, part, splits, L, X, ldx, st, bar, err, s);
+    default: return launch_decorrelate_dx<128>(Ginv, w, part, splits, L, X, ldx, st, bar, err, s);
   }
 }
 

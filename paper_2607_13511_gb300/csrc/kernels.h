@@ -130,8 +130,10 @@ cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int
 // Statistics chunks the decorrelation writes per vector of length L for a block of w components (at most
 // cdiv(L, 16)).
 int decorrelate_chunks(int L, int w);
+// With bar (2 zero words, left zero) and err given and the grid resident at once, the grid is launched
+// cooperatively and finalizes the thresholds in parallel after a grid barrier (2 s limit, err set on expiry).
 cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
-                               Stats st, cudaStream_t s);
+                               Stats st, cudaStream_t s, unsigned* bar = nullptr, unsigned* err = nullptr);
 // The decorrelation followed by the ternarization of its output (launch_decorrelate + launch_apply, with X kept
 // on chip) in one cooperative grid, for w <= 64 and grids that fit the GPU at once; *used tells whether it ran
 // (if not, nothing was launched and the caller runs the two kernels). T16 / Tk / gram as launch_apply's (gram:
