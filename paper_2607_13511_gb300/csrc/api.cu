@@ -251,6 +251,7 @@ struct Plan {
 struct Bufs {
   float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE, *maxpart, *maxabs, *theta;
   unsigned *err, *arg, *ticket, *bar;
+  unsigned* gop;   // Ginv as the tensor-core decorrelation's shared-memory operand (written by the inverse)
   int *fallback, *GintU, *GintV;
   GramScratch gram;   // per-CTA partials and group tickets of the fused Gram
   int8_t *Ut, *Vt;
@@ -314,6 +315,7 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "GrawU", (size_t)w * w, &B->GrawU));
   TRY(need(ws, "GrawV", (size_t)w * w, &B->GrawV));
   TRY(need(ws, "Ginv", (size_t)w * w, &B->Ginv));
+  TRY(need(ws, "gop", ginv_operand_bytes() / sizeof(unsigned), &B->gop));
   TRY(need(ws, "d", (size_t)w, &B->d));
   TRY(need(ws, "r", (size_t)w, &B->r));
   TRY(need(ws, "J", (size_t)w, &B->J, true));
@@ -435,7 +437,8 @@ int targets_step(const Bufs& B, const float* Ginv, int w, int splits, int L, con
     if (used) return EXTERND_OK;
     return cuda_fail(cudaErrorInvalidValue, "launch_decorrelate_apply");
   }
-  KL(kDecor, 1, launch_decorrelate(Ginv, w, B.part, splits, L, B.X, L, st, s, coop_enabled() ? B.bar : nullptr, B.err));
+  KL(kDecor, 1, launch_decorrelate(Ginv, w, B.part, splits, L, B.X, L, st, s, coop_enabled() ? B.bar : nullptr, B.err,
+                                   B.gop));
   KL(kApply, 1, launch_apply(B.X, w, L, L, st.th, T, ldt, gram, s, T16, ldt16, Tk, B.ldk, B.gram));
   return EXTERND_OK;
 }
@@ -458,6 +461,7 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
   const bool fusedU = w <= 128, fusedV = w <= 128 && h == nullptr;
   __half* const U16 = use_tc(w) ? B.Ut16 : nullptr;
   __half* const V16 = use_tc(w) ? B.Vt16 : nullptr;
+  void* const gop = decorrelate_needs_operand(w) ? B.gop : nullptr;   // Ginv's tensor-core operand
   if (!staged) {
     KL(kStart, 2, launch_select_with(B.colpart, nrt, n, h, w, B.J, B.colE, s));
     KL(kStart, 1, launch_gather(B.R, m, n, B.J, w, B.X, m, q.st_g, s));
@@ -473,10 +477,10 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
     if (w > 1) {
       FORK();
       if (fusedU && !(staged && it == 0)) {
-        KLS(kSolve, 1, side, launch_inverse_int(B.GintU, w, B.GrawU, B.Ginv, side));
+        KLS(kSolve, 1, side, launch_inverse_int(B.GintU, w, B.GrawU, B.Ginv, side, gop));
       } else {
         KLS(kGram, 1, side, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, side));
-        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side));
+        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side, gop));
       }
     }
     KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
@@ -486,10 +490,10 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
     // U-step: U <- T(R H V (V^T H V + eps I)^-1)
     FORK();
     if (fusedV) {
-      KLS(kSolve, 1, side, launch_inverse_int(B.GintV, w, B.GrawV, B.Ginv, side));
+      KLS(kSolve, 1, side, launch_inverse_int(B.GintV, w, B.GrawV, B.Ginv, side, gop));
     } else {
       KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
-      KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side));
+      KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side, gop));
     }
     KL(kUstep, 1, product_u(B.R, m, n, B.Vt, V16, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s));
     JOIN();
@@ -1113,9 +1117,11 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   TRY(get_one(*ws, &one));
   if (vstep) LK(product_v(R, (int)m, (int)n, T, T16, (int)ldt, w, part, splits, mx, err, g_stream));
   else LK(product_u(R, (int)m, (int)n, T, T16, (int)ldt, w, h, part, splits, mx, err, g_stream));
+  unsigned* gop = nullptr;
+  if (decorrelate_needs_operand(w)) TRY(need(*ws, "gop", ginv_operand_bytes() / sizeof(unsigned), &gop));
   if (w > 1) {
     LK(launch_gram(T, (int)ldt, w, (int)Lred, vstep ? nullptr : h, Gpart, gs, g_stream));
-    LK(launch_inverse(Gpart, gs, w, Graw, Ginv, g_stream));
+    LK(launch_inverse(Gpart, gs, w, Graw, Ginv, g_stream, gop));
   }
   float* theta;
   int* fb;
@@ -1126,9 +1132,9 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   TRY(need(*ws, "ticket", 1, &ticket, true));
   Stats st{sp, nchunk, Thresh{theta, fb, arg, ticket, 0.0, (int)L}};
   if (vstep) {
-    LK(launch_decorrelate(w > 1 ? Ginv : one, w, part, splits, (int)L, out, (int)L, st, g_stream));
+    LK(launch_decorrelate(w > 1 ? Ginv : one, w, part, splits, (int)L, out, (int)L, st, g_stream, nullptr, err, gop));
   } else {
-    LK(launch_decorrelate(w > 1 ? Ginv : one, w, part, splits, (int)L, X, (int)L, st, g_stream));
+    LK(launch_decorrelate(w > 1 ? Ginv : one, w, part, splits, (int)L, X, (int)L, st, g_stream, nullptr, err, gop));
     LK(launch_transpose_f32(X, L, w, (int)L, out, w, g_stream));
   }
   return check_device_error(*ws, err, g_stream);

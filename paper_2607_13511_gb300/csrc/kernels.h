@@ -132,8 +132,19 @@ cudaError_t launch_product_u(const float* R, int m, int n, const int8_t* Vt, int
 int decorrelate_chunks(int L, int w);
 // With bar (2 zero words, left zero) and err given and the grid resident at once, the grid is launched
 // cooperatively and finalizes the thresholds in parallel after a grid barrier (2 s limit, err set on expiry).
+// Where decorrelate_needs_operand(w) (blocks of 65 to 128 components, on the tensor cores: decorrelate_tc.cu;
+// EXTERND_TCDECOR=0 keeps the FMA tiles), it reads Ginv from op, written by launch_inverse(_int), and needs err.
 cudaError_t launch_decorrelate(const float* Ginv, int w, const float* part, int splits, int L, float* X, int ldx,
-                               Stats st, cudaStream_t s, unsigned* bar = nullptr, unsigned* err = nullptr);
+                               Stats st, cudaStream_t s, unsigned* bar = nullptr, unsigned* err = nullptr,
+                               const void* op = nullptr);
+bool decorrelate_needs_operand(int w);
+// The tensor-core decorrelation (decorrelate_tc.cu): one statistics chunk per decorrelate_tc_positions(L)
+// positions. Its Ginv operand (ginv_operand_bytes(), 16-byte aligned) is written by launch_inverse(_int).
+bool decorrelate_tc_eligible(int w);
+int decorrelate_tc_positions(int L);
+size_t ginv_operand_bytes();
+cudaError_t launch_decorrelate_tc(const void* op, int w, const float* part, int splits, int L, float* X, int ldx,
+                                  Stats st, cudaStream_t s, unsigned* bar, unsigned* err);
 // The decorrelation followed by the ternarization of its output (launch_decorrelate + launch_apply, with X kept
 // on chip) in one cooperative grid, for w <= 64 and grids that fit the GPU at once; *used tells whether it ran
 // (if not, nothing was launched and the caller runs the two kernels). T16 / Tk / gram as launch_apply's (gram:
@@ -243,10 +254,12 @@ int gram_splits(int w, int L);
 // Gpart[s][a][b] = sum_{y in split s} T[a][y] T[b][y] (* h[y] if h)
 cudaError_t launch_gram(const int8_t* T, int ldt, int w, int L, const float* h, float* Gpart, int splits,
                         cudaStream_t s);
-// Graw = sum_s Gpart[s]; Ginv = (Graw + eps I)^-1 with eps = kEpsRel * trace / w.
-cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s);
+// Graw = sum_s Gpart[s]; Ginv = (Graw + eps I)^-1 with eps = kEpsRel * trace / w. With op (65 to 128
+// components), Ginv also as the tensor-core decorrelation's operand (ginv_operand_bytes(), 16-byte aligned).
+cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s,
+                           void* op = nullptr);
 // Same from an integer upper-triangle Gram (as written by launch_apply), which is reset to zero after reading.
-cudaError_t launch_inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s);
+cudaError_t launch_inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s, void* op = nullptr);
 // r[a] = sum_y Ut[a][y] * sum_s part[s][a][y]
 cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, float* r,
                         cudaStream_t s);

@@ -7,6 +7,7 @@
 // 1024/W_PAD threads, and sweeps the w pivots with one barrier per pivot. Sweeping every pivot of S = G turns S
 // into -G^-1.
 #include "kernels.h"
+#include "umma.cuh"
 
 namespace externd {
 
@@ -382,7 +383,8 @@ __device__ __forceinline__ void warp_sweep(float (&A)[NB * NB / 32], int lane) {
 template <int W_PAD, int NB, int MODE, bool IN_INT>
 __global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ Gpart, int splits, int w,
                                                       const float* __restrict__ GVraw, const float* __restrict__ r,
-                                                      float* __restrict__ Graw, float* __restrict__ out, int* Gint) {
+                                                      float* __restrict__ Graw, float* __restrict__ out, int* Gint,
+                                                      uint8_t* __restrict__ op) {
   constexpr int RPT = W_PAD / 16, CPT = W_PAD / 32, EPL = NB * NB / 32, LPR = NB / EPL, TLD = NB + 4;
   static_assert(W_PAD % NB == 0 && 32 % NB == 0 && (NB * NB) % 32 == 0 && NB % 4 == 0 && RPT >= 1 && CPT >= 1,
                 "bad shape");
@@ -632,6 +634,36 @@ __global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ 
         if (j < w) out[(long long)i * w + j] = -S[a][c];
       }
     }
+    if (W_PAD == 128 && op != nullptr) {
+      // Ginv * 2^sg as hi / lo fp16 K-major operands (zero outside w x w) for the tensor-core decorrelation, with
+      // sg from the largest magnitude; sg (int) follows the two 32 KB images.
+      float mx = 0.f;
+#pragma unroll
+      for (int a = 0; a < RPT; ++a)
+#pragma unroll
+        for (int c = 0; c < CPT; ++c)
+          if (i0 + a < w && tx + 32 * c < w) mx = fmaxf(mx, fabsf(S[a][c]));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      if (lane == 0) red[warp] = mx;
+      asm volatile("bar.sync 1, 512;" ::: "memory");   // the 16 tile warps (the pivot warp has left)
+#pragma unroll
+      for (int q = 0; q < 16; ++q) mx = fmaxf(mx, red[q]);
+      const int sg = fp16_scale_exp(mx);
+      const float sc = ldexpf(1.f, sg);
+#pragma unroll
+      for (int a = 0; a < RPT; ++a)
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) {
+          const int i = i0 + a, j = tx + 32 * c;
+          __half hi, lo;
+          split_f16((i < w && j < w) ? -S[a][c] * sc : 0.f, hi, lo);
+          const uint32_t off = k_major_offset(128u, (uint32_t)i, (uint32_t)j);
+          *reinterpret_cast<__half*>(op + off) = hi;
+          *reinterpret_cast<__half*>(op + 2 * 16384u + off) = lo;
+        }
+      if (tid == 0) *reinterpret_cast<int*>(op + 4 * 16384u) = sg;
+    }
   } else {
 #pragma unroll
     for (int a = 0; a < RPT; ++a) {
@@ -664,7 +696,7 @@ int gram_chunk(int w, int L, int* splits) {
 
 template <int W_PAD, int NB, int MODE>
 cudaError_t launch_sweep_int_w(int* Gint, int w, const float* GVraw, const float* r, float* Graw, float* out,
-                               cudaStream_t s) {
+                               cudaStream_t s, uint8_t* op) {
   const size_t smem = (size_t)W_PAD * (W_PAD + 1) * sizeof(int);   // the staged integer Gram
   static bool configured = false;
   if (!configured) {
@@ -673,27 +705,27 @@ cudaError_t launch_sweep_int_w(int* Gint, int w, const float* GVraw, const float
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  sweep32_kernel<W_PAD, NB, MODE, true><<<1, 544, smem, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint);
+  sweep32_kernel<W_PAD, NB, MODE, true><<<1, 544, smem, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint, op);
   return cudaGetLastError();
 }
 
 template <int MODE>
 cudaError_t launch_sweep_int(int* Gint, int w, const float* GVraw, const float* r, float* Graw, float* out,
-                             cudaStream_t s) {
-  if (w <= 32) return launch_sweep_int_w<32, 8, MODE>(Gint, w, GVraw, r, Graw, out, s);
-  if (w <= 64) return launch_sweep_int_w<64, 16, MODE>(Gint, w, GVraw, r, Graw, out, s);
-  if (w <= 128) return launch_sweep_int_w<128, 16, MODE>(Gint, w, GVraw, r, Graw, out, s);
+                             cudaStream_t s, uint8_t* op = nullptr) {
+  if (w <= 32) return launch_sweep_int_w<32, 8, MODE>(Gint, w, GVraw, r, Graw, out, s, nullptr);
+  if (w <= 64) return launch_sweep_int_w<64, 16, MODE>(Gint, w, GVraw, r, Graw, out, s, nullptr);
+  if (w <= 128) return launch_sweep_int_w<128, 16, MODE>(Gint, w, GVraw, r, Graw, out, s, op);
   return cudaErrorInvalidValue;   // callers use the float-partial Gram above 128 components
 }
 
 template <int MODE>
 cudaError_t launch_sweep(const float* Gpart, int splits, int w, const float* GVraw, const float* r, float* Graw,
-                         float* out, cudaStream_t s) {
+                         float* out, cudaStream_t s, uint8_t* op = nullptr) {
   // elements per lane RPW * CPL = W_PAD^2 / (32 * NWARP): 4 / 8 / 32 / 64
   // pivot-block sizes measured fastest on GB300: 8 up to w = 64, 16 at w = 128
-  if (w <= 32) sweep32_kernel<32, 8, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
-  else if (w <= 64) sweep32_kernel<64, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
-  else if (w <= 128) sweep32_kernel<128, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr);
+  if (w <= 32) sweep32_kernel<32, 8, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
+  else if (w <= 64) sweep32_kernel<64, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
+  else if (w <= 128) sweep32_kernel<128, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, op);
   else sweep_kernel<256, 32, MODE><<<1, 32 * 32, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
   return cudaGetLastError();
 }
@@ -714,12 +746,15 @@ cudaError_t launch_gram(const int8_t* T, int ldt, int w, int L, const float* h, 
   return cudaGetLastError();
 }
 
-cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s) {
-  return launch_sweep<0>(Gpart, splits, w, nullptr, nullptr, Graw, Ginv, s);
+cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s,
+                           void* op) {
+  if (op != nullptr && (w <= 64 || w > 128 || (reinterpret_cast<uintptr_t>(op) & 15) != 0)) return cudaErrorInvalidValue;
+  return launch_sweep<0>(Gpart, splits, w, nullptr, nullptr, Graw, Ginv, s, static_cast<uint8_t*>(op));
 }
 
-cudaError_t launch_inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s) {
-  return launch_sweep_int<0>(Gint, w, nullptr, nullptr, Graw, Ginv, s);
+cudaError_t launch_inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s, void* op) {
+  if (op != nullptr && (w <= 64 || w > 128 || (reinterpret_cast<uintptr_t>(op) & 15) != 0)) return cudaErrorInvalidValue;
+  return launch_sweep_int<0>(Gint, w, nullptr, nullptr, Graw, Ginv, s, static_cast<uint8_t*>(op));
 }
 
 cudaError_t launch_scales_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s,

@@ -57,6 +57,11 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigne
   }
 }
 
+// Arrives once on the mbarrier and adds `bytes` to the transaction count its current phase waits for.
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
 __device__ __forceinline__ void fence_barrier_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
@@ -132,6 +137,21 @@ __device__ __forceinline__ void split_f16(float x, __half& hi, __half& lo) {
 // Byte offset of the 16-byte chunk j (0..7) of row r in a 128-byte-swizzled K-major tile.
 __device__ __forceinline__ uint32_t sw128_offset(uint32_t r, uint32_t j) {
   return (r >> 3) * 1024u + (r & 7u) * 128u + ((j ^ (r & 7u)) << 4);
+}
+
+// Byte offset of element (r, k) in a K-major fp16 operand of `rows` rows stored as 64-wide, 128-byte-swizzled
+// K atoms of rows x 128 B each (atom k / 64, 16-byte chunk (k % 64) / 8 of row r, element k % 8).
+__host__ __device__ __forceinline__ uint32_t k_major_offset(uint32_t rows, uint32_t r, uint32_t k) {
+  return (k >> 6) * rows * 128u + (r >> 3) * 1024u + (r & 7u) * 128u + ((((k & 63u) >> 3) ^ (r & 7u)) << 4) +
+         2u * (k & 7u);
+}
+
+// Power-of-two exponent s for which mx * 2^s lies in [2^13, 2^14): fp16 hi / lo splits of values up to mx then
+// keep their full precision with room for the sums of an MMA. Clamped to [-100, 100]; 14 for mx = 0.
+__device__ __forceinline__ int fp16_scale_exp(float mx) {
+  int ex = 0;
+  if (mx > 0.f && mx <= 3.0e38f) frexpf(mx, &ex);
+  return max(-100, min(100, 14 - ex));
 }
 
 }  // namespace externd
