@@ -252,6 +252,7 @@ struct Bufs {
   float *R, *part, *X, *Gpart, *GrawU, *GrawV, *Ginv, *d, *one, *colpart, *colE, *maxpart, *maxabs, *theta;
   unsigned *err, *arg, *ticket, *bar;
   unsigned* gop;   // Ginv as the tensor-core decorrelation's shared-memory operand (written by the inverse)
+  int8_t* gsc;     // tile Grams of the fused tensor-core decorrelation + ternarization
   int *fallback, *GintU, *GintV;
   GramScratch gram;   // per-CTA partials and group tickets of the fused Gram
   int8_t *Ut, *Vt;
@@ -299,7 +300,7 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "fallback", (size_t)w, &B->fallback));
   TRY(need(ws, "arg", (size_t)w, &B->arg));
   TRY(need(ws, "ticket", 1, &B->ticket, true));
-  TRY(need(ws, "bar", 3, &B->bar, true));
+  TRY(need(ws, "bar", 4, &B->bar, true));
   TRY(need(ws, "GintU", (size_t)w * w, &B->GintU, true));
   TRY(need(ws, "GintV", (size_t)w * w, &B->GintV, true));
   {
@@ -316,6 +317,9 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   TRY(need(ws, "GrawV", (size_t)w * w, &B->GrawV));
   TRY(need(ws, "Ginv", (size_t)w * w, &B->Ginv));
   TRY(need(ws, "gop", ginv_operand_bytes() / sizeof(unsigned), &B->gop));
+  B->gsc = nullptr;
+  if (decorrelate_needs_operand(w))
+    TRY(need(ws, "gsc", std::max(decorrelate_apply_tc_scratch(p.m), decorrelate_apply_tc_scratch(p.n)), &B->gsc));
   TRY(need(ws, "d", (size_t)w, &B->d));
   TRY(need(ws, "r", (size_t)w, &B->r));
   TRY(need(ws, "J", (size_t)w, &B->J, true));
@@ -436,6 +440,11 @@ int targets_step(const Bufs& B, const float* Ginv, int w, int splits, int L, con
                                            B.err, s, &used));
     if (used) return EXTERND_OK;
     return cuda_fail(cudaErrorInvalidValue, "launch_decorrelate_apply");
+  }
+  if (fused_enabled() && decorrelate_needs_operand(w) && decorrelate_apply_tc_fits(w, L)) {
+    KL(kDecor, 1, launch_decorrelate_apply_tc(B.gop, w, B.part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, B.ldk,
+                                              B.gsc, B.bar, B.err, s));
+    return EXTERND_OK;
   }
   KL(kDecor, 1, launch_decorrelate(Ginv, w, B.part, splits, L, B.X, L, st, s, coop_enabled() ? B.bar : nullptr, B.err,
                                    B.gop));

@@ -13,6 +13,8 @@
 // lo.hi; lo.lo is below float32 resolution) accumulate X^T in TMEM, one lane per component; in the epilogue the
 // warp pair (q, q + 4) reads lane quadrant q, each warp half of the positions, and writes X and the Eq. 2
 // statistics of its half, which the pair then combines into the CTA's chunk.
+#include <algorithm>
+
 #include "grid.cuh"
 #include "kernels.h"
 #include "umma.cuh"
@@ -61,15 +63,37 @@ __device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&v)[8]) {
                : "r"(taddr));
 }
 
-// COOP: thresholds finalized after a grid barrier by every CTA (bar: 2 zero words, left zero), as in the FMA
-// decorrelation; otherwise by the last CTA.
-template <int NPOS, bool COOP>
+// Outputs of the fused ternarization (MODE 2), as launch_apply's: T (int8, rows of ldt), its fp16 copy T16 (rows
+// of ldt16; may be null), the K-major fp16 copy Tk (rows of ldk per position; may be null) and the exact Gram
+// upper triangle gram[a * w + b], a <= b, added to (may be null).
+struct ApplyOut {
+  int8_t* T;
+  long long ldt;
+  __half* T16;
+  long long ldt16;
+  __half* Tk;
+  long long ldk;
+  int* gram;
+  int8_t* gsc;   // with gram: the grid's tile Grams, gridDim.x x 128 x 128 int8 (counts of at most 64 trits)
+};
+
+// MODE 0: X and the statistics; the last CTA finalizes the thresholds.
+// MODE 1 (cooperative; bar: 2 zero words, left zero): every CTA finalizes its share of the thresholds after a
+//   grid barrier, as in the FMA decorrelation.
+// MODE 2 (cooperative; bar: 4 zero words, left zero): no X; after a second grid barrier every CTA ternarizes its
+//   tile from TMEM (Eq. 2 with the finalized thresholds) and writes the factor layouts of `out`. With out.gram,
+//   the tile's Gram T T^T is one more MMA (M = N = 128, K = NPOS) on the fp16 trits in shared memory, stored to
+//   out.gsc as int8 (|count| <= NPOS); after a third barrier the warps of the grid sum the tiles' Grams, one warp
+//   per 16 entries of the upper triangle (8 lane groups over the tiles, 4 entries per lane, then shuffles), and
+//   add them to out.gram. Integer sums: the order does not matter.
+template <int NPOS, int MODE>
 __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* __restrict__ op, int w,
                                                                 const float* __restrict__ part, int splits, int L,
                                                                 float* __restrict__ X, int ldx, Stats st,
                                                                 unsigned* __restrict__ bar,
-                                                                unsigned* __restrict__ err) {
+                                                                unsigned* __restrict__ err, ApplyOut out) {
   using C = TcDecor<NPOS>;
+  constexpr uint32_t kCols = MODE == 2 ? 256u : C::kTmemCols;   // MODE 2: the tile's Gram at column 128
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t sbase = (raw + 1023u) & ~1023u;
@@ -95,7 +119,7 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
     for (uint32_t c = 0; c < kOpBytes / kOpCopy; ++c) bulk_copy(a_hi + c * kOpCopy, op + c * kOpCopy, kOpCopy, smem_addr(&op_bar));
   }
   if (warp == 0) {
-    tmem_alloc(smem_addr(&tmem_slot), C::kTmemCols);
+    tmem_alloc(smem_addr(&tmem_slot), kCols);
     tmem_relinquish();
   }
   const int sg = __ldg(reinterpret_cast<const int*>(op + kOpBytes));
@@ -191,11 +215,12 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
   // ---- epilogue: warp q reads lane quadrant q % 4, positions (q / 4) NPOS / 2 .. + NPOS / 2 - 1
   const int quad = warp & 3, hpos = warp >> 2;
   const int a = 32 * quad + lane;
+  const float ig = ldexpf(1.f, -sg), ip = ldexpf(1.f, -sp);
+  const uint32_t trow = tmem + ((uint32_t)(32 * quad) << 16);   // this warp's lane quadrant
   {
     const bool ok = mbar_wait(smem_addr(&done_bar), 0u, err);
     const bool have = __all_sync(0xffffffffu, ok) != 0;
     tc_fence_after();
-    const float ig = ldexpf(1.f, -sg), ip = ldexpf(1.f, -sp);
     AbsSum sum;
     u64 key = 0;
 #pragma unroll
@@ -203,7 +228,7 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
       const int col = hpos * (NPOS / 2) + 8 * ch;
       uint32_t d[8];
       if (have) {
-        tmem_ld8(tmem + ((uint32_t)(32 * quad) << 16) + (uint32_t)col, d);
+        tmem_ld8(trow + (uint32_t)col, d);
         tmem_wait_ld();
       } else {
 #pragma unroll
@@ -215,7 +240,8 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
         for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(d[i]) * ig * ip;
         const int xb = x0 + col;
         float* dst = X + (long long)a * ldx + xb;
-        if (xb + 7 < L && (ldx & 3) == 0) {
+        if (MODE == 2) {
+        } else if (xb + 7 < L && (ldx & 3) == 0) {
           *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
           *reinterpret_cast<float4*>(dst + 4) = make_float4(v[4], v[5], v[6], v[7]);
         } else {
@@ -245,49 +271,239 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
       put_stat(st, a, blockIdx.x, s2, k2);
     }
   }
-  if (warp == 0) {
+  if (MODE != 2 && warp == 0) {
     tc_fence_after();
-    tmem_dealloc(tmem, C::kTmemCols);
+    tmem_dealloc(tmem, kCols);
   }
-  if (!COOP) {
+  if (MODE == 0) {
     stats_done(st, w);
     return;
   }
   const unsigned G = gridDim.x;
-  if (!grid_barrier(bar, G, err)) return;
-  finalize_range(st, w, (int)blockIdx.x, (int)G);
+  if (MODE == 1) {
+    if (!grid_barrier(bar, G, err)) return;
+    finalize_range(st, w, (int)blockIdx.x, (int)G);
+    __syncthreads();
+    if (threadIdx.x == 0) {   // exit ticket: the last CTA resets both words
+      unsigned old;
+      asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(bar + 1) : "memory");
+      if (old == G - 1u) {
+        bar[0] = 0u;
+        bar[1] = 0u;
+      }
+    }
+    return;
+  }
+  // ---- MODE 2: thresholds of vectors blockIdx.x, blockIdx.x + G, ..., then every CTA ternarizes its tile
+  bool ok = grid_barrier(bar + 0, G, err);
+  if (ok) {
+    finalize_range(st, w, (int)blockIdx.x, (int)G);
+    ok = grid_barrier(bar + 1, G, err);
+  }
+  if (ok) {
+    if (blockIdx.x == 0 && tid == 0) bar[0] = 0u;   // everyone has left barrier 1
+    tc_fence_after();
+    const float thv = a < w ? __ldcg(st.th.theta + a) : 0.f;
+    const int fbv = a < w ? __ldcg(st.th.fallback + a) : 0;
+    const unsigned argv = a < w ? __ldcg(st.th.arg + a) : 0u;
+    uint8_t* const ts = gbase;   // the tile's trits as a K-major fp16 operand (rows a): the free A region
+#pragma unroll
+    for (int ch = 0; ch < NPOS / 16; ++ch) {
+      const int col = hpos * (NPOS / 2) + 8 * ch, xb = x0 + col;
+      uint32_t d[8];
+      tmem_ld8(trow + (uint32_t)col, d);
+      tmem_wait_ld();
+      short t[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float v = __uint_as_float(d[i]) * ig * ip;   // as in the statistics above
+        int8_t tt = 0;
+        if (a < w && xb + i < L) {
+          tt = ternary_of(v, thv);
+          if (fbv && (uint32_t)(xb + i) == argv) tt = v < 0.f ? (int8_t)-1 : (int8_t)1;
+        }
+        t[i] = tt;
+      }
+      uint32_t h[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        h[e] = (uint32_t)__half_as_ushort(__short2half_rn(t[2 * e])) |
+               ((uint32_t)__half_as_ushort(__short2half_rn(t[2 * e + 1])) << 16);
+      if (a < w) {
+        int8_t* Tr = out.T + (long long)a * out.ldt + xb;
+        __half* Hr = out.T16 != nullptr ? out.T16 + (long long)a * out.ldt16 + xb : nullptr;
+        if (xb + 7 < L) {
+          uint32_t b0 = 0u, b1 = 0u;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            b0 |= (uint32_t)(uint8_t)t[i] << (8 * i);
+            b1 |= (uint32_t)(uint8_t)t[4 + i] << (8 * i);
+          }
+          *reinterpret_cast<uint2*>(Tr) = make_uint2(b0, b1);
+          if (Hr != nullptr) *reinterpret_cast<uint4*>(Hr) = make_uint4(h[0], h[1], h[2], h[3]);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (xb + i < L) {
+              Tr[i] = (int8_t)t[i];
+              if (Hr != nullptr) Hr[i] = __short2half_rn(t[i]);
+            }
+        }
+      }
+      // position rows of the K-major copy (the warp's 32 components are 64 contiguous bytes), with zeros up to the
+      // next multiple of 8 components
+      if (out.Tk != nullptr && a < ((w + 7) & ~7) && a < out.ldk) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          if (xb + i < L) out.Tk[(long long)(xb + i) * out.ldk + a] = __short2half_rn(t[i]);
+      }
+      if (out.gram != nullptr)
+        *reinterpret_cast<uint4*>(ts + k_major_offset(128u, (uint32_t)a, (uint32_t)col)) =
+            make_uint4(h[0], h[1], h[2], h[3]);
+    }
+    if (out.gram != nullptr) {
+      fence_async_shared();
+      tc_fence_before();
+      __syncthreads();
+      tc_fence_after();
+      if (tid == 0) {
+        const uint32_t idesc = f16_idesc((uint32_t)kWp, (uint32_t)kWp);
+#pragma unroll
+        for (int kk = 0; kk < NPOS / 16; ++kk) {
+          const uint64_t dsc = sw128_desc(sbase + 32u * (uint32_t)kk);
+          mma_f16(tmem + 128u, dsc, dsc, idesc, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(smem_addr(&done_bar));
+      }
+      __syncwarp();
+      const bool gok = mbar_wait(smem_addr(&done_bar), 1u, err);
+      const bool have = __all_sync(0xffffffffu, gok) != 0;
+      tc_fence_after();
+      if (have) {   // row a, columns 64 hpos .. + 63 of the tile's Gram (the loads are warp-collective)
+        int8_t* dst = out.gsc + ((long long)blockIdx.x * kWp + a) * kWp + 64 * hpos;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t g[16];
+          tmem_ld16(trow + 128u + (uint32_t)(64 * hpos + 16 * c), g);
+          tmem_wait_ld();
+          uint32_t pk[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            pk[e] = 0u;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) pk[e] |= ((uint32_t)(int)__uint_as_float(g[4 * e + i]) & 0xffu) << (8 * i);
+          }
+          if (a < w) *reinterpret_cast<uint4*>(dst + 16 * c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        }
+      }
+      ok = grid_barrier(bar + 2, G, err);
+      if (ok) {
+        if (blockIdx.x == 0 && tid == 0) bar[1] = 0u;   // everyone has left barrier 2
+        // tasks: (row a, 16 columns from 16 u) for u = a / 16 .. cdiv(w, 16) - 1, rows in order; lane (q, j)
+        // sums entries (a, 16 u + 4 j .. + 3) of the tiles q, q + 8, ...
+        const int ng = (w + 15) >> 4, w16 = w >> 4, q = lane >> 2, j = lane & 3;
+        const int ntask = ng * w - 16 * (w16 * (w16 - 1) / 2) - (w & 15) * w16;
+        for (int task = (int)blockIdx.x * 8 + warp; task < ntask; task += (int)G * 8) {
+          int ra = 0, t = task;
+          for (; ra < w; ++ra) {
+            const int n = ng - (ra >> 4);
+            if (t < n) break;
+            t -= n;
+          }
+          const int b0 = 16 * ((ra >> 4) + t) + 4 * j;
+          const int8_t* src = out.gsc + (long long)ra * kWp + b0;
+          int acc[4] = {0, 0, 0, 0};
+          for (int c0 = q; c0 < (int)G; c0 += 8 * 24) {
+            unsigned v[24];
+#pragma unroll
+            for (int k = 0; k < 24; ++k) {
+              const int c = c0 + 8 * k;
+              v[k] = c < (int)G ? __ldcg(reinterpret_cast<const unsigned*>(src + (long long)c * kWp * kWp)) : 0u;
+            }
+#pragma unroll
+            for (int k = 0; k < 24; ++k)
+#pragma unroll
+              for (int i = 0; i < 4; ++i) acc[i] += (int)(int8_t)(v[k] >> (8 * i));
+          }
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], 4);
+            acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], 8);
+            acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], 16);
+          }
+          if (q == 0) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int b = b0 + i;
+              if (b >= ra && b < w && acc[i] != 0) atomicAdd(out.gram + (long long)ra * w + b, acc[i]);
+            }
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
   __syncthreads();
-  if (threadIdx.x == 0) {   // exit ticket: the last CTA resets both words
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kCols);
+  }
+  if (!ok) return;
+  if (tid == 0) {   // exit ticket: the last CTA resets the words still set (barrier 2 without a Gram)
     unsigned old;
-    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(bar + 1) : "memory");
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(bar + 3) : "memory");
     if (old == G - 1u) {
-      bar[0] = 0u;
       bar[1] = 0u;
+      bar[2] = 0u;
+      bar[3] = 0u;
     }
   }
 }
 
-// Sets the kernels' shared-memory limit (once) and returns how many CTAs of the cooperative variant the GPU holds
-// at once (0 if the query failed).
+// Sets the kernels' shared-memory limit (once) and returns how many CTAs of the cooperative variants the GPU
+// holds at once (0 if the query failed).
 template <int NPOS>
 long long coop_capacity() {
   static long long cap = -1;
   if (cap < 0) {
     using C = TcDecor<NPOS>;
     cap = 0;
-    int per_sm = 0, sms = 0, dev = 0;
-    if (cudaFuncSetAttribute(decorrelate_tc_kernel<NPOS, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)C::kSmem) == cudaSuccess &&
-        cudaFuncSetAttribute(decorrelate_tc_kernel<NPOS, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)C::kSmem) == cudaSuccess &&
+    int p1 = 0, p2 = 0, sms = 0, dev = 0;
+    const int sm = (int)C::kSmem;
+    if (cudaFuncSetAttribute(decorrelate_tc_kernel<NPOS, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm) ==
+            cudaSuccess &&
+        cudaFuncSetAttribute(decorrelate_tc_kernel<NPOS, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm) ==
+            cudaSuccess &&
+        cudaFuncSetAttribute(decorrelate_tc_kernel<NPOS, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm) ==
+            cudaSuccess &&
         cudaGetDevice(&dev) == cudaSuccess &&
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decorrelate_tc_kernel<NPOS, true>, 256, C::kSmem) ==
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p1, decorrelate_tc_kernel<NPOS, 1>, 256, C::kSmem) ==
+            cudaSuccess &&
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p2, decorrelate_tc_kernel<NPOS, 2>, 256, C::kSmem) ==
             cudaSuccess)
-      cap = (long long)per_sm * sms;
+      cap = (long long)std::min(p1, p2) * sms;
     cudaGetLastError();
   }
   return cap;
+}
+
+template <int NPOS, int MODE>
+cudaError_t launch_coop(const uint8_t* op, int w, const float* part, int splits, int L, float* X, int ldx, Stats st,
+                        cudaStream_t s, unsigned* bar, unsigned* err, const ApplyOut& out) {
+  using C = TcDecor<NPOS>;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)cdiv(L, NPOS));
+  cfg.blockDim = dim3(256);
+  cfg.dynamicSmemBytes = C::kSmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decorrelate_tc_kernel<NPOS, MODE>, op, w, part, splits, L, X, ldx, st, bar, err,
+                            out);
 }
 
 template <int NPOS>
@@ -295,22 +511,12 @@ cudaError_t launch_npos(const uint8_t* op, int w, const float* part, int splits,
                         cudaStream_t s, unsigned* bar, unsigned* err) {
   using C = TcDecor<NPOS>;
   const long long grid = cdiv(L, NPOS);
-  if (bar != nullptr && grid <= coop_capacity<NPOS>()) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)grid);
-    cfg.blockDim = dim3(256);
-    cfg.dynamicSmemBytes = C::kSmem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeCooperative;
-    attr[0].val.cooperative = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, decorrelate_tc_kernel<NPOS, true>, op, w, part, splits, L, X, ldx, st, bar, err);
-  }
+  const ApplyOut none{};
+  if (bar != nullptr && grid <= coop_capacity<NPOS>())
+    return launch_coop<NPOS, 1>(op, w, part, splits, L, X, ldx, st, s, bar, err, none);
   coop_capacity<NPOS>();   // the shared-memory limit
-  decorrelate_tc_kernel<NPOS, false><<<(unsigned)grid, 256, C::kSmem, s>>>(op, w, part, splits, L, X, ldx, st,
-                                                                           nullptr, err);
+  decorrelate_tc_kernel<NPOS, 0><<<(unsigned)grid, 256, C::kSmem, s>>>(op, w, part, splits, L, X, ldx, st, nullptr,
+                                                                       err, none);
   return cudaGetLastError();
 }
 
@@ -326,6 +532,37 @@ int decorrelate_tc_positions(int L) {
   if (cdiv(L, 16) <= coop_capacity<16>()) return 16;
   if (cdiv(L, 32) <= coop_capacity<32>()) return 32;
   return 64;
+}
+
+bool decorrelate_apply_tc_fits(int w, int L) {
+  if (!decorrelate_tc_eligible(w)) return false;
+  switch (decorrelate_tc_positions(L)) {
+    case 16: return cdiv(L, 16) <= coop_capacity<16>();
+    case 32: return cdiv(L, 32) <= coop_capacity<32>();
+    default: return cdiv(L, 64) <= coop_capacity<64>();
+  }
+}
+
+size_t decorrelate_apply_tc_scratch(int L) { return (size_t)cdiv(L, decorrelate_tc_positions(L)) * kWp * kWp; }
+
+cudaError_t launch_decorrelate_apply_tc(const void* op, int w, const float* part, int splits, int L, Stats st,
+                                        int8_t* T, long long ldt, int* gram, __half* T16, long long ldt16, __half* Tk,
+                                        long long ldk, int8_t* gsc, unsigned* bar, unsigned* err, cudaStream_t s) {
+  const int npos = decorrelate_tc_positions(L);
+  if (!decorrelate_apply_tc_fits(w, L) || st.nchunk != (int)cdiv(L, npos) || op == nullptr || err == nullptr ||
+      (gram != nullptr && (gsc == nullptr || (reinterpret_cast<uintptr_t>(gsc) & 15) != 0)) ||
+      bar == nullptr || T == nullptr || (reinterpret_cast<uintptr_t>(op) & 15) != 0 || (ldt & 7) != 0 ||
+      (reinterpret_cast<uintptr_t>(T) & 7) != 0 ||
+      (T16 != nullptr && ((ldt16 & 7) != 0 || (reinterpret_cast<uintptr_t>(T16) & 15) != 0)) ||
+      (Tk != nullptr && ldk < w))
+    return cudaErrorInvalidValue;
+  const uint8_t* o = static_cast<const uint8_t*>(op);
+  const ApplyOut out{T, ldt, T16, ldt16, Tk, ldk, gram, gsc};
+  switch (npos) {
+    case 16: return launch_coop<16, 2>(o, w, part, splits, L, nullptr, 0, st, s, bar, err, out);
+    case 32: return launch_coop<32, 2>(o, w, part, splits, L, nullptr, 0, st, s, bar, err, out);
+    default: return launch_coop<64, 2>(o, w, part, splits, L, nullptr, 0, st, s, bar, err, out);
+  }
 }
 
 cudaError_t launch_decorrelate_tc(const void* op, int w, const float* part, int splits, int L, float* X, int ldx,

@@ -145,6 +145,15 @@ int decorrelate_tc_positions(int L);
 size_t ginv_operand_bytes();
 cudaError_t launch_decorrelate_tc(const void* op, int w, const float* part, int splits, int L, float* X, int ldx,
                                   Stats st, cudaStream_t s, unsigned* bar, unsigned* err);
+// The tensor-core decorrelation followed by the ternarization of its output in one cooperative grid (the X tile
+// stays in tensor memory; the tile's Gram is one more MMA), where decorrelate_apply_tc_fits(w, L). Arguments as
+// launch_decorrelate_apply's, with op as launch_decorrelate's; with gram, gsc is scratch of
+// decorrelate_apply_tc_scratch(L) bytes (16-byte aligned); bar: 4 zero words, left zero.
+bool decorrelate_apply_tc_fits(int w, int L);
+size_t decorrelate_apply_tc_scratch(int L);
+cudaError_t launch_decorrelate_apply_tc(const void* op, int w, const float* part, int splits, int L, Stats st,
+                                        int8_t* T, long long ldt, int* gram, __half* T16, long long ldt16, __half* Tk,
+                                        long long ldk, int8_t* gsc, unsigned* bar, unsigned* err, cudaStream_t s);
 // The decorrelation followed by the ternarization of its output (launch_decorrelate + launch_apply, with X kept
 // on chip) in one cooperative grid, for w <= 64 and grids that fit the GPU at once; *used tells whether it ran
 // (if not, nothing was launched and the caller runs the two kernels). T16 / Tk / gram as launch_apply's (gram:
