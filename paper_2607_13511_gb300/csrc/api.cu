@@ -434,17 +434,17 @@ bool coop_enabled() {
 // Eq. 3 targets of the product partials and Eq. 2 on them: T (and its fp16 / K-major copies, its integer Gram).
 int targets_step(const Bufs& B, const float* Ginv, int w, int splits, int L, const Stats& st, int8_t* T, int ldt,
                  int* gram, __half* T16, long long ldt16, __half* Tk, cudaStream_t s) {
-  if (fused_enabled() && decorrelate_apply_fits(w, L)) {
+  if (fused_enabled() && decorrelate_needs_operand(w) && decorrelate_apply_tc_fits(w, L)) {
+    KL(kDecor, 1, launch_decorrelate_apply_tc(B.gop, w, B.part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, B.ldk,
+                                              B.gsc, B.bar, B.err, s));
+    return EXTERND_OK;
+  }
+  if (fused_enabled() && !decorrelate_needs_operand(w) && decorrelate_apply_fits(w, L)) {
     bool used = false;
     KL(kDecor, 1, launch_decorrelate_apply(Ginv, w, B.part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, B.ldk, B.bar,
                                            B.err, s, &used));
     if (used) return EXTERND_OK;
     return cuda_fail(cudaErrorInvalidValue, "launch_decorrelate_apply");
-  }
-  if (fused_enabled() && decorrelate_needs_operand(w) && decorrelate_apply_tc_fits(w, L)) {
-    KL(kDecor, 1, launch_decorrelate_apply_tc(B.gop, w, B.part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, B.ldk,
-                                              B.gsc, B.bar, B.err, s));
-    return EXTERND_OK;
   }
   KL(kDecor, 1, launch_decorrelate(Ginv, w, B.part, splits, L, B.X, L, st, s, coop_enabled() ? B.bar : nullptr, B.err,
                                    B.gop));

@@ -24,6 +24,7 @@ namespace externd {
 namespace {
 
 constexpr int kWp = 128;                                    // components, padded (MMA M, and K)
+constexpr int kTcMinBlock = 64;   // narrower blocks keep the FMA kernels (faster there: fused targets at 2048^2)
 constexpr uint32_t kAtomA = (uint32_t)kWp * 128u;           // one 64-wide K atom of A: 128 rows x 128 B
 constexpr uint32_t kOpBytes = 4 * kAtomA;                   // A image: hi atoms 0, 1 then lo atoms 0, 1 (64 KB)
 constexpr uint32_t kOpCopy = 16384;                         // bytes per bulk copy
@@ -522,7 +523,7 @@ cudaError_t launch_npos(const uint8_t* op, int w, const float* part, int splits,
 
 }  // namespace
 
-bool decorrelate_tc_eligible(int w) { return w > 64 && w <= kWp; }
+bool decorrelate_tc_eligible(int w) { return w > kTcMinBlock && w <= kWp; }
 
 size_t ginv_operand_bytes() { return (size_t)kOpBytes + 16; }
 
