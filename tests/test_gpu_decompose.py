@@ -59,6 +59,9 @@ CASES = [  # m, n, mu, tau, block, iters, kind, weighted
     (7, 5, 3.0, 0.7, 16, 4, "gaussian", False),         # min < 8: cap 0, sequential
     (1, 9, 2.0, 0.7, 1, 4, "gaussian", False),          # a single row
     (520, 64, 2.0, 0.7, 8, 4, "student_t", True),
+    (640, 768, 1.2, 0.7, 80, 3, "student_t", False),   # tensor-core targets (w = 80), tail 48
+    (576, 700, 1.1, 0.7, 72, 3, "gaussian", True),     # tensor-core targets weighted (w = 72), tail 57
+    (1000, 1100, 0.3, 0.7, 128, 2, "gaussian", False), # block capped to 125, tail 50
 ]
 
 
