@@ -576,15 +576,30 @@ __global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ 
         for (int q = 0; q < 4; ++q)
 #pragma unroll
           for (int c = 0; c < CPT; ++c) rv[q][c] = Rk[cur][b + q][tx + 32 * c];
+        if constexpr (CPT % 2 == 0) {   // column pairs on the paired FMA (each lane the same fmaf as below)
 #pragma unroll
-        for (int a = 0; a < RPT; ++a)
+          for (int a = 0; a < RPT; ++a)
 #pragma unroll
-          for (int c = 0; c < CPT; ++c) {
-            S[a][c] = fmaf(-tv[a].x, rv[0][c], S[a][c]);
-            S[a][c] = fmaf(-tv[a].y, rv[1][c], S[a][c]);
-            S[a][c] = fmaf(-tv[a].z, rv[2][c], S[a][c]);
-            S[a][c] = fmaf(-tv[a].w, rv[3][c], S[a][c]);
-          }
+            for (int c = 0; c < CPT; c += 2) {
+              float2 s2 = make_float2(S[a][c], S[a][c + 1]);
+              s2 = __ffma2_rn(make_float2(-tv[a].x, -tv[a].x), make_float2(rv[0][c], rv[0][c + 1]), s2);
+              s2 = __ffma2_rn(make_float2(-tv[a].y, -tv[a].y), make_float2(rv[1][c], rv[1][c + 1]), s2);
+              s2 = __ffma2_rn(make_float2(-tv[a].z, -tv[a].z), make_float2(rv[2][c], rv[2][c + 1]), s2);
+              s2 = __ffma2_rn(make_float2(-tv[a].w, -tv[a].w), make_float2(rv[3][c], rv[3][c + 1]), s2);
+              S[a][c] = s2.x;
+              S[a][c + 1] = s2.y;
+            }
+        } else {
+#pragma unroll
+          for (int a = 0; a < RPT; ++a)
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) {
+              S[a][c] = fmaf(-tv[a].x, rv[0][c], S[a][c]);
+              S[a][c] = fmaf(-tv[a].y, rv[1][c], S[a][c]);
+              S[a][c] = fmaf(-tv[a].z, rv[2][c], S[a][c]);
+              S[a][c] = fmaf(-tv[a].w, rv[3][c], S[a][c]);
+            }
+        }
       }
       const int cK = k0 >> 5;
       const int jk = tx + 32 * cK - k0;   // this lane's column within K, when in [0, NB)
