@@ -431,14 +431,22 @@ bool coop_enabled() {
   return enabled;
 }
 
+// Whether targets_step takes the fused tensor-core grid (65 to 128 components, co-resident).
+bool fused_targets_tc(int w, int L) {
+  return fused_enabled() && decorrelate_needs_operand(w) && decorrelate_apply_tc_fits(w, L);
+}
+
 // Eq. 3 targets of the product partials and Eq. 2 on them: T (and its fp16 / K-major copies, its integer Gram).
+// With hw and gramf (the fused tensor-core path only: fused_targets_tc), the weighted Gram T H T^T goes to gramf.
 int targets_step(const Bufs& B, const float* Ginv, int w, int splits, int L, const Stats& st, int8_t* T, int ldt,
-                 int* gram, __half* T16, long long ldt16, __half* Tk, cudaStream_t s) {
-  if (fused_enabled() && decorrelate_needs_operand(w) && decorrelate_apply_tc_fits(w, L)) {
+                 int* gram, __half* T16, long long ldt16, __half* Tk, cudaStream_t s, const float* hw = nullptr,
+                 float* gramf = nullptr) {
+  if (fused_targets_tc(w, L)) {
     KL(kDecor, 1, launch_decorrelate_apply_tc(B.gop, w, B.part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, B.ldk,
-                                              B.gsc, B.bar, B.err, s));
+                                              B.gsc, B.bar, B.err, s, hw, gramf));
     return EXTERND_OK;
   }
+  if (gramf != nullptr) return cuda_fail(cudaErrorInvalidValue, "targets_step");
   if (fused_enabled() && !decorrelate_needs_operand(w) && decorrelate_apply_fits(w, L)) {
     bool used = false;
     KL(kDecor, 1, launch_decorrelate_apply(Ginv, w, B.part, splits, L, st, T, ldt, gram, T16, ldt16, Tk, B.ldk, B.bar,
@@ -468,6 +476,8 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
   // Exact Gram matrices of unweighted ternary factors are accumulated by the apply that writes the factor
   // (integer atomics) up to 128 components; wider blocks and the weighted V^T H V use the Gram kernel.
   const bool fusedU = w <= 128, fusedV = w <= 128 && h == nullptr;
+  // weighted V^T H V from the fused tensor-core targets of the V-step (into Gpart, one slice)
+  const bool fusedVw = h != nullptr && w > 1 && fused_targets_tc(w, n);
   __half* const U16 = use_tc(w) ? B.Ut16 : nullptr;
   __half* const V16 = use_tc(w) ? B.Vt16 : nullptr;
   void* const gop = decorrelate_needs_operand(w) ? B.gop : nullptr;   // Ginv's tensor-core operand
@@ -495,11 +505,14 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
     KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
     if (w > 1) JOIN();
     TRY(targets_step(B, w > 1 ? B.Ginv : B.one, w, sv, n, q.st_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, V16,
-                     p.ldn, (last && use_tc(w)) ? B.Vk16 : nullptr, s));
+                     p.ldn, (last && use_tc(w)) ? B.Vk16 : nullptr, s, fusedVw ? h : nullptr,
+                     fusedVw ? B.Gpart : nullptr));
     // U-step: U <- T(R H V (V^T H V + eps I)^-1)
     FORK();
     if (fusedV) {
       KLS(kSolve, 1, side, launch_inverse_int(B.GintV, w, B.GrawV, B.Ginv, side, gop));
+    } else if (fusedVw) {
+      KLS(kSolve, 1, side, launch_inverse(B.Gpart, 1, w, B.GrawV, B.Ginv, side, gop));
     } else {
       KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
       KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side, gop));

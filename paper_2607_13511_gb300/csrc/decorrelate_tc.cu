@@ -75,7 +75,9 @@ struct ApplyOut {
   __half* Tk;
   long long ldk;
   int* gram;
-  int8_t* gsc;   // with gram: the grid's tile Grams, gridDim.x x 128 x 128 int8 (counts of at most 64 trits)
+  int8_t* gsc;         // with a Gram: the grid's tile Grams, gridDim.x x 128 x 128 (int8 counts, or float32)
+  const float* h;      // weighted Gram T H T^T (per-position weights) into gramf instead of gram
+  float* gramf;        // w x w float32, both triangles, written (not added to)
 };
 
 // MODE 0: X and the statistics; the last CTA finalizes the thresholds.
@@ -86,7 +88,9 @@ struct ApplyOut {
 //   the tile's Gram T T^T is one more MMA (M = N = 128, K = NPOS) on the fp16 trits in shared memory, stored to
 //   out.gsc as int8 (|count| <= NPOS); after a third barrier the warps of the grid sum the tiles' Grams, one warp
 //   per 16 entries of the upper triangle (8 lane groups over the tiles, 4 entries per lane, then shuffles), and
-//   add them to out.gram. Integer sums: the order does not matter.
+//   add them to out.gram. Integer sums: the order does not matter. With out.h (the weighted V^T H V of §2.5) the
+//   B operand is t_b(x) h(x) as a scaled fp16 hi + lo pair (two MMAs per K step), the tile Grams are float32 and
+//   the sums, in a fixed order, are written to both triangles of out.gramf.
 template <int NPOS, int MODE>
 __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* __restrict__ op, int w,
                                                                 const float* __restrict__ part, int splits, int L,
@@ -308,6 +312,23 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
     const int fbv = a < w ? __ldcg(st.th.fallback + a) : 0;
     const unsigned argv = a < w ? __ldcg(st.th.arg + a) : 0u;
     uint8_t* const ts = gbase;   // the tile's trits as a K-major fp16 operand (rows a): the free A region
+    uint8_t* const th_hi = gbase + 16384u;   // weighted: t h 2^sh as fp16 hi / lo, the same layout
+    uint8_t* const th_lo = gbase + 32768u;
+    const bool wgram = out.h != nullptr, anyg = wgram || out.gram != nullptr;
+    int sh = 0;
+    if (wgram) {   // 2^sh from the tile's largest weight
+      float hm = 0.f;
+      if (tid < NPOS && x0 + tid < L) hm = fabsf(__ldg(out.h + x0 + tid));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) hm = fmaxf(hm, __shfl_xor_sync(0xffffffffu, hm, o));
+      if (lane == 0) red[warp] = hm;
+      __syncthreads();
+      hm = red[0];
+#pragma unroll
+      for (int q = 1; q < 8; ++q) hm = fmaxf(hm, red[q]);
+      sh = fp16_scale_exp(hm);
+    }
+    const float sch = ldexpf(1.f, sh);
 #pragma unroll
     for (int ch = 0; ch < NPOS / 16; ++ch) {
       const int col = hpos * (NPOS / 2) + 8 * ch, xb = x0 + col;
@@ -358,11 +379,21 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
         for (int i = 0; i < 8; ++i)
           if (xb + i < L) out.Tk[(long long)(xb + i) * out.ldk + a] = __short2half_rn(t[i]);
       }
-      if (out.gram != nullptr)
+      if (anyg)
         *reinterpret_cast<uint4*>(ts + k_major_offset(128u, (uint32_t)a, (uint32_t)col)) =
             make_uint4(h[0], h[1], h[2], h[3]);
+      if (wgram) {
+        float v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = xb + i < L ? (float)t[i] * __ldg(out.h + xb + i) : 0.f;
+        uint32_t hh[4], hl[4];
+        split_pack<8>(v, sch, hh, hl);
+        const uint32_t off = k_major_offset(128u, (uint32_t)a, (uint32_t)col);
+        *reinterpret_cast<uint4*>(th_hi + off) = make_uint4(hh[0], hh[1], hh[2], hh[3]);
+        *reinterpret_cast<uint4*>(th_lo + off) = make_uint4(hl[0], hl[1], hl[2], hl[3]);
+      }
     }
-    if (out.gram != nullptr) {
+    if (anyg) {
       fence_async_shared();
       tc_fence_before();
       __syncthreads();
@@ -372,7 +403,12 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
 #pragma unroll
         for (int kk = 0; kk < NPOS / 16; ++kk) {
           const uint64_t dsc = sw128_desc(sbase + 32u * (uint32_t)kk);
-          mma_f16(tmem + 128u, dsc, dsc, idesc, kk > 0 ? 1u : 0u);
+          if (wgram) {
+            mma_f16(tmem + 128u, dsc, sw128_desc(sbase + 16384u + 32u * (uint32_t)kk), idesc, kk > 0 ? 1u : 0u);
+            mma_f16(tmem + 128u, dsc, sw128_desc(sbase + 32768u + 32u * (uint32_t)kk), idesc, 1u);
+          } else {
+            mma_f16(tmem + 128u, dsc, dsc, idesc, kk > 0 ? 1u : 0u);
+          }
         }
         mma_commit(smem_addr(&done_bar));
       }
@@ -380,7 +416,23 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
       const bool gok = mbar_wait(smem_addr(&done_bar), 1u, err);
       const bool have = __all_sync(0xffffffffu, gok) != 0;
       tc_fence_after();
-      if (have) {   // row a, columns 64 hpos .. + 63 of the tile's Gram (the loads are warp-collective)
+      if (have && wgram) {   // row a, columns 64 hpos .. + 63, unscaled, as float32
+        float* dst = reinterpret_cast<float*>(out.gsc) + ((long long)blockIdx.x * kWp + a) * kWp + 64 * hpos;
+        const float ih = ldexpf(1.f, -sh);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t g[16];
+          tmem_ld16(trow + 128u + (uint32_t)(64 * hpos + 16 * c), g);
+          tmem_wait_ld();
+          if (a < w) {
+#pragma unroll
+            for (int i = 0; i < 16; i += 4)
+              *reinterpret_cast<float4*>(dst + 16 * c + i) =
+                  make_float4(__uint_as_float(g[i]) * ih, __uint_as_float(g[i + 1]) * ih,
+                              __uint_as_float(g[i + 2]) * ih, __uint_as_float(g[i + 3]) * ih);
+          }
+        }
+      } else if (have) {   // row a, columns 64 hpos .. + 63 of the tile's Gram (the loads are warp-collective)
         int8_t* dst = out.gsc + ((long long)blockIdx.x * kWp + a) * kWp + 64 * hpos;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
@@ -412,6 +464,43 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
             t -= n;
           }
           const int b0 = 16 * ((ra >> 4) + t) + 4 * j;
+          if (wgram) {   // float32 tiles, 12 loads of 16 bytes in flight per lane
+            const float* srcf = reinterpret_cast<const float*>(out.gsc) + (long long)ra * kWp + b0;
+            float facc[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int c0 = q; c0 < (int)G; c0 += 8 * 12) {
+              float4 v[12];
+#pragma unroll
+              for (int k = 0; k < 12; ++k) {
+                const int c = c0 + 8 * k;
+                v[k] = c < (int)G ? __ldcg(reinterpret_cast<const float4*>(srcf + (long long)c * kWp * kWp))
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+              }
+#pragma unroll
+              for (int k = 0; k < 12; ++k) {
+                facc[0] += v[k].x;
+                facc[1] += v[k].y;
+                facc[2] += v[k].z;
+                facc[3] += v[k].w;
+              }
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              facc[i] += __shfl_xor_sync(0xffffffffu, facc[i], 4);
+              facc[i] += __shfl_xor_sync(0xffffffffu, facc[i], 8);
+              facc[i] += __shfl_xor_sync(0xffffffffu, facc[i], 16);
+            }
+            if (q == 0) {
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const int b = b0 + i;
+                if (b >= ra && b < w) {
+                  out.gramf[(long long)ra * w + b] = facc[i];
+                  out.gramf[(long long)b * w + ra] = facc[i];
+                }
+              }
+            }
+            continue;
+          }
           const int8_t* src = out.gsc + (long long)ra * kWp + b0;
           int acc[4] = {0, 0, 0, 0};
           for (int c0 = q; c0 < (int)G; c0 += 8 * 24) {
@@ -544,12 +633,17 @@ bool decorrelate_apply_tc_fits(int w, int L) {
   }
 }
 
-size_t decorrelate_apply_tc_scratch(int L) { return (size_t)cdiv(L, decorrelate_tc_positions(L)) * kWp * kWp; }
+size_t decorrelate_apply_tc_scratch(int L) {
+  return (size_t)cdiv(L, decorrelate_tc_positions(L)) * kWp * kWp * sizeof(float);
+}
 
 cudaError_t launch_decorrelate_apply_tc(const void* op, int w, const float* part, int splits, int L, Stats st,
                                         int8_t* T, long long ldt, int* gram, __half* T16, long long ldt16, __half* Tk,
-                                        long long ldk, int8_t* gsc, unsigned* bar, unsigned* err, cudaStream_t s) {
+                                        long long ldk, int8_t* gsc, unsigned* bar, unsigned* err, cudaStream_t s,
+                                        const float* h, float* gramf) {
   const int npos = decorrelate_tc_positions(L);
+  if ((h == nullptr) != (gramf == nullptr) || (h != nullptr && (gram != nullptr || gsc == nullptr)))
+    return cudaErrorInvalidValue;
   if (!decorrelate_apply_tc_fits(w, L) || st.nchunk != (int)cdiv(L, npos) || op == nullptr || err == nullptr ||
       (gram != nullptr && (gsc == nullptr || (reinterpret_cast<uintptr_t>(gsc) & 15) != 0)) ||
       bar == nullptr || T == nullptr || (reinterpret_cast<uintptr_t>(op) & 15) != 0 || (ldt & 7) != 0 ||
@@ -558,7 +652,7 @@ cudaError_t launch_decorrelate_apply_tc(const void* op, int w, const float* part
       (Tk != nullptr && ldk < w))
     return cudaErrorInvalidValue;
   const uint8_t* o = static_cast<const uint8_t*>(op);
-  const ApplyOut out{T, ldt, T16, ldt16, Tk, ldk, gram, gsc};
+  const ApplyOut out{T, ldt, T16, ldt16, Tk, ldk, gram, gsc, h, gramf};
   switch (npos) {
     case 16: return launch_coop<16, 2>(o, w, part, splits, L, nullptr, 0, st, s, bar, err, out);
     case 32: return launch_coop<32, 2>(o, w, part, splits, L, nullptr, 0, st, s, bar, err, out);

@@ -147,13 +147,15 @@ cudaError_t launch_decorrelate_tc(const void* op, int w, const float* part, int 
                                   Stats st, cudaStream_t s, unsigned* bar, unsigned* err);
 // The tensor-core decorrelation followed by the ternarization of its output in one cooperative grid (the X tile
 // stays in tensor memory; the tile's Gram is one more MMA), where decorrelate_apply_tc_fits(w, L). Arguments as
-// launch_decorrelate_apply's, with op as launch_decorrelate's; with gram, gsc is scratch of
-// decorrelate_apply_tc_scratch(L) bytes (16-byte aligned); bar: 4 zero words, left zero.
+// launch_decorrelate_apply's, with op as launch_decorrelate's; with a Gram, gsc is scratch of
+// decorrelate_apply_tc_scratch(L) bytes (16-byte aligned); bar: 4 zero words, left zero. With h (weights of the
+// L positions; gram must be null) the weighted Gram T H T^T is written to both triangles of gramf (w x w float32).
 bool decorrelate_apply_tc_fits(int w, int L);
 size_t decorrelate_apply_tc_scratch(int L);
 cudaError_t launch_decorrelate_apply_tc(const void* op, int w, const float* part, int splits, int L, Stats st,
                                         int8_t* T, long long ldt, int* gram, __half* T16, long long ldt16, __half* Tk,
-                                        long long ldk, int8_t* gsc, unsigned* bar, unsigned* err, cudaStream_t s);
+                                        long long ldk, int8_t* gsc, unsigned* bar, unsigned* err, cudaStream_t s,
+                                        const float* h = nullptr, float* gramf = nullptr);
 // The decorrelation followed by the ternarization of its output (launch_decorrelate + launch_apply, with X kept
 // on chip) in one cooperative grid, for w <= 64 and grids that fit the GPU at once; *used tells whether it ran
 // (if not, nothing was launched and the caller runs the two kernels). T16 / Tk / gram as launch_apply's (gram:
