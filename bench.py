@@ -27,6 +27,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -143,7 +144,8 @@ class ClockSampler:
 
     def __init__(self, device_index):
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{env_int('RANK', 0)}.csv")
+        out_dir = os.environ.get("EXTERND_CLOCKS_DIR", tempfile.gettempdir())   # where the raw samples go
+        self.path = os.path.join(out_dir, f"clocks_rank{env_int('RANK', 0)}.csv")
         self.idx = device_index
 
     def __enter__(self):

@@ -12,7 +12,7 @@ CPU-baseline leg of ``bench.py`` may import it; the product path never does, and
   than the fitted component.
 * Refinement sweeps (§2.4): revisit each block, add it back, refit, deflate again.
 
-Readings taken where the paper is silent (listed in the design doc):
+Readings taken where the paper is silent:
 
 * Safeguard with importance weights: the single-entry pair u = e_i, v = sgn(R_ij) e_j removes h_j R_ij^2 from
   the weighted residual, so the best pair is the argmax of h_j R_ij^2 (ties to the lowest row, then column).

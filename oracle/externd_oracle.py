@@ -8,7 +8,7 @@ Every function follows the ExTernD paper (arxiv 2607.13511, "Expanded-Rank Terna
 the section or equation it restates. Everything is computed in float64 with numpy; a numpy library primitive
 (matmul, solve, sort) serves as a single step, with no blocking or reordering beyond what the paper states.
 
-Readings taken where the paper is silent (each is listed in the design doc):
+Readings taken where the paper is silent:
 
 * Ridge in Eq. 3: ``eps = EPS_REL * trace(G) / w`` (relative, so scaling the importances does not change the
   factors). Eq. 4 gets the same relative ridge when the block has ``w > 1`` components; a 1x1 system is

@@ -1,7 +1,7 @@
 """Per-kernel parity: each step of the CUDA path, called through the C ABI, against the CPU oracle on the same
 seeded inputs.
 
-Bars (derived in the design doc):
+Bars (derived from the arithmetic of each step):
 * Eq. 2 ternarization: bit-exact (both sides decide |x| > tau * mean|x| for the same float32 x).
 * Residual products U^T R and R H V: ||dP||_F / ||P||_F <= 1e-5 and |dP_ij| <= 1e-5 * (|U|^T |R|)_ij elementwise.
 * Decorrelated targets (Eq. 3) and scales (Eq. 4): relative Frobenius error <= 2e-5 + 4 kappa 2^-24, kappa the
