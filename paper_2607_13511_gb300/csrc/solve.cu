@@ -568,28 +568,30 @@ __global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ 
           for (int c = 0; c < CPT; ++c) S[a][c] = 0.f;
 #pragma unroll
       for (int b = 0; b < NB; b += 4) {
-        float4 tv[RPT];
         float rv[4][CPT];
-#pragma unroll
-        for (int a = 0; a < RPT; ++a) tv[a] = *reinterpret_cast<const float4*>(&T[i0 + a][b]);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
 #pragma unroll
           for (int c = 0; c < CPT; ++c) rv[q][c] = Rk[cur][b + q][tx + 32 * c];
         if constexpr (CPT % 2 == 0) {   // column pairs on the paired FMA (each lane the same fmaf as below)
 #pragma unroll
-          for (int a = 0; a < RPT; ++a)
+          for (int a = 0; a < RPT; ++a) {   // one row's T' at a time (a broadcast load): fewer live registers
+            const float4 t = *reinterpret_cast<const float4*>(&T[i0 + a][b]);
 #pragma unroll
             for (int c = 0; c < CPT; c += 2) {
               float2 s2 = make_float2(S[a][c], S[a][c + 1]);
-              s2 = __ffma2_rn(make_float2(-tv[a].x, -tv[a].x), make_float2(rv[0][c], rv[0][c + 1]), s2);
-              s2 = __ffma2_rn(make_float2(-tv[a].y, -tv[a].y), make_float2(rv[1][c], rv[1][c + 1]), s2);
-              s2 = __ffma2_rn(make_float2(-tv[a].z, -tv[a].z), make_float2(rv[2][c], rv[2][c + 1]), s2);
-              s2 = __ffma2_rn(make_float2(-tv[a].w, -tv[a].w), make_float2(rv[3][c], rv[3][c + 1]), s2);
+              s2 = __ffma2_rn(make_float2(-t.x, -t.x), make_float2(rv[0][c], rv[0][c + 1]), s2);
+              s2 = __ffma2_rn(make_float2(-t.y, -t.y), make_float2(rv[1][c], rv[1][c + 1]), s2);
+              s2 = __ffma2_rn(make_float2(-t.z, -t.z), make_float2(rv[2][c], rv[2][c + 1]), s2);
+              s2 = __ffma2_rn(make_float2(-t.w, -t.w), make_float2(rv[3][c], rv[3][c + 1]), s2);
               S[a][c] = s2.x;
               S[a][c + 1] = s2.y;
             }
+          }
         } else {
+          float4 tv[RPT];
+#pragma unroll
+          for (int a = 0; a < RPT; ++a) tv[a] = *reinterpret_cast<const float4*>(&T[i0 + a][b]);
 #pragma unroll
           for (int a = 0; a < RPT; ++a)
 #pragma unroll
