@@ -9,10 +9,10 @@
 // B[x][b] = P * 2^sp (N = NPOS positions), the powers of two putting each operand's largest magnitude just under
 // 2^14 (Ginv's over the whole matrix, P's over the CTA's tile). The Gram inverse writes A (on the side branch,
 // beside the product) as the exact shared-memory image, which every CTA fetches with bulk copies while its
-// threads sum the P slots. Three MMAs per 16-deep K step (hi.hi, hi.lo,
-// lo.hi; lo.lo is below float32 resolution) accumulate X^T in TMEM, one lane per component; in the epilogue the
-// warp pair (q, q + 4) reads lane quadrant q, each warp half of the positions, and writes X and the Eq. 2
-// statistics of its half, which the pair then combines into the CTA's chunk.
+// threads sum the P slots. Three MMAs per 16-deep K step (hi.hi, hi.lo, lo.hi; lo.lo is below float32
+// resolution) accumulate X^T in TMEM, one lane per component; in the epilogue the warp pair (q, q + 4) reads
+// lane quadrant q, each warp half of the positions, and writes X and the Eq. 2 statistics of its half, which the
+// pair then combines into the CTA's chunk.
 #include <algorithm>
 
 #include "grid.cuh"
