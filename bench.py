@@ -207,6 +207,22 @@ def algorithmic_bytes(kind, wl):
     raise ValueError(kind)
 
 
+def max_over_ranks(value, device, world):
+    """The largest of the ranks' values, returned on every rank (value itself for one rank)."""
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(world, units_per_rank, ms):
+    """Whole-job throughput: every rank's units over the slowest rank's time (weak scaling, replicas)."""
+    return world * units_per_rank / (ms / 1e3)
+
+
 def source_sha(path):
     return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
 
@@ -258,12 +274,8 @@ def run_gpu(args):
             res = step()
         ev1.record(stream)
         barrier()
-    ms = ev0.elapsed_time(ev1)
-    t = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_max = float(t.item())
-    value = world * k * args.steps / (ms_max / 1e3)
+    ms_max = max_over_ranks(ev0.elapsed_time(ev1), dev, world)
+    value = job_rate(world, k * args.steps, ms_max)
     energy = res.energy
 
     # ---- end to end through the host entry point: H2D of A (and h), decomposition, D2H of B, D, C, energies
@@ -282,10 +294,7 @@ def run_gpu(args):
         X.decompose_host(A_pin, wl.mu, wl.tau, wl.block, wl.iters, h_pin, out=hout)
     e1.record(stream)
     barrier()
-    t = torch.tensor([e0.elapsed_time(e1)], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    e2e_value = world * k * args.steps / (float(t.item()) / 1e3)
+    e2e_value = job_rate(world, k * args.steps, max_over_ranks(e0.elapsed_time(e1), dev, world))
     nblocks = -(-k // block_width(wl))
     h2d = 4 * wl.m * wl.n + (4 * wl.n if wl.weighted else 0)
     d2h = wl.m * k + k * wl.n + 4 * k + 8 * nblocks
