@@ -1,21 +1,24 @@
 #!/usr/bin/env python3
 """Throughput of the GB300 ExTernD library: ternary components fitted per second.
 
-One step is one complete decomposition of one synthetic matrix (every block, every ALS iteration, the joint
-scales and the deflation), by default the 2048 x 2048 N(0, 0.02^2) matrix with 0.1 % outliers x20, mu = 3
-(k = 6144 components), tau = 0.7, block 64, 4 ALS iterations. The matrix is generated once, resident in HBM;
-its 16.8 MB residual fits in L2, so L2 is flushed (a 512 MB write) before every step, inside the timed region.
+One step is one complete decomposition (every block, every ALS iteration, the joint scales and the deflation) of
+the workload's matrices. The default workload is the largest single matrix of the benchmark set, the 2560 x 9728
+Student-t (nu = 5) MLP up-projection, mu = 3 (k = 7680 components), tau = 1.0, block 128, 4 ALS iterations; its
+99.6 MB residual is below the 129 MB L2, so L2 is flushed (a 512 MB write) before every step, inside the timed
+region. ``--workload decoder36`` runs the whole 36-layer 4B-class decoder conversion (252 matrices, q/k/v/o/gate/
+up/down) back to back on one GPU as one step.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference] [--workload NAME]
 
-With N > 1 (torchrun, one rank per GPU) every rank decomposes its own matrix (independent problems, no
-collective on the data path): value = all ranks' components / the slowest rank's time ("scaling": "weak").
+With N > 1 (torchrun, one rank per GPU) every rank decomposes its own copy of the workload (independent problems,
+no collective on the data path): value = all ranks' components / the slowest rank's time ("scaling": "weak").
 ``--impl reference`` times the CPU oracle (the plain fp64 restatement of the method) on a bounded sample of the
 same workload: the first blocks of the same matrix, which by the greedy prefix property are the same work.
 
-``--row safeguard|refine|packed`` measures an extension instead (one GPU, its own JSON line): the decomposition
-with Prop. 2's safeguard, one refinement sweep (§2.4) of the workload's decomposition, or the packed inference
-product y = B diag(D) (C x) (§2.6) on factors of the workload's shape.
+``--row safeguard|refine|packed|sequential`` measures an extension instead (one GPU, its own JSON line): the
+decomposition with Prop. 2's safeguard, one refinement sweep (§2.4) of the workload's decomposition, the packed
+inference product y = B diag(D) (C x) (§2.6) on factors of the workload's shape, or the sequential algorithm
+(§2.3, block width 1) beside the block algorithm on the same matrix.
 """
 from __future__ import annotations
 
@@ -37,13 +40,16 @@ from paper_2607_13511_gb300 import workloads as W  # noqa: E402
 
 METRIC = "ternary components fitted/sec per matrix"
 UNIT = "components/s"
-DEFAULT_WORKLOAD = W.OUTLIER_2048.name
-ROOFLINE_KIND = "vstep"   # the largest HBM stream of the path: the V-step residual product (profiles/)
+DEFAULT_WORKLOAD = W.MLP_UP_2560x9728.name
+ROOFLINE_KIND = "products"   # the largest HBM streams of the path: both residual products (profiles/)
+
+# A job is the list of matrices one step decomposes: each single-matrix workload, or the 36-layer conversion.
+JOBS = {name: [wl] for name, wl in W.WORKLOADS.items()}
+JOBS["decoder36"] = list(W.decoder_conversion())
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch of the profiled kernel, from one ncu capture, valid
 # only while the kernel's source is unchanged (sha256 of the file that holds it).
-NCU_TRAFFIC: dict = {"kind": "vstep", "file": "product_tma.cu", "sha": "1f7f86b6f6599f85", "workload": "outlier2048_mu3_b64",
-               "bytes_per_launch": 17081600}
+NCU_TRAFFIC: dict = {}
 
 
 def env_int(name, default):
@@ -70,7 +76,8 @@ def golden_energy(name):
 
 
 def workload(name) -> W.Workload:
-    return W.WORKLOADS[name]
+    """The first (for single-matrix workloads, the only) matrix of a job."""
+    return JOBS[name][0]
 
 
 def block_width(wl):
@@ -79,6 +86,25 @@ def block_width(wl):
 
 def inner_rank(wl, mu=None):
     return int(math.floor((wl.mu if mu is None else mu) * min(wl.m, wl.n) + 0.5))
+
+
+def job_components(wls):
+    return sum(inner_rank(wl) for wl in wls)
+
+
+def _matrix(wl):
+    return wl.matrix()
+
+
+def job_matrices(wls):
+    """The job's matrices on the host, generated in a spawned process pool when there are many."""
+    if len(wls) <= 4:
+        return [wl.matrix() for wl in wls]
+    import concurrent.futures
+    import multiprocessing
+    ctx = multiprocessing.get_context("spawn")
+    with concurrent.futures.ProcessPoolExecutor(max_workers=min(16, os.cpu_count() or 1), mp_context=ctx) as pool:
+        return list(pool.map(_matrix, wls, chunksize=1))
 
 
 # ----------------------------------------------------------------------------------------------- CPU oracle
@@ -104,11 +130,17 @@ def cpu_cores():
     return os.cpu_count()
 
 
+def sample_workload(name):
+    """The matrix a bounded CPU sample of the job runs on: for the decoder, its largest projection (gate)."""
+    wls = JOBS[name]
+    return max(wls, key=lambda wl: wl.m * wl.n * inner_rank(wl)) if len(wls) > 1 else wls[0]
+
+
 def run_reference(args):
     rank = env_int("RANK", 0)
     if rank != 0:
         return
-    wl = workload(args.workload)
+    wl = sample_workload(args.workload)
     blocks = args.reference_blocks
     for _ in range(args.warmup):
         oracle_sample(wl, blocks)
@@ -123,17 +155,29 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": config_of(wl),
+        "config": config_of(args.workload),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
 
 
-def config_of(wl):
-    return {"workload": wl.name, "m": wl.m, "n": wl.n, "mu": wl.mu, "k": inner_rank(wl), "tau": wl.tau,
-            "block": block_width(wl), "iters": wl.iters, "weighted": wl.weighted, "matrix": wl.kind,
-            "seed": wl.seed, "l2": "flushed before every step (512 MB write, inside the timed region)"}
+def config_of(name):
+    wls = JOBS[name]
+    l2 = "flushed before every step (512 MB write, inside the timed region)"
+    if len(wls) == 1:
+        wl = wls[0]
+        return {"workload": wl.name, "m": wl.m, "n": wl.n, "mu": wl.mu, "k": inner_rank(wl), "tau": wl.tau,
+                "block": block_width(wl), "iters": wl.iters, "weighted": wl.weighted, "matrix": wl.kind,
+                "seed": wl.seed, "l2": l2}
+    shapes = {}
+    for wl in wls:
+        shapes.setdefault(wl.name.split(".", 1)[1], [wl.m, wl.n, inner_rank(wl)])
+    first = wls[0]
+    return {"workload": name, "matrices": len(wls), "layers": len({wl.name.split(".")[0] for wl in wls}),
+            "shapes_m_n_k": shapes, "k_total": job_components(wls), "mu": first.mu, "tau": first.tau,
+            "block": first.block, "iters": first.iters, "weighted": False, "matrix": first.kind,
+            "seed": "1000 + 10 * layer + projection index", "l2": l2 + "; 14.5 GB of inputs per step"}
 
 
 # ----------------------------------------------------------------------------------------------- clocks
@@ -202,9 +246,18 @@ def algorithmic_bytes(kind, wl):
         return 4 * m * n + m * b + 4 * b * n
     if kind == "ustep":      # read R, V (and h), write R H V
         return 4 * m * n + n * b + hbytes + 4 * m * b
+    if kind == "products":   # V-steps and U-steps launch equally often
+        return (algorithmic_bytes("vstep", wl) + algorithmic_bytes("ustep", wl)) / 2
     if kind == "deflate":    # read and write R, read U, V, d
         return 8 * m * n + (m + n) * b + 4 * b + hbytes
     raise ValueError(kind)
+
+
+def decomposition_bytes(wl):
+    """Least HBM traffic of one whole decomposition: per block 2 * iters passes over R plus the read-modify-write
+    of the deflation, plus the initial copy R = A (read A, write R)."""
+    nblocks = -(-inner_rank(wl) // block_width(wl))
+    return nblocks * (2 * wl.iters * 4 + 8) * wl.m * wl.n + 8 * wl.m * wl.n
 
 
 def max_over_ranks(value, device, world):
@@ -231,97 +284,112 @@ def run_gpu(args):
     import torch
     import torch.distributed as dist
 
+    rank, world, local = env_int("RANK", 0), env_int("WORLD_SIZE", 1), env_int("LOCAL_RANK", 0)
+    wls = JOBS[args.workload]
+    host_A = job_matrices(wls)          # before the first CUDA call (the pool is spawned, not forked)
+
     import paper_2607_13511_gb300 as X
 
-    rank, world, local = env_int("RANK", 0), env_int("WORLD_SIZE", 1), env_int("LOCAL_RANK", 0)
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
     X.load()
 
-    wl = workload(args.workload)
-    A_host = torch.from_numpy(wl.matrix())
-    h_np = wl.weights()
-    A = A_host.to(dev)
-    h = None if h_np is None else torch.from_numpy(h_np).to(dev)
-    k = X.rank(wl.m, wl.n, wl.mu)
-    out = (torch.empty((wl.m, k), dtype=torch.int8, device=dev), torch.empty((k,), dtype=torch.float32, device=dev),
-           torch.empty((k, wl.n), dtype=torch.int8, device=dev))
+    host_A = [torch.from_numpy(a) for a in host_A]
+    host_h = [None if wl.weights() is None else torch.from_numpy(wl.weights()) for wl in wls]
+    As = [a.to(dev) for a in host_A]
+    hs = [None if h is None else h.to(dev) for h in host_h]
+    ks = [X.rank(wl.m, wl.n, wl.mu) for wl in wls]
+    outs = [(torch.empty((wl.m, k), dtype=torch.int8, device=dev), torch.empty((k,), dtype=torch.float32, device=dev),
+             torch.empty((k, wl.n), dtype=torch.int8, device=dev)) for wl, k in zip(wls, ks)]
     flush = torch.empty(128 * 1024 * 1024, dtype=torch.float32, device=dev)   # 512 MB > L2
+    comps = sum(ks)
 
     def step():
-        return X.decompose(A, wl.mu, wl.tau, wl.block, wl.iters, h, out=out)
+        energies, launches = [], 0
+        for i, wl in enumerate(wls):
+            energies.append(X.decompose(As[i], wl.mu, wl.tau, wl.block, wl.iters, hs[i], out=outs[i]).energy)
+            launches += X.kernel_launches()
+        return energies, launches
 
     for _ in range(args.warmup):
         flush.fill_(0.0)
-        res = step()
-    launches_per_step = X.kernel_launches()
+        step()
 
     def barrier():
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
 
-    # ---- timed region: K decompositions, device-timed with CUDA events on the current stream
+    # ---- timed region: K steps, device-timed with CUDA events on the current stream
     stream = torch.cuda.current_stream(dev)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches = 0
     with ClockSampler(local) as clocks:
         barrier()
         ev0.record(stream)
         for i in range(args.steps):
             flush.fill_(float(i))
-            res = step()
+            energies, nl = step()
+            launches += nl
         ev1.record(stream)
         barrier()
     ms_max = max_over_ranks(ev0.elapsed_time(ev1), dev, world)
-    value = job_rate(world, k * args.steps, ms_max)
-    energy = res.energy
+    value = job_rate(world, comps * args.steps, ms_max)
 
-    # ---- end to end through the host entry point: H2D of A (and h), decomposition, D2H of B, D, C, energies
-    A_pin = A_host.pin_memory()
-    h_pin = None if h_np is None else torch.from_numpy(h_np).pin_memory()
-    hout = (torch.empty((wl.m, k), dtype=torch.int8, pin_memory=True),
-            torch.empty((k,), dtype=torch.float32, pin_memory=True),
-            torch.empty((k, wl.n), dtype=torch.int8, pin_memory=True))
+    # ---- end to end through the host entry point: H2D of A (and h), decomposition, D2H of B, D, C, energy
+    A_pin = [a.pin_memory() for a in host_A]
+    h_pin = [None if h is None else h.pin_memory() for h in host_h]
+    hout = {}
+    for wl, k in zip(wls, ks):
+        if (wl.m, wl.n, k) not in hout:
+            hout[(wl.m, wl.n, k)] = (torch.empty((wl.m, k), dtype=torch.int8, pin_memory=True),
+                                     torch.empty((k,), dtype=torch.float32, pin_memory=True),
+                                     torch.empty((k, wl.n), dtype=torch.int8, pin_memory=True))
+
+    def e2e_step():
+        for i, (wl, k) in enumerate(zip(wls, ks)):
+            X.decompose_host(A_pin[i], wl.mu, wl.tau, wl.block, wl.iters, h_pin[i], out=hout[(wl.m, wl.n, k)])
+
     for _ in range(max(1, min(args.warmup, 2))):
-        X.decompose_host(A_pin, wl.mu, wl.tau, wl.block, wl.iters, h_pin, out=hout)
+        e2e_step()
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for i in range(args.steps):
         flush.fill_(float(i))
-        X.decompose_host(A_pin, wl.mu, wl.tau, wl.block, wl.iters, h_pin, out=hout)
+        e2e_step()
     e1.record(stream)
     barrier()
-    e2e_value = job_rate(world, k * args.steps, max_over_ranks(e0.elapsed_time(e1), dev, world))
-    nblocks = -(-k // block_width(wl))
-    h2d = 4 * wl.m * wl.n + (4 * wl.n if wl.weighted else 0)
-    d2h = wl.m * k + k * wl.n + 4 * k + 8 * nblocks
+    e2e_value = job_rate(world, comps * args.steps, max_over_ranks(e0.elapsed_time(e1), dev, world))
+    h2d = sum(4 * wl.m * wl.n + (4 * wl.n if wl.weighted else 0) for wl in wls)
+    d2h = sum(wl.m * k + k * wl.n + 4 * k + 8 for wl, k in zip(wls, ks))
 
-    # ---- live roofline of the dominant kernel: event pairs inside the graph, over a second timed pass
+    # ---- live roofline of the dominant kernel class: event pairs inside the graph, over a second timed pass
     kind = args.roofline_kind
     X.profile(kind)
     for _ in range(2):
         flush.fill_(0.0)
         step()
-    X.profile_read()
-    prof_ms, prof_n = 0.0, 0
+    prof_ms, prof_n, prof_bytes = 0.0, 0, 0.0
     for i in range(args.steps):
         flush.fill_(float(i))
-        step()
-        a, b = X.profile_read()
-        prof_ms += a
-        prof_n += b
+        for j, wl in enumerate(wls):
+            X.decompose(As[j], wl.mu, wl.tau, wl.block, wl.iters, hs[j], out=outs[j])
+            a, b = X.profile_read()
+            prof_ms += a
+            prof_n += b
+            prof_bytes += b * algorithmic_bytes(kind, wl)
     X.profile("off")
     per_launch_s = prof_ms / 1e3 / max(prof_n, 1)
-    bytes_per_launch = algorithmic_bytes(kind, wl)
+    bytes_per_launch = prof_bytes / max(prof_n, 1)
     achieved = bytes_per_launch / per_launch_s / 1e9
     peak, peak_src = peaks()
-    src = os.path.join(ROOT, "paper_2607_13511_gb300", "csrc", NCU_TRAFFIC.get("file", "gemm.cu"))
     traffic = None
-    if NCU_TRAFFIC.get("kind") == kind and NCU_TRAFFIC.get("sha") == source_sha(src) \
-            and NCU_TRAFFIC.get("workload") == wl.name:
+    src = os.path.join(ROOT, "paper_2607_13511_gb300", "csrc", NCU_TRAFFIC.get("file", "gemm.cu"))
+    if NCU_TRAFFIC.get("kind") == kind and os.path.exists(src) and NCU_TRAFFIC.get("sha") == source_sha(src) \
+            and NCU_TRAFFIC.get("workload") == args.workload:
         traffic = NCU_TRAFFIC["bytes_per_launch"]
 
     if rank != 0:
@@ -329,30 +397,45 @@ def run_gpu(args):
             dist.destroy_process_group()
         return
 
+    step_bytes = sum(decomposition_bytes(wl) for wl in wls)
+    ms_step = ms_max / args.steps
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded numpy PCG64; see workloads.py)",
-        "config": {**config_of(wl), "parallelism": f"replicas x{world}"},
-        "energy": energy,
+        "config": {**config_of(args.workload), "parallelism": f"replicas x{world}"},
     }
-    g = golden_energy(wl.name)
-    line["delta_E_vs_oracle"] = None if g is None else energy - g
+    deltas = {}
+    for wl, e in zip(wls, energies):
+        g = golden_energy(wl.name)
+        if g is not None:
+            deltas[wl.name] = e - g
+    if len(wls) == 1:
+        line["energy"] = energies[0]
+        line["delta_E_vs_oracle"] = deltas.get(wls[0].name)
+    else:
+        line["energy"] = {"min": min(energies), "median": statistics.median(energies), "max": max(energies)}
+        line["delta_E_vs_oracle"] = {"matrices": len(deltas),
+                                     "max_abs": max((abs(d) for d in deltas.values()), default=None),
+                                     "per_matrix": deltas}
     line["e2e"] = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                    "path": "externd_decompose_host (pinned host buffers)"}
-    line["gpu_launches"] = launches_per_step * args.steps
+    line["gpu_launches"] = launches
     line["roofline"] = {"bound": "hbm", "kernel": kind, "achieved": achieved, "peak": peak, "unit": "GB/s",
                         "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
                         "bytes_per_launch": bytes_per_launch, "launches": prof_n,
                         "us_per_launch": per_launch_s * 1e6}
+    line["step_roofline"] = {"algorithmic_bytes": step_bytes, "lower_bound_ms": step_bytes / (peak * 1e6),
+                             "frac": step_bytes / (peak * 1e6) / ms_step}
     cs = clocks.summary()
     if cs is not None:
         line["clocks"] = cs
     if world == 1 and not args.no_cpu_baseline:
-        kk, dt = oracle_sample(wl, args.cpu_blocks)
+        swl = sample_workload(args.workload)
+        kk, dt = oracle_sample(swl, args.cpu_blocks)
         line["cpu_baseline"] = {"value": kk / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
-                                "sample": f"first {args.cpu_blocks} blocks ({kk} of {k} components) of {wl.name}, "
-                                          f"{dt:.1f} s"}
+                                "sample": f"first {args.cpu_blocks} blocks ({kk} of {inner_rank(swl)} components) "
+                                          f"of {swl.name}, {dt:.1f} s"}
     print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -390,7 +473,7 @@ def run_row(args):
     k = X.rank(wl.m, wl.n, wl.mu)
     peak, peak_src = peaks()
     line = {"row": args.row, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "vs_baseline": None,
-            "data": "synthetic (seeded numpy PCG64; see workloads.py)", "config": config_of(wl)}
+            "data": "synthetic (seeded numpy PCG64; see workloads.py)", "config": config_of(wl.name)}
     if args.row in ("safeguard", "refine"):
         A_np = wl.matrix()
         A = torch.from_numpy(A_np).to(dev)
@@ -494,10 +577,10 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
-    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(W.WORKLOADS))
-    ap.add_argument("--roofline-kind", default=ROOFLINE_KIND, choices=["vstep", "ustep", "deflate"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(JOBS))
+    ap.add_argument("--roofline-kind", default=ROOFLINE_KIND, choices=["products", "vstep", "ustep", "deflate"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-blocks", type=int, default=48, help="blocks of the workload the CPU baseline times")
+    ap.add_argument("--cpu-blocks", type=int, default=16, help="blocks of the workload the CPU baseline times")
     ap.add_argument("--reference-blocks", type=int, default=2, help="blocks per step of the reference arm")
     ap.add_argument("--row", default="decompose", choices=["decompose", "safeguard", "refine", "packed"],
                     help="an extension row instead of the headline decomposition (one GPU)")

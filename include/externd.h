@@ -59,24 +59,32 @@ int externd_rank(int64_t m, int64_t n, double mu, int64_t *k);
 int externd_block_width(int64_t m, int64_t n, int block, int *b);
 
 /*
- * The whole method (§2.3 when the block width is 1, §2.4 otherwise; §2.5 when weights != NULL).
+ * The whole method (§2.3 when the block width is 1, §2.4 otherwise; §2.5 when weights != NULL), for the
+ * problem statement of §2.1 (Eq. 1).
  *   A        m x n float32, read only.
  *   mu > 0   rank multiplier; k = externd_rank(m, n, mu).   tau >= 0: Eq. 2 threshold scale.
  *   block >= 1 requested block width (clamped as externd_block_width; the last block is k mod b wide when
  *            that is non-zero).   iters >= 1: ALS iterations per component/block (one V-step + one U-step).
  *   weights  n float32 or NULL.
  *   B        m x k int8 out;  D  k float32 out;  C  k x n int8 out.
- *   energy   host double out: E = 1 - ||R||^2 / ||A||^2 (weighted by h~ when weights != NULL, §2.5) from the
- *            final residual R = A - B diag(D) C kept in float32 on the device.
- *   trace    host double[nblocks] out or NULL: the energy after each block (nblocks = ceil(k / b)).
+ *   energy   host double out, or NULL: E = 1 - ||R||^2 / ||A||^2 (weighted by h~ when weights != NULL, §2.5)
+ *            from the final residual R = A - B diag(D) C kept in float32 on the device. With energy != NULL the
+ *            call returns after the energy reached the host; with NULL it only enqueues the work.
  */
 int externd_decompose(const float *A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
-                      const float *weights, int8_t *B, float *D, int8_t *C, double *energy, double *trace);
+                      const float *weights, int8_t *B, float *D, int8_t *C, double *energy);
+
+/* externd_decompose that also reports the energy after every block, the E(k) curve at k = b, 2b, ..., k that
+ * the rank budgets below read (greedy deflation, §2.3 / §2.4, makes it the energy of every shorter run).
+ *   trace    host double[nblocks] out or NULL (nblocks = ceil(k / b)).
+ * Everything else as externd_decompose; the factors are identical. */
+int externd_decompose_traced(const float *A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
+                             const float *weights, int8_t *B, float *D, int8_t *C, double *energy, double *trace);
 
 /* Same as externd_decompose with every array in HOST memory (pageable or pinned): the library copies A and
  * weights to the device, runs the method, and copies B, D, C back before returning. */
 int externd_decompose_host(const float *A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
-                           const float *weights, int8_t *B, float *D, int8_t *C, double *energy, double *trace);
+                           const float *weights, int8_t *B, float *D, int8_t *C, double *energy);
 
 /* Eq. 1 (weighted form of §2.5): energy = 1 - sum_ij h_j (A - B diag(D) C)_ij^2 / sum_ij h_j A_ij^2, with B
  * m x k, D k, C k x n on the device; energy is a host double. */
@@ -101,7 +109,8 @@ int externd_energy_noalloc(const float *A, int64_t m, int64_t n, const int8_t *B
  * Measurement. Not part of the method: lets a caller time one kernel class inside externd_decompose with CUDA
  * events (recorded as nodes of the captured graph, on the stream the kernels run on).
  *   kind: 0 off, 1 V-step product, 2 U-step product, 3 deflation, 4 decorrelation (Eq. 3), 5 Eq. 2 apply,
- *         6 Gram matrices, 7 small solves (inverse + Eq. 4), 8 block start (select + gather).
+ *         6 Gram matrices, 7 small solves (inverse + Eq. 4), 8 block start (select + gather), 9 both residual
+ *         products (1 and 2).
  * ------------------------------------------------------------------------------------------------------- */
 int externd_profile(int kind);
 

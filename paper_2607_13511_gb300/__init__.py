@@ -14,7 +14,8 @@ from dataclasses import dataclass
 from typing import Optional
 
 __all__ = [
-    "ExterndError", "Decomposition", "library_path", "load", "rank", "block_width", "decompose", "decompose_host",
+    "ExterndError", "Decomposition", "library_path", "load", "rank", "block_width", "decompose", "decompose_traced",
+    "decompose_host",
     "energy", "ternarize", "vstep_product", "ustep_product", "vstep_target", "ustep_target", "block_scales",
     "deflate", "profile", "profile_read", "kernel_launches", "PROFILE_KINDS", "Packed", "pack_ternary",
     "ternary_apply", "block_boundaries", "rank_for_energy", "allocate_ranks", "decompose_safeguarded", "refine",
@@ -35,9 +36,11 @@ _SIGNATURES = {
     "externd_rank": (_c_int, [_c_i64, _c_i64, _c_double, ctypes.POINTER(_c_i64)]),
     "externd_block_width": (_c_int, [_c_i64, _c_i64, _c_int, ctypes.POINTER(_c_int)]),
     "externd_decompose": (_c_int, [_c_void, _c_i64, _c_i64, _c_double, _c_double, _c_int, _c_int, _c_void,
-                                   _c_void, _c_void, _c_void, _c_dptr, _c_dptr]),
+                                   _c_void, _c_void, _c_void, _c_dptr]),
+    "externd_decompose_traced": (_c_int, [_c_void, _c_i64, _c_i64, _c_double, _c_double, _c_int, _c_int,
+                                          _c_void, _c_void, _c_void, _c_void, _c_dptr, _c_dptr]),
     "externd_decompose_host": (_c_int, [_c_void, _c_i64, _c_i64, _c_double, _c_double, _c_int, _c_int, _c_void,
-                                        _c_void, _c_void, _c_void, _c_dptr, _c_dptr]),
+                                        _c_void, _c_void, _c_void, _c_dptr]),
     "externd_energy": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_void, _c_i64, _c_void, _c_dptr]),
     "externd_energy_noalloc": (_c_int, [_c_void, _c_i64, _c_i64, _c_void, _c_void, _c_void, _c_i64, _c_void,
                                         _c_dptr]),
@@ -123,7 +126,7 @@ def _stream(lib, device) -> None:
 
 
 PROFILE_KINDS = {"off": 0, "vstep": 1, "ustep": 2, "deflate": 3, "decorrelate": 4, "apply": 5, "gram": 6,
-                 "solve": 7, "start": 8}
+                 "solve": 7, "start": 8, "products": 9}
 
 
 def profile(kind: str) -> None:
@@ -165,19 +168,15 @@ class Decomposition:
     D: "object"          # k float32
     C: "object"          # k x n int8 {-1, 0, 1}
     energy: float        # 1 - ||A - B diag(D) C||_H^2 / ||A||_H^2 (tracked residual)
-    trace: list          # energy after each block
+    trace: Optional[list] = None   # energy after each block (decompose_traced, the extension entry points)
 
 
-def decompose(A, mu: float, tau: float, block: int, iters: int, weights=None, out=None) -> Decomposition:
-    """ExTernD of a CUDA float32 matrix A (m x n): §2.3 (block 1) / §2.4 block ALS, §2.5 when weights is given.
-
-    ``out`` may pass preallocated (B, D, C) tensors to reuse."""
+def _decompose_call(fn_name, A, mu, tau, block, iters, weights, out, traced):
     torch = _torch()
     lib = load()
     A = _prep(A, torch.float32, "A")
     m, n = A.shape
     k = rank(m, n, mu)
-    nblocks = -(-k // block_width(m, n, block))
     h = None if weights is None else _prep(weights, torch.float32, "weights")
     if out is None:
         B = torch.empty((m, k), dtype=torch.int8, device=A.device)
@@ -186,12 +185,28 @@ def decompose(A, mu: float, tau: float, block: int, iters: int, weights=None, ou
     else:
         B, D, C = out
     e = _c_double()
-    tr = (_c_double * nblocks)()
+    args = [_ptr(A), m, n, mu, tau, block, iters, _ptr(h), _ptr(B), _ptr(D), _ptr(C), ctypes.byref(e)]
+    tr = None
+    if traced:
+        tr = (_c_double * -(-k // block_width(m, n, block)))()
+        args.append(tr)
     with torch.cuda.device(A.device):
         _stream(lib, A.device)
-        _check(lib.externd_decompose(_ptr(A), m, n, mu, tau, block, iters, _ptr(h), _ptr(B), _ptr(D), _ptr(C),
-                                     ctypes.byref(e), tr))
-    return Decomposition(B, D, C, e.value, list(tr))
+        _check(getattr(lib, fn_name)(*args))
+    return Decomposition(B, D, C, e.value, None if tr is None else list(tr))
+
+
+def decompose(A, mu: float, tau: float, block: int, iters: int, weights=None, out=None) -> Decomposition:
+    """ExTernD of a CUDA float32 matrix A (m x n): §2.3 (block 1) / §2.4 block ALS, §2.5 when weights is given.
+
+    ``out`` may pass preallocated (B, D, C) tensors to reuse. The result carries no per-block trace (see
+    ``decompose_traced``)."""
+    return _decompose_call("externd_decompose", A, mu, tau, block, iters, weights, out, False)
+
+
+def decompose_traced(A, mu: float, tau: float, block: int, iters: int, weights=None, out=None) -> Decomposition:
+    """``decompose`` that also returns the energy after every block (``trace``): E(k) at k = b, 2b, ..., k."""
+    return _decompose_call("externd_decompose_traced", A, mu, tau, block, iters, weights, out, True)
 
 
 def decompose_safeguarded(A, mu: float, tau: float, block: int, iters: int, weights=None, out=None):
@@ -256,7 +271,6 @@ def decompose_host(A, mu: float, tau: float, block: int, iters: int, weights=Non
     A = A.contiguous()
     m, n = A.shape
     k = rank(m, n, mu)
-    nblocks = -(-k // block_width(m, n, block))
     h = None if weights is None else weights.contiguous()
     if out is None:
         pin = torch.cuda.is_available()
@@ -266,11 +280,10 @@ def decompose_host(A, mu: float, tau: float, block: int, iters: int, weights=Non
     else:
         B, D, C = out
     e = _c_double()
-    tr = (_c_double * nblocks)()
     _stream(lib, torch.cuda.current_device())
     _check(lib.externd_decompose_host(_ptr(A), m, n, mu, tau, block, iters, _ptr(h), _ptr(B), _ptr(D), _ptr(C),
-                                      ctypes.byref(e), tr))
-    return Decomposition(B, D, C, e.value, list(tr))
+                                      ctypes.byref(e)))
+    return Decomposition(B, D, C, e.value)
 
 
 def energy(A, B, D, C, weights=None) -> float:

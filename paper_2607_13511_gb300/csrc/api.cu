@@ -269,6 +269,7 @@ struct Bufs {
   int nbest;
   BlockChoice* choice;
   long long* counts;      // activations (safeguard) or replaced blocks per sweep (refinement)
+  IoTable* io;            // the caller's A, B, D, C for this run (decompose modes; set before each replay)
 };
 
 int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
@@ -330,6 +331,7 @@ int plan_buffers(Workspace& ws, const Plan& p, Bufs* B) {
   B->norm_r = B->norm_a + 1;
   B->norm_add = B->norm_a + 2;
   TRY(need(ws, "trace", (size_t)std::max(p.nblocks, p.sweeps), &B->trace));
+  TRY(need(ws, "io", 1, &B->io, true));
   B->K = nullptr;
   B->best = nullptr;
   B->nbest = 0;
@@ -374,13 +376,17 @@ Plan make_plan(long long m, long long n, long long k, int block, int iters, doub
 // A kernel launch of class `kind` that launches `nk` kernels: counted, and bracketed by events when profiled.
 #define KLS(kind_, nk, st_, call)                           \
   do {                                                      \
-    const bool prof_ = g_prof.kind != 0 && g_prof.kind == (kind_); \
+    const bool prof_ = g_prof.kind != 0 && prof_match(kind_); \
     if (prof_) LK(prof_mark(st_));                          \
     LK(call);                                               \
     if (prof_) LK(prof_mark(st_));                          \
     g_prof.launches += (nk);                                \
   } while (0)
 #define KL(kind_, nk, call) KLS(kind_, nk, s, call)
+// Whether a launch of class kind is instrumented under the current selector.
+inline bool prof_match(int kind) {
+  return g_prof.kind == kind || (g_prof.kind == 9 && (kind == 1 || kind == 2));
+}
 // Fork the side branch from stream s / join it back into s.
 #define FORK()                                              \
   do {                                                      \
@@ -395,7 +401,8 @@ Plan make_plan(long long m, long long n, long long k, int block, int iters, doub
     LK(cudaStreamWaitEvent(s, ws.ev_join, 0));              \
   } while (0)
 
-enum Kind { kVstep = 1, kUstep = 2, kDeflate = 3, kDecor = 4, kApply = 5, kGram = 6, kSolve = 7, kStart = 8 };
+enum Kind { kVstep = 1, kUstep = 2, kDeflate = 3, kDecor = 4, kApply = 5, kGram = 6, kSolve = 7, kStart = 8,
+            kProducts = 9 /* both residual products: profiling selector only */ };
 
 // Thresholds and statistics of the Eq. 2 producers (per-block chunk counts set by fit_block).
 struct Eq2 {
@@ -559,9 +566,13 @@ int deflate_step(const Plan& p, const Bufs& B, const float* h, int w, double* no
   return EXTERND_OK;
 }
 
-// R = A with column energies, ||A||_H^2 and the fp16 scaling scalars.
+// R = A with column energies, ||A||_H^2 and the fp16 scaling scalars. A == nullptr: A is B.io->A, copied first.
 int start_residual(const Plan& p, const Bufs& B, const float* A, const float* h, cudaStream_t s) {
   const int m = p.m, n = p.n;
+  if (A == nullptr) {
+    KL(0, 1, launch_io_copy_in(B.io, B.R, (long long)m * n, s));
+    A = B.R;
+  }
   KL(kDeflate, 1, launch_deflate(A, B.R, m, n, nullptr, 0, false, nullptr, nullptr, 0, 0, h, B.colpart, B.normpart, s,
                                  B.maxpart));
   KL(0, 1, launch_norm(B.normpart, deflate_tiles(m, n), B.norm_a, nullptr, nullptr, s, B.maxpart, B.maxabs));
@@ -569,15 +580,15 @@ int start_residual(const Plan& p, const Bufs& B, const float* A, const float* h,
   return EXTERND_OK;
 }
 
-// Enqueues the whole decomposition on stream s (with Prop. 2's safeguard when p.mode == kSafeguard).
-int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* A, const float* h, int8_t* Bout,
-                      float* Dout, int8_t* Cout, cudaStream_t s) {
+// Enqueues the whole decomposition on stream s (with Prop. 2's safeguard when p.mode == kSafeguard). The caller's
+// A, B, D, C are not named here: the graph reads them from B.io, set on the stream before each run.
+int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* h, cudaStream_t s) {
   cudaStream_t side = ws.side;
   const int m = p.m, n = p.n;
   Eq2 q = make_eq2(p, B);
   g_prof.used = 0;
   g_prof.launches = 0;
-  TRY(start_residual(p, B, A, h, s));
+  TRY(start_residual(p, B, nullptr, h, s));
   const bool guard = p.mode == kSafeguard;
   for (int blk = 0; blk < p.nblocks; ++blk) {
     const long long j0 = (long long)blk * p.b;
@@ -589,9 +600,8 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
       // The block's outputs leave on the side branch: B from the final U and C from the final V now, D after the
       // scales; the next block joins before it overwrites Ut.
       FORK();
-      KLS(0, 1, side, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, side));
-      LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
-                           cudaMemcpyDeviceToDevice, side));
+      KLS(0, 1, side, launch_write_b(B.Ut, (int)p.ldm, w, m, nullptr, p.k, j0, side, B.io));
+      KLS(0, 1, side, launch_io_write_c(B.Vt, p.ldn, w, p.n, B.io, j0, side));
     }
     TRY(block_scales_step(p, B, w, guard ? B.K : nullptr, s));
     if (guard) {
@@ -599,13 +609,12 @@ int enqueue_decompose(Workspace& ws, const Plan& p, const Bufs& B, const float* 
       KL(0, 1, launch_safeguard_replace(B.choice, w, m, n, B.Ut, p.ldm, B.Vt, p.ldn, use_tc(w) ? B.Uk16 : nullptr,
                                         use_tc(w) ? B.Vk16 : nullptr, B.ldk, s));
       FORK();
-      KLS(0, 1, side, launch_write_b(B.Ut, (int)p.ldm, w, m, Bout, p.k, j0, side));
-      LK(cudaMemcpy2DAsync(Cout + j0 * n, (size_t)n, B.Vt, (size_t)p.ldn, (size_t)n, (size_t)w,
-                           cudaMemcpyDeviceToDevice, side));
+      KLS(0, 1, side, launch_write_b(B.Ut, (int)p.ldm, w, m, nullptr, p.k, j0, side, B.io));
+      KLS(0, 1, side, launch_io_write_c(B.Vt, p.ldn, w, p.n, B.io, j0, side));
     } else {
       FORK();
     }
-    LK(cudaMemcpyAsync(Dout + j0, B.d, sizeof(float) * w, cudaMemcpyDeviceToDevice, side));
+    KLS(0, 1, side, launch_io_write_d(B.d, w, B.io, j0, side));
     TRY(deflate_step(p, B, h, w, B.norm_r, B.trace + blk, s));
   }
   if (p.nblocks > 0) JOIN();
@@ -701,13 +710,17 @@ int run_plan(const Plan& p, const float* A, const float* h, int8_t* Bout, float*
   int dev;
   CK(cudaGetDevice(&dev));
   cudaStream_t s = g_stream;
+  // The decompose modes read the caller's arrays through B.io, so their graphs serve every A, B, D, C of a shape;
+  // refinement updates the factors in place at many nodes and keeps them in its graph.
+  const bool via_io = p.mode != kRefine;
   auto enqueue = [&](cudaStream_t st) {
     return p.mode == kRefine ? enqueue_refine(*ws, p, B, A, h, Bout, Dout, Cout, st)
-                             : enqueue_decompose(*ws, p, B, A, h, Bout, Dout, Cout, st);
+                             : enqueue_decompose(*ws, p, B, h, st);
   };
+  if (via_io) LK(launch_io_set(B.io, A, Bout, Dout, Cout, s));
   if (graphs_enabled()) {
-    GraphKey key{A, h, Bout, Dout, Cout, p.m, p.n, p.k, p.b, p.iters, p.tau, ws->generation, g_prof.kind, p.mode,
-                 p.sweeps};
+    GraphKey key{via_io ? nullptr : A, h, via_io ? nullptr : Bout, via_io ? nullptr : Dout, via_io ? nullptr : Cout,
+                 p.m, p.n, p.k, p.b, p.iters, p.tau, ws->generation, g_prof.kind, p.mode, p.sweeps};
     auto& cache = g_graphs[dev];
     auto it = cache.find(key);
     if (it == cache.end()) {
@@ -729,11 +742,11 @@ int run_plan(const Plan& p, const float* A, const float* h, int8_t* Bout, float*
     }
     CK(cudaGraphLaunch(it->second.exec, s));
     g_prof.last_used = it->second.events;
-    g_prof.last_launches = it->second.launches;
+    g_prof.last_launches = it->second.launches + (via_io ? 1 : 0);
   } else {
     TRY(enqueue(s));
     g_prof.last_used = g_prof.used;
-    g_prof.last_launches = g_prof.launches;
+    g_prof.last_launches = g_prof.launches + (via_io ? 1 : 0);
   }
   if (energy != nullptr || trace != nullptr || counts != nullptr) {
     const size_t tb = sizeof(double) * (size_t)ntrace, cb = sizeof(long long) * (size_t)ncounts;
@@ -871,7 +884,7 @@ int externd_set_stream(void* cuda_stream) {
 
 int externd_profile(int kind) {
   std::lock_guard<std::mutex> lock(g_mutex);
-  if (kind < 0 || kind > 8) return EXTERND_EINVAL;
+  if (kind < 0 || kind > 9) return EXTERND_EINVAL;
   g_prof.kind = kind;
   return EXTERND_OK;
 }
@@ -914,13 +927,16 @@ int externd_block_width(int64_t m, int64_t n, int block, int* b) {
 }
 
 int externd_decompose(const float* A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
-                      const float* weights, int8_t* B, float* D, int8_t* C, double* energy, double* trace) {
+                      const float* weights, int8_t* B, float* D, int8_t* C, double* energy) {
+  return externd_decompose_traced(A, m, n, mu, tau, block, iters, weights, B, D, C, energy, nullptr);
+}
+
+int externd_decompose_traced(const float* A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
+                             const float* weights, int8_t* B, float* D, int8_t* C, double* energy, double* trace) {
   std::lock_guard<std::mutex> lock(g_mutex);
   TRY(check_common(m, n));
   TRY(check_params(mu, tau, block, iters));
-  if (energy == nullptr && trace == nullptr) {
-    // results still land in B, D, C; nothing to report on the host
-  }
+  // with energy == trace == NULL the results still land in B, D, C and nothing is read back
   TRY(check_dev(A));
   TRY(check_dev(B));
   TRY(check_dev(D));
@@ -970,7 +986,7 @@ int externd_refine(const float* A, int64_t m, int64_t n, double tau, int block, 
 }
 
 int externd_decompose_host(const float* A, int64_t m, int64_t n, double mu, double tau, int block, int iters,
-                           const float* weights, int8_t* B, float* D, int8_t* C, double* energy, double* trace) {
+                           const float* weights, int8_t* B, float* D, int8_t* C, double* energy) {
   std::lock_guard<std::mutex> lock(g_mutex);
   TRY(check_common(m, n));
   TRY(check_params(mu, tau, block, iters));
@@ -989,7 +1005,7 @@ int externd_decompose_host(const float* A, int64_t m, int64_t n, double mu, doub
   cudaStream_t s = g_stream;
   CK(cudaMemcpyAsync(dA, A, sizeof(float) * m * n, cudaMemcpyHostToDevice, s));
   if (weights) CK(cudaMemcpyAsync(dh, weights, sizeof(float) * n, cudaMemcpyHostToDevice, s));
-  TRY(run_decompose(dA, m, n, mu, tau, block, iters, dh, dB, dD, dC, energy, trace));
+  TRY(run_decompose(dA, m, n, mu, tau, block, iters, dh, dB, dD, dC, energy, nullptr));
   CK(cudaMemcpyAsync(B, dB, (size_t)m * k, cudaMemcpyDeviceToHost, s));
   CK(cudaMemcpyAsync(C, dC, (size_t)k * n, cudaMemcpyDeviceToHost, s));
   CK(cudaMemcpyAsync(D, dD, sizeof(float) * k, cudaMemcpyDeviceToHost, s));

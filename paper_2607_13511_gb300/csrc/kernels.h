@@ -18,6 +18,23 @@
 
 namespace externd {
 
+// Addresses of the caller's arrays of one decomposition, read on the device by the graph nodes that touch them
+// (io.cu), so one captured graph serves every matrix of its shape.
+struct IoTable {
+  const float* A;
+  int8_t* B;
+  float* D;
+  int8_t* C;
+};
+cudaError_t launch_io_set(IoTable* t, const float* A, int8_t* B, float* D, int8_t* C, cudaStream_t s);
+// R = t->A (count floats)
+cudaError_t launch_io_copy_in(const IoTable* t, float* R, long long count, cudaStream_t s);
+// rows j0 .. j0 + w - 1 of t->C (k x n) = Vt's w rows (ld ldv, a multiple of 16)
+cudaError_t launch_io_write_c(const int8_t* Vt, long long ldv, int w, int n, const IoTable* t, long long j0,
+                              cudaStream_t s);
+// t->D[j0 .. j0 + w) = d
+cudaError_t launch_io_write_d(const float* d, int w, const IoTable* t, long long j0, cudaStream_t s);
+
 // Eq. 2 thresholds of nv vectors of length L: theta = RD_float(tau * S / L), whether nothing passes, and the
 // fallback index. The last CTA of the statistics producer writes them (ticket counts finished CTAs and is reset
 // to zero by that CTA).
@@ -250,8 +267,9 @@ cudaError_t launch_norm(const F2* normpart, int count, double* out, const double
                         cudaStream_t s, const float* maxpart = nullptr, float* maxout = nullptr);
 // out[0] = max |x_i|
 cudaError_t launch_absmax(const float* x, long long n, float* out, cudaStream_t s);
+// B[r][j0 + a] = Ut[a][r]; with io, B is io->B (read on the device).
 cudaError_t launch_write_b(const int8_t* Ut, int ldu, int w, int m, int8_t* B, long long k, long long j0,
-                           cudaStream_t s);
+                           cudaStream_t s, const IoTable* io = nullptr);
 // dst[c][r] = src[r][c] for an rows x cols int8 / float32 matrix (leading dims given).
 cudaError_t launch_transpose_i8(const int8_t* src, long long lds, int rows, int cols, int8_t* dst, long long ldd,
                                 cudaStream_t s);

@@ -49,9 +49,13 @@ extern "C" int externd_energy_noalloc(const float* A, int64_t m, int64_t n, cons
   using namespace externd;
   std::lock_guard<std::mutex> lock(library_mutex());
   if (A == nullptr || B == nullptr || D == nullptr || C == nullptr || energy == nullptr) return EXTERND_EINVAL;
-  if (m < 1 || n < 1 || k < 1 || m > 65535LL * 64 || n > (1LL << 30) || k > (1LL << 31)) return EXTERND_EINVAL;
-  const long long tiles = deflate_tiles((int)m, (int)n);
+  // the size limits of every other entry point (row tiles of 64 in gridDim.y, m * n <= 2^40) and k below 2^31
+  if (m < 1 || n < 1 || k < 1 || m > 65535LL * 64 || n > (1LL << 30) || m * n > (1LL << 40) || k >= (1LL << 31))
+    return EXTERND_EINVAL;
+  // tiles of 64 rows x 128 columns (the deflation kernel's), counted in 64 bits so no size can wrap
+  const long long tiles = cdiv(m, 64) * cdiv(n, 128);
   if (tiles + 3 > kScratch) return EXTERND_EINVAL;   // larger than the fixed scratch: see the header
+  if (tiles != (long long)deflate_tiles((int)m, (int)n)) return EXTERND_EINVAL;
   if (!device_reachable(A) || !device_reachable(B) || !device_reachable(D) || !device_reachable(C) ||
       (weights != nullptr && !device_reachable(weights)))
     return EXTERND_EPTR;

@@ -370,15 +370,17 @@ __global__ void __launch_bounds__(1024) absmax_kernel(const float* __restrict__ 
 // B[r][j0 + a] = Ut[a][r] for a 64-row slab: read Ut rows coalesced, transpose in shared memory, write each
 // row's w bytes as 4-byte words when aligned.
 __global__ void __launch_bounds__(256) write_b_kernel(const int8_t* __restrict__ Ut, int ldu, int w, int m,
-                                                      int8_t* __restrict__ B, long long k, long long j0) {
+                                                      int8_t* __restrict__ B, long long k, long long j0,
+                                                      const IoTable* __restrict__ io) {
   __shared__ int8_t tile[kMaxBlock][68];
+  if (io != nullptr) B = io->B;
   const int r0 = blockIdx.x * 64;
   for (int i = threadIdx.x; i < w * 64; i += 256) {
     const int a = i >> 6, r = i & 63;
     tile[a][r] = (r0 + r < m) ? Ut[(long long)a * ldu + r0 + r] : (int8_t)0;
   }
   __syncthreads();
-  const bool words = ((k & 3) == 0) && ((j0 & 3) == 0) && ((w & 3) == 0);
+  const bool words = ((k & 3) == 0) && ((j0 & 3) == 0) && ((w & 3) == 0) && ((reinterpret_cast<uintptr_t>(B) & 3) == 0);
   if (words) {
     const int wq = w >> 2;
     for (int i = threadIdx.x; i < 64 * wq; i += 256) {
@@ -522,8 +524,8 @@ cudaError_t launch_absmax(const float* x, long long n, float* out, cudaStream_t 
 }
 
 cudaError_t launch_write_b(const int8_t* Ut, int ldu, int w, int m, int8_t* B, long long k, long long j0,
-                           cudaStream_t s) {
-  write_b_kernel<<<(unsigned)cdiv(m, 64), 256, 0, s>>>(Ut, ldu, w, m, B, k, j0);
+                           cudaStream_t s, const IoTable* io) {
+  write_b_kernel<<<(unsigned)cdiv(m, 64), 256, 0, s>>>(Ut, ldu, w, m, B, k, j0, io);
   return cudaGetLastError();
 }
 

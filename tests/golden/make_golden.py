@@ -4,7 +4,9 @@ Calls only ``oracle/`` (the fp64 CPU restatement of the method) and the seeded g
 from the CUDA path. The GPU tests compare the library's final energy with these values (|dE| <= 1e-4) at sizes
 where rerunning the oracle inside a test would take minutes.
 
-    python tests/golden/make_golden.py [workload names...]      # default: all, plus decoder layer 0
+    python tests/golden/make_golden.py [workload names...]      # default: all, plus decoder layers 0, 17, 35
+
+Decoder matrices are named L<layer>.<projection> (e.g. L17.gate); any of the 36 layers can be asked for.
 """
 import json
 import os
@@ -43,8 +45,10 @@ def run(wl: W.Workload) -> dict:
 def main(names):
     table = json.load(open(OUT)) if os.path.exists(OUT) else {}
     todo = {w.name: w for w in W.WORKLOADS.values()}
-    todo.update({w.name: w for w in W.decoder_conversion(layers=1)})
+    decoder = {w.name: w for w in W.decoder_conversion()}
+    todo.update({name: wl for name, wl in decoder.items() if name.split(".")[0] in ("L0", "L17", "L35")})
     for name in names or list(todo):
+        todo.setdefault(name, decoder.get(name))
         print(f"{name} ...", flush=True)
         table[name] = run(todo[name])
         print(f"  E = {table[name]['energy']:.8f} in {table[name]['oracle_seconds']:.1f} s", flush=True)

@@ -43,9 +43,59 @@ def test_library_exports_every_declared_symbol(lib):
     assert not missing, missing
 
 
+def prototypes():
+    """name -> (return type, [(parameter type, parameter name), ...]) for every declaration in the header."""
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    text = re.sub(r"#.*", "", text)
+    out = {}
+    for ret, name, params in re.findall(r"([A-Za-z_][\w \t*]*?)\b(externd_\w+)\s*\(([^)]*)\)\s*;", text):
+        plist = []
+        params = " ".join(params.split())
+        if params not in ("", "void"):
+            for p in params.split(","):
+                m = re.match(r"^\s*(.*?)\s*\b(\w+)\s*$", p)
+                plist.append((re.sub(r"\s*\*\s*", "*", m.group(1)).strip(), m.group(2)))
+        out[name] = (re.sub(r"\s*\*\s*", "*", " ".join(ret.split())).strip(), plist)
+    return out
+
+
+# The boundary calls exactly as the problem statement of §2.1 (Eq. 1), Eq. 2 and §2.5 fix them:
+# A (m x n), mu, tau, block, iters, optional weights, factors B, D, C, and the energy.
+BOUNDARY = {
+    "externd_decompose": ("int", [("const float*", "A"), ("int64_t", "m"), ("int64_t", "n"), ("double", "mu"),
+                                  ("double", "tau"), ("int", "block"), ("int", "iters"),
+                                  ("const float*", "weights"), ("int8_t*", "B"), ("float*", "D"),
+                                  ("int8_t*", "C"), ("double*", "energy")]),
+    "externd_energy": ("int", [("const float*", "A"), ("int64_t", "m"), ("int64_t", "n"), ("const int8_t*", "B"),
+                               ("const float*", "D"), ("const int8_t*", "C"), ("int64_t", "k"),
+                               ("const float*", "weights"), ("double*", "energy")]),
+    "externd_rank": ("int", [("int64_t", "m"), ("int64_t", "n"), ("double", "mu"), ("int64_t*", "k")]),
+    "externd_set_stream": ("int", [("void*", "cuda_stream")]),
+    "externd_strerror": ("const char*", [("int", "status")]),
+}
+
+
+def test_boundary_prototypes_are_exact():
+    protos = prototypes()
+    for name, want in BOUNDARY.items():
+        assert protos[name] == want, (name, protos[name])
+    # the host variant takes the same twelve parameters
+    assert protos["externd_decompose_host"] == BOUNDARY["externd_decompose"]
+    # the traced variant appends the per-block energies and nothing else
+    ret, params = protos["externd_decompose_traced"]
+    assert (ret, params[:-1]) == BOUNDARY["externd_decompose"] and params[-1] == ("double*", "trace")
+
+
 def test_binding_declares_every_symbol():
     import paper_2607_13511_gb300 as X
     assert sorted(X._SIGNATURES) == declared_symbols()
+
+
+def test_binding_argument_counts_match_the_header():
+    import paper_2607_13511_gb300 as X
+    protos = prototypes()
+    for name, (_, args) in X._SIGNATURES.items():
+        assert len(args) == len(protos[name][1]), name
 
 
 def test_host_side_rank_and_block_width_match_the_oracle(lib):

@@ -25,11 +25,11 @@ def X():
 def test_gpu_prefix_and_rank_for_energy(X, m, n, block):
     A = torch.from_numpy(W.student_t(m, n, 5.0, 0.015, m + n).astype(np.float32)).cuda()
     mu = 1.5
-    big = X.decompose(A, mu, 1.0, block, 3)
+    big = X.decompose_traced(A, mu, 1.0, block, 3)
     ranks = X.block_boundaries(m, n, mu, block)
     assert len(big.trace) == len(ranks)
     k1 = ranks[len(ranks) // 2 - 1]
-    small = X.decompose(A, k1 / min(m, n), 1.0, block, 3)
+    small = X.decompose_traced(A, k1 / min(m, n), 1.0, block, 3)
     torch.cuda.synchronize()
     assert small.B.shape[1] == k1
     assert torch.equal(small.B, big.B[:, :k1]) and torch.equal(small.C, big.C[:k1])

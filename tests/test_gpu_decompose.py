@@ -42,7 +42,8 @@ def check_valid(X, A, res, h, k):
     assert set(np.unique(B)) <= {-1, 0, 1} and set(np.unique(C)) <= {-1, 0, 1}
     assert (np.abs(B).sum(0) > 0).all() and (np.abs(C).sum(1) > 0).all()
     assert np.all(np.isfinite(D))
-    assert np.all(np.diff(res.trace) >= -1e-6)
+    if res.trace is not None:
+        assert np.all(np.diff(res.trace) >= -1e-6)
     e2 = X.energy(cuda(A), res.B, res.D, res.C, None if h is None else cuda(h))
     assert abs(e2 - res.energy) <= 1e-5
     return B, D, C
@@ -75,6 +76,12 @@ def test_decompose_matches_oracle(X, case):
     res = X.decompose(cuda(A), mu, tau, block, iters, None if h is None else cuda(h))
     check_valid(X, A, res, h, ref.D.size)
     assert abs(res.energy - ref.energy) <= 1e-4
+    # the traced entry point runs the same method: identical factors, and a monotone trace ending at E
+    tr = X.decompose_traced(cuda(A), mu, tau, block, iters, None if h is None else cuda(h))
+    check_valid(X, A, tr, h, ref.D.size)
+    assert torch.equal(tr.B, res.B) and torch.equal(tr.C, res.C) and torch.equal(tr.D, res.D)
+    assert tr.energy == res.energy == tr.trace[-1]
+    assert len(tr.trace) == len(ref.trace)
 
 
 def test_block_width_one_first_components_match_exactly(X):
@@ -131,12 +138,19 @@ def test_full_workloads_match_oracle_energy(X, name):
     assert abs(res.energy - golden[name]["energy"]) <= 1e-4
 
 
-def test_decoder_layer0_matches_oracle_energy(X):
+@pytest.mark.parametrize("layer", [0, 17, 35])
+def test_decoder_layers_match_oracle_energy(X, layer):
+    """Every projection of decoder layers 0, 17 and 35 of the 36-layer conversion, at full size."""
     golden = json.load(open(GOLDEN))
-    for wl in W.decoder_conversion(layers=1):
+    wls = [wl for wl in W.decoder_conversion() if wl.name.startswith(f"L{layer}.")]
+    if not any(wl.name in golden for wl in wls):
+        pytest.skip(f"decoder layer {layer} not in golden table")
+    for wl in wls:
         if wl.name not in golden:
             continue
-        res = X.decompose(cuda(wl.matrix()), wl.mu, wl.tau, wl.block, wl.iters)
+        A = wl.matrix()
+        res = X.decompose(cuda(A), wl.mu, wl.tau, wl.block, wl.iters)
+        assert res.D.numel() == golden[wl.name]["k"], wl.name
         assert abs(res.energy - golden[wl.name]["energy"]) <= 1e-4, wl.name
 
 
@@ -151,7 +165,7 @@ def test_error_conventions(X):
     e = ctypes.c_double()
 
     def call(Ap, m, n, mu, tau, block, iters, Bp=B.data_ptr(), Dp=D.data_ptr(), Cp=C.data_ptr()):
-        return lib.externd_decompose(Ap, m, n, mu, tau, block, iters, None, Bp, Dp, Cp, ctypes.byref(e), None)
+        return lib.externd_decompose(Ap, m, n, mu, tau, block, iters, None, Bp, Dp, Cp, ctypes.byref(e))
 
     assert call(A.data_ptr(), 32, 32, 1.0, 0.7, 4, 2) == 0
     assert call(A.data_ptr(), 0, 32, 1.0, 0.7, 4, 2) == -1          # bad size

@@ -77,7 +77,7 @@ def test_safeguard_matches_oracle_on_spikes(X, m, n, block):
 def test_safeguard_inactive_is_the_plain_method(X, block):
     A = W.gaussian(96, 200, 0.02, 9).astype(np.float32)
     res, act = X.decompose_safeguarded(cuda(A), 1.0, 0.7, block, 3)
-    plain = X.decompose(cuda(A), 1.0, 0.7, block, 3)
+    plain = X.decompose_traced(cuda(A), 1.0, 0.7, block, 3)
     torch.cuda.synchronize()
     assert act == 0
     assert torch.equal(res.B, plain.B) and torch.equal(res.C, plain.C) and torch.equal(res.D, plain.D)
@@ -111,7 +111,7 @@ def test_refine_matches_oracle(X, case):
     A = W.student_t(m, n, 5.0, 0.015, m * 7 + n).astype(np.float32)
     h = W.importance(n, m).astype(np.float32) if weighted else None
     hc = None if h is None else cuda(h)
-    dec = X.decompose(cuda(A), mu, tau, block, iters, hc)
+    dec = X.decompose_traced(cuda(A), mu, tau, block, iters, hc)
     ref_in = O.Result(*host(dec), dec.energy, dec.trace, None)
     out, replaced = X.refine(cuda(A), dec, tau, block, iters, sweeps, hc)
     ref, ref_replaced = N.refine(A.astype(np.float64), ref_in, tau, block, iters, sweeps,

@@ -58,3 +58,7 @@ def test_noalloc_rejects_problems_larger_than_its_scratch(lib):
     p = tiny.data_ptr()
     assert lib.externd_energy_noalloc(p, 16384, 16384, p, p, p, 1, None, ctypes.byref(e)) == -1
     assert lib.externd_energy_noalloc(None, 10, 10, p, p, p, 1, None, ctypes.byref(e)) == -1
+    # sizes whose tile count would wrap a 32-bit product, and k at 2^31: rejected, nothing launched
+    assert lib.externd_energy_noalloc(p, 65535 * 64, 4_300_000, p, p, p, 1, None, ctypes.byref(e)) == -1
+    assert lib.externd_energy_noalloc(p, 64, 1 << 30, p, p, p, 1, None, ctypes.byref(e)) == -1
+    assert lib.externd_energy_noalloc(p, 10, 10, p, p, p, 1 << 31, None, ctypes.byref(e)) == -1
