@@ -210,20 +210,26 @@ int splits_max(int w, int Lx, int Ly) { return std::max(splits_of(w, Lx, Ly, fal
 
 // The factor comes as int8 rows (FMA tiles) and as the same values in fp16 rows (tensor cores), both with
 // leading dimension ld elements.
+// The TMA-fed product of this shape and factor layout (the one that can run beside a cluster inverse).
+bool tma_path(int w, const float* R, int n, const __half* T16, int ld) {
+  return use_tc(w) && use_tma() && T16 != nullptr && tma_product_ok(R, n, T16, ld);
+}
+
 cudaError_t product_v(const float* R, int m, int n, const int8_t* Ut, const __half* Ut16, int ldu, int w, float* part,
-                      int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
+                      int splits, const float* maxabs, unsigned* err, cudaStream_t s, bool pdl = false) {
   if (use_tc(w)) {
     if (use_tma() && tma_product_ok(R, n, Ut16, ldu))
-      return launch_product_v_tma(R, m, n, Ut16, ldu, w, part, splits, maxabs, err, s);
+      return launch_product_v_tma(R, m, n, Ut16, ldu, w, part, splits, maxabs, err, s, pdl);
     return launch_product_v_tc(R, m, n, Ut16, ldu, w, part, splits, maxabs, err, s);
   }
   return launch_product_v(R, m, n, Ut, ldu, w, part, splits, s);
 }
 cudaError_t product_u(const float* R, int m, int n, const int8_t* Vt, const __half* Vt16, int ldv, int w,
-                      const float* h, float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
+                      const float* h, float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s,
+                      bool pdl = false) {
   if (use_tc(w)) {
     if (use_tma() && tma_product_ok(R, n, Vt16, ldv))
-      return launch_product_u_tma(R, m, n, Vt16, ldv, w, h, part, splits, maxabs, err, s);
+      return launch_product_u_tma(R, m, n, Vt16, ldv, w, h, part, splits, maxabs, err, s, pdl);
     return launch_product_u_tc(R, m, n, Vt16, ldv, w, h, part, splits, maxabs, err, s);
   }
   return launch_product_u(R, m, n, Vt, ldv, w, h, part, splits, s);
@@ -488,6 +494,7 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
   __half* const U16 = use_tc(w) ? B.Ut16 : nullptr;
   __half* const V16 = use_tc(w) ? B.Vt16 : nullptr;
   void* const gop = decorrelate_needs_operand(w) ? B.gop : nullptr;   // Ginv's tensor-core operand
+  const bool cinv = inverse_cluster_size(w) > 0;                       // the cluster inverse covers this width
   if (!staged) {
     KL(kStart, 2, launch_select_with(B.colpart, nrt, n, h, w, B.J, B.colE, s));
     KL(kStart, 1, launch_gather(B.R, m, n, B.J, w, B.X, m, q.st_g, s));
@@ -500,7 +507,12 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
     // V-step: V <- T([(U^T U + eps I)^-1 U^T R]^T)   (plain R even when weighted, §2.5).
     // The Gram inverse depends only on U: it runs on the side branch while the product streams R. A staged U has
     // no integer Gram yet, so its first inverse takes the Gram kernel.
-    if (w > 1) {
+    // With a cluster inverse (the TMA product, integer Gram ready) both run on the main stream: the inverse's
+    // cluster lets the product launch as soon as it is resident, and the product completes only after it.
+    const bool clusterV = w > 1 && cinv && fusedU && !(staged && it == 0) && tma_path(w, B.R, n, U16, (int)p.ldm);
+    if (clusterV) {
+      KL(kSolve, 1, launch_inverse_cluster_int(B.GintU, w, nullptr, B.Ginv, s, gop, true));
+    } else if (w > 1) {
       FORK();
       if (fusedU && !(staged && it == 0)) {
         KLS(kSolve, 1, side, launch_inverse_int(B.GintU, w, B.GrawU, B.Ginv, side, gop));
@@ -509,23 +521,30 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
         KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side, gop));
       }
     }
-    KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s));
-    if (w > 1) JOIN();
+    KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s, clusterV));
+    if (w > 1 && !clusterV) JOIN();
     TRY(targets_step(B, w > 1 ? B.Ginv : B.one, w, sv, n, q.st_n, B.Vt, (int)p.ldn, fusedV ? B.GintV : nullptr, V16,
                      p.ldn, (last && use_tc(w)) ? B.Vk16 : nullptr, s, fusedVw ? h : nullptr,
                      fusedVw ? B.Gpart : nullptr));
     // U-step: U <- T(R H V (V^T H V + eps I)^-1)
-    FORK();
-    if (fusedV) {
-      KLS(kSolve, 1, side, launch_inverse_int(B.GintV, w, B.GrawV, B.Ginv, side, gop));
-    } else if (fusedVw) {
-      KLS(kSolve, 1, side, launch_inverse(B.Gpart, 1, w, B.GrawV, B.Ginv, side, gop));
+    const bool clusterU = cinv && (fusedV || fusedVw) && tma_path(w, B.R, n, V16, (int)p.ldn);
+    if (clusterU && fusedV) {
+      KL(kSolve, 1, launch_inverse_cluster_int(B.GintV, w, B.GrawV, B.Ginv, s, gop, true));
+    } else if (clusterU) {
+      KL(kSolve, 1, launch_inverse_cluster(B.Gpart, 1, w, B.GrawV, B.Ginv, s, gop, true));
     } else {
-      KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
-      KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side, gop));
+      FORK();
+      if (fusedV) {
+        KLS(kSolve, 1, side, launch_inverse_int(B.GintV, w, B.GrawV, B.Ginv, side, gop));
+      } else if (fusedVw) {
+        KLS(kSolve, 1, side, launch_inverse(B.Gpart, 1, w, B.GrawV, B.Ginv, side, gop));
+      } else {
+        KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
+        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side, gop));
+      }
     }
-    KL(kUstep, 1, product_u(B.R, m, n, B.Vt, V16, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s));
-    JOIN();
+    KL(kUstep, 1, product_u(B.R, m, n, B.Vt, V16, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s, clusterU));
+    if (!clusterU) JOIN();
     // the next V-step's inverse (w > 1) or, after the last iteration, Eq. 4 consumes U's Gram
     // (the fp16 copy of U is not needed after the last iteration)
     TRY(targets_step(B, w > 1 ? B.Ginv : B.one, w, su, m, q.st_m, B.Ut, (int)p.ldm,
@@ -541,7 +560,9 @@ int block_scales_step(const Plan& p, const Bufs& B, int w, float* K, cudaStream_
   const int m = p.m, n = p.n;
   const int su = splits_u(w, m, n, B.R, use_tc(w) ? B.Vt16 : nullptr, (int)p.ldn);
   KL(kSolve, 1, launch_rvec(B.Ut, (int)p.ldm, w, m, B.part, su, B.r, s));
-  if (w <= 128) {
+  if (inverse_cluster_size(w) > 0) {
+    KL(kSolve, 1, launch_scales_cluster_int(B.GintU, B.GrawV, B.r, w, B.d, s, K));
+  } else if (w <= 128) {
     KL(kSolve, 1, launch_scales_int(B.GintU, B.GrawV, B.r, w, B.d, s, K));
   } else {
     KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));

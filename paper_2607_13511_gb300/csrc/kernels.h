@@ -215,10 +215,13 @@ void tc_split(int w, int Lx, int Ly, int* splits, int* chunk);
 bool tma_product_ok(const float* R, int n, const __half* T, int ldt);
 // Partial slots the TMA-fed product writes (its classic split count, or more under its stream plan).
 int tma_product_slots(int w, int Lx, int Ly);
+// pdl: launched with programmatic stream serialization behind a cluster inverse (launch_inverse_cluster*), which
+// lets it start once the inverse's CTAs are resident; it completes only after the inverse has.
 cudaError_t launch_product_v_tma(const float* R, int m, int n, const __half* Ut, int ldu, int w, float* part,
-                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s);
+                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s, bool pdl = false);
 cudaError_t launch_product_u_tma(const float* R, int m, int n, const __half* Vt, int ldv, int w, const float* h,
-                                 float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s);
+                                 float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s,
+                                 bool pdl = false);
 // ---- packed inference (packed.cu, §2.6): 2-bit codes in tensor-core fragment order (packed_words(rows, cols)
 // 32-bit words; layout in packed.cu) and the row product out[r] = scale[r] * sum_j T[r][j] v[j] (scale optional)
 // with the vector given as B fragments (fragment_words(cols) words, from launch_fragments). With zf the product also
@@ -289,6 +292,16 @@ cudaError_t launch_inverse(const float* Gpart, int splits, int w, float* Graw, f
                            void* op = nullptr);
 // Same from an integer upper-triangle Gram (as written by launch_apply), which is reset to zero after reading.
 cudaError_t launch_inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s, void* op = nullptr);
+// The same inverses on a thread-block cluster of inverse_cluster_size(w) CTAs (0: not available for this width),
+// which distributed shared memory connects; with pdl the next kernel on the stream may launch as soon as the
+// cluster is resident (it must not read Ginv before its griddepcontrol.wait).
+int inverse_cluster_size(int w);
+cudaError_t launch_inverse_cluster(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s,
+                                   void* op, bool pdl);
+cudaError_t launch_inverse_cluster_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s, void* op, bool pdl);
+// Eq. 4 on the cluster (launch_scales_int).
+cudaError_t launch_scales_cluster_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s,
+                                      float* K = nullptr);
 // r[a] = sum_y Ut[a][y] * sum_s part[s][a][y]
 cudaError_t launch_rvec(const int8_t* Ut, int ldu, int w, int L, const float* part, int splits, float* r,
                         cudaStream_t s);

@@ -27,6 +27,8 @@
 // next tile's last unit, so the MMAs keep going.
 #include <cuda.h>
 
+#include <algorithm>
+
 #include "kernels.h"
 #include "umma.cuh"
 
@@ -34,10 +36,12 @@ namespace externd {
 
 namespace {
 
-constexpr int kConvWarps = 8;
+constexpr int kConvWarps = 16;
 constexpr int kConv = kConvWarps * 32;
-constexpr int kProducerWarp = kConvWarps, kMmaWarp = kConvWarps + 1;
-constexpr int kThreads = (kConvWarps + 2) * 32;
+constexpr int kItems = 128 * 8 / kConv;   // (position, 8-deep K chunk) items per converter thread and stage
+static_assert(kConv % 128 == 0 && kItems >= 1, "a converter thread keeps one position");
+constexpr int kProducerWarp = kConvWarps, kMmaWarp = kConvWarps + 1, kBWarp = kConvWarps + 2;
+constexpr int kThreads = (kConvWarps + 3) * 32;
 constexpr int kStageK = 64;
 constexpr uint32_t kTileA = 128u * 128u;      // 128 rows x 64 fp16
 constexpr uint32_t kStage32 = 128u * 64u * 4u;   // float32 R tile of one stage
@@ -115,12 +119,23 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
   }
   const int nk = (int)(u1 > u0 ? u1 - u0 : 0);
 
-  float mx = __ldg(p.maxabs);
-  if (USTEP && p.h != nullptr) mx *= __ldg(p.maxabs + 1);
-  int ex = 0;
-  if (mx > 0.f && mx <= 3.0e38f) frexpf(mx, &ex);
-  const int sexp = max(-100, min(100, 14 - ex));
-  const float scale = ldexpf(1.f, sexp), inv_scale = ldexpf(1.f, -sexp);
+  // the power-of-two scale of the fp16 split: read by the converters once the roles split, so that the first
+  // copies do not wait for this load
+  float scale = 1.f, inv_scale = 1.f;
+  auto load_scale = [&]() {
+    float mx = __ldg(p.maxabs);
+    if (USTEP && p.h != nullptr) mx *= __ldg(p.maxabs + 1);
+    int ex = 0;
+    if (mx > 0.f && mx <= 3.0e38f) frexpf(mx, &ex);
+    const int sexp = max(-100, min(100, 14 - ex));
+    scale = ldexpf(1.f, sexp);
+    inv_scale = ldexpf(1.f, -sexp);
+  };
+  if (warp == kProducerWarp && lane == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapR)) : "memory");
+  } else if (warp == kBWarp && lane == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapT)) : "memory");
+  }
 
   if (tid == 0) {
     for (int s = 0; s < p.s32; ++s) {
@@ -200,9 +215,9 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
     return have;
   };
   if (warp == kProducerWarp) {
-    // ------------------------------------------------------------------ TMA producer
+    // ------------------------------------------------------------------ TMA producer of R
     if (lane == 0) {
-      int k = 0, kb = 0;   // stages whose R copies / B copies were issued
+      int k = 0;   // stages whose R copies were issued
       int t = (int)(u0 / p.nkt), kc = (int)(u0 - (long long)t * p.nkt);   // advanced without divisions
       for (; k < nk; ++k) {
         if (STREAM && k > 0 && ++kc == p.nkt) {
@@ -210,7 +225,7 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
           ++t;
         }
         const int x0 = t * 128, y0 = (STREAM ? kc : kc + k) * kStageK;   // a classic run stays in its tile
-        const int s = k % p.s32, sb = k % p.sb;
+        const int s = k % p.s32;
         if (k >= p.s32 && !mbar_wait(empty32 + 8u * s, (uint32_t)(k / p.s32 - 1) & 1u, p.err)) break;
         mbar_expect_tx(full32 + 8u * s, kStage32);
         if (!USTEP) {
@@ -220,17 +235,25 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
 #pragma unroll
           for (int b = 0; b < 2; ++b) tma_load_2d(r32 + s * kStage32 + b * 16384u, &mapR, y0 + 32 * b, x0, full32 + 8u * s);
         }
-        if (k >= p.sb && !mbar_wait(emptyB + 8u * sb, (uint32_t)(k / p.sb - 1) & 1u, p.err)) {
-          ++k;   // stage k's R copies are in flight, its B copy is not
-          break;
-        }
-        mbar_expect_tx(fullB + 8u * sb, tileB);
-        tma_load_2d(rb + sb * tileB, &mapT, y0, 0, fullB + 8u * sb);
-        kb = k + 1;
       }
       // every copy this thread issued lands before the CTA can exit (bounded waits)
       for (int j = max(0, k - p.s32); j < k; ++j) mbar_wait(full32 + 8u * (j % p.s32), (uint32_t)(j / p.s32) & 1u, p.err);
-      for (int j = max(0, kb - p.sb); j < kb; ++j) mbar_wait(fullB + 8u * (j % p.sb), (uint32_t)(j / p.sb) & 1u, p.err);
+    }
+  } else if (warp == kBWarp) {
+    // ------------------------------------------------------------------ TMA producer of the ternary operand
+    // (its own thread, so that a B slot still held by the MMAs never holds up the next R copies)
+    if (lane == 0) {
+      int k = 0;
+      int kc = (int)(u0 % p.nkt);
+      for (; k < nk; ++k) {
+        if (STREAM && k > 0 && ++kc == p.nkt) kc = 0;
+        const int y0 = (STREAM ? kc : kc + k) * kStageK;
+        const int sb = k % p.sb;
+        if (k >= p.sb && !mbar_wait(emptyB + 8u * sb, (uint32_t)(k / p.sb - 1) & 1u, p.err)) break;
+        mbar_expect_tx(fullB + 8u * sb, tileB);
+        tma_load_2d(rb + sb * tileB, &mapT, y0, 0, fullB + 8u * sb);
+      }
+      for (int j = max(0, k - p.sb); j < k; ++j) mbar_wait(fullB + 8u * (j % p.sb), (uint32_t)(j / p.sb) & 1u, p.err);
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------------ MMA issuer
@@ -272,7 +295,17 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
     }
   } else {
     // ------------------------------------------------------------------ converters (and the epilogues)
-    // item i = tid + 256 q (q < 4): A row x = i % 128 (lanes on consecutive rows), K chunk o = i / 128
+    load_scale();
+    // item i = tid + kConv q (q < kItems): A row x = i % 128 = tid % 128 (lanes on consecutive rows, the same
+    // position for every item of a thread), K chunk o = i / 128
+    const int x = tid & 127, o0 = tid >> 7;
+    // V-step: float x of rows 8o + j sits at (8o + j) * 128 + (((x % 32) / 4 ^ j) * 16) + (x % 4) * 4 in box x / 32
+    // (the 128-byte swizzle; 8o is a multiple of 8), the same offsets for every stage
+    uint32_t voff[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      voff[j] = (uint32_t)(x >> 5) * 8192u + (uint32_t)j * 128u + ((((uint32_t)(x & 31) >> 2) ^ (uint32_t)j) << 4) +
+                ((uint32_t)(x & 3) << 2);
     int prev_tile = -1;
     int t = (int)(u0 / p.nkt), kc = (int)(u0 - (long long)t * p.nkt);   // advanced without divisions
     for (int k = 0; k < nk && ok; ++k) {
@@ -286,44 +319,57 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
         seg_tile = t;
       }
       const int s = k % p.s32, s16 = k % p.s16;
-      const bool got = mbar_wait(full32 + 8u * s, (uint32_t)(k / p.s32) & 1u, p.err) &&
-                       (k < p.s16 || mbar_wait(empty16 + 8u * s16, (uint32_t)(k / p.s16 - 1) & 1u, p.err));
+      bool got = mbar_wait(full32 + 8u * s, (uint32_t)(k / p.s32) & 1u, p.err);
       ok = __all_sync(0xffffffffu, got) != 0;
       if (!ok) break;
+      // read the stage into registers and hand its slot back to the producer at once (the split below then
+      // overlaps the next copies), then wait for the A slot the split writes into
       const uint8_t* st = gbase + (r32 - sbase) + (size_t)s * kStage32;
-      uint8_t* a_hi = gbase + (ra - sbase) + (size_t)s16 * 2u * kTileA;
-      uint8_t* a_lo = a_hi + kTileA;
       const int y0 = (STREAM ? kc : kc + k) * kStageK;
+      float v[kItems][8];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int i = tid + kConv * q;
-        const int x = i & 127, o = i >> 7;
-        const int valid = Ly - (y0 + 8 * o);   // elements of this chunk inside R
-        float v[8];
+      for (int q = 0; q < kItems; ++q) {
+        const int o = o0 + (kConv / 128) * q;
         if (!USTEP) {
-          // R[y0 + 8o + j][x0 + x]: box x / 32, row 8o + j, float x % 32
-          const uint8_t* bx = st + (x >> 5) * 8192;
+          const uint8_t* bx = st + o * 1024;
 #pragma unroll
-          for (int j = 0; j < 8; ++j) v[j] = *reinterpret_cast<const float*>(bx + sw128_f32(8 * o + j, x & 31));
+          for (int j = 0; j < 8; ++j) v[q][j] = *reinterpret_cast<const float*>(bx + voff[j]);
         } else {
           // R[x0 + x][y0 + 8o .. +7]: box o / 4, row x, floats 8 (o % 4) .. +7 (two 16-byte chunks)
           const uint8_t* bx = st + (o >> 2) * 16384;
           const float4 a = *reinterpret_cast<const float4*>(bx + sw128_f32(x, 8 * (o & 3)));
           const float4 b = *reinterpret_cast<const float4*>(bx + sw128_f32(x, 8 * (o & 3) + 4));
-          v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-          v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-          if (p.h != nullptr) {
-            const int c = y0 + 8 * o;
+          v[q][0] = a.x; v[q][1] = a.y; v[q][2] = a.z; v[q][3] = a.w;
+          v[q][4] = b.x; v[q][5] = b.y; v[q][6] = b.z; v[q][7] = b.w;
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty32 + 8u * s);
+      got = k < p.s16 || mbar_wait(empty16 + 8u * s16, (uint32_t)(k / p.s16 - 1) & 1u, p.err);
+      ok = __all_sync(0xffffffffu, got) != 0;
+      if (!ok) break;
+      uint8_t* a_hi = gbase + (ra - sbase) + (size_t)s16 * 2u * kTileA;
+      uint8_t* a_lo = a_hi + kTileA;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) v[j] *= (c + j < Ly) ? __ldg(p.h + c + j) : 0.f;
-          }
+      for (int q = 0; q < kItems; ++q) {
+        const int o = o0 + (kConv / 128) * q;
+        const int valid = Ly - (y0 + 8 * o);   // elements of this chunk inside R
+        if (USTEP && p.h != nullptr) {
+          const int c = y0 + 8 * o;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) v[q][j] *= (c + j < Ly) ? __ldg(p.h + c + j) : 0.f;
         }
         uint32_t hi[4], lo[4];
+        if (valid >= 8) {
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float x0v = 2 * e < valid ? v[2 * e] * scale : 0.f;
-          const float x1v = 2 * e + 1 < valid ? v[2 * e + 1] * scale : 0.f;
-          split_pair(x0v, x1v, hi[e], lo[e]);
+          for (int e = 0; e < 4; ++e) split_pair(v[q][2 * e] * scale, v[q][2 * e + 1] * scale, hi[e], lo[e]);
+        } else {   // the last chunk of R: rows past its end enter as zeros
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float x0v = 2 * e < valid ? v[q][2 * e] * scale : 0.f;
+            const float x1v = 2 * e + 1 < valid ? v[q][2 * e + 1] * scale : 0.f;
+            split_pair(x0v, x1v, hi[e], lo[e]);
+          }
         }
         const uint32_t off = sw128_offset((uint32_t)x, (uint32_t)o);
         *reinterpret_cast<uint4*>(a_hi + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
@@ -331,10 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
       }
       fence_async_shared();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(full16 + 8u * s16);
-        mbar_arrive(empty32 + 8u * s);
-      }
+      if (lane == 0) mbar_arrive(full16 + 8u * s16);
       // the previous segment's partials, once this segment is fully converted (its MMAs are then queued)
       const bool seg_end = k == nk - 1 || kc == p.nkt - 1;
       if (STREAM && seg_end && seg >= 1) ok = epilogue(seg - 1, prev_tile);
@@ -350,6 +393,9 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
     tc_fence_after();
     tmem_dealloc(tmem, p.tmem_cols);
   }
+  // Launched early beside a w x w inverse (programmatic dependent launch): do not complete before it has, so that
+  // the kernels after this one see its result. Without such a prerequisite this returns at once.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 typedef CUresult (*EncodeTiled)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -381,11 +427,12 @@ TmaPlan tma_plan(int w) {
   t.wpad = (int)round_up(w, 16);
   const size_t tileB = (size_t)t.wpad * 128;
   t.s16 = 2;
-  const size_t budget = 227 * 1024 - 1024 - 512 - (size_t)t.s16 * 2 * kTileA;
-  int s = 4;
-  while (s > 1 && (size_t)s * kStage32 + round_up((long long)s * tileB, 1024) > budget) --s;
-  t.s32 = t.sb = s;
-  t.smem = 1024 + (size_t)s * kStage32 + round_up((long long)s * tileB, 1024) + (size_t)t.s16 * 2 * kTileA + 512;
+  t.sb = 2;   // the ternary tiles come from L2: two slots keep the MMAs fed; the rest of the space holds R in flight
+  const size_t budget = 227 * 1024 - 1024 - 512 - (size_t)t.s16 * 2 * kTileA - round_up((long long)t.sb * tileB, 1024);
+  int s = 6;
+  while (s > 1 && (size_t)s * kStage32 > budget) --s;
+  t.s32 = s;
+  t.smem = 1024 + (size_t)s * kStage32 + round_up((long long)t.sb * tileB, 1024) + (size_t)t.s16 * 2 * kTileA + 512;
   return t;
 }
 
@@ -402,8 +449,9 @@ TmaWork tma_work(int w, int Lx, int Ly) {
   tc_split(w, Lx, Ly, &sp, &chunk);
   const int tiles = (int)cdiv(Lx, 128), nkt = (int)cdiv(Ly, kStageK);
   TmaWork t{0, nkt, chunk / kStageK, sp, tiles, sp, (long long)tiles * nkt};
-  const long long G = sms - 1;
-  if ((long long)tiles * sp >= sms && G >= 1 && t.U >= G) {
+  // SMs left to the product: the w x w inverse of the same half-step holds one (single CTA) or a cluster's worth
+  const long long G = sms - std::max(1, inverse_cluster_size(w));
+  if ((long long)tiles * sp > G && G >= 1 && t.U >= G) {
     int S = 0;
     for (long long tt = 0; tt < tiles; ++tt) {
       const long long a = tt * nkt, b = a + nkt - 1;
@@ -423,7 +471,7 @@ TmaWork tma_work(int w, int Lx, int Ly) {
 
 template <bool USTEP>
 cudaError_t launch_tma(const float* R, int m, int n, const __half* T, int ldt, int w, const float* h, float* part,
-                       int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
+                       int splits, const float* maxabs, unsigned* err, cudaStream_t s, bool pdl) {
   EncodeTiled enc = encoder();
   if (enc == nullptr) return cudaErrorNotSupported;
   const int Lx = USTEP ? m : n, Ly = USTEP ? n : m;
@@ -463,12 +511,18 @@ cudaError_t launch_tma(const float* R, int m, int n, const __half* T, int ldt, i
   uint32_t cols = 32;
   while ((int)cols < (wk.stream ? 2 : 1) * t.wpad) cols <<= 1;   // the stream plan alternates two accumulators
   TmaArgs a{m, n, w, t.wpad, h, part, maxabs, err, t.s32, t.sb, t.s16, cols, wk.nkt, wk.cu, wk.U, wk.slots};
-  dim3 grid((unsigned)wk.grid_x, 1, (unsigned)wk.grid_z);
-  if (wk.stream)
-    product_tma_kernel<USTEP, true><<<grid, kThreads, t.smem, s>>>(mapR, mapT, a);
-  else
-    product_tma_kernel<USTEP, false><<<grid, kThreads, t.smem, s>>>(mapR, mapT, a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)wk.grid_x, 1, (unsigned)wk.grid_z);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = t.smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // may start once the inverse is resident
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = pdl ? at : nullptr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  if (wk.stream) return cudaLaunchKernelEx(&cfg, product_tma_kernel<USTEP, true>, mapR, mapT, a);
+  return cudaLaunchKernelEx(&cfg, product_tma_kernel<USTEP, false>, mapR, mapT, a);
 }
 
 }  // namespace
@@ -481,13 +535,14 @@ bool tma_product_ok(const float* R, int n, const __half* T, int ldt) {
 int tma_product_slots(int w, int Lx, int Ly) { return tma_work(w, Lx, Ly).slots; }
 
 cudaError_t launch_product_v_tma(const float* R, int m, int n, const __half* Ut, int ldu, int w, float* part,
-                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
-  return launch_tma<false>(R, m, n, Ut, ldu, w, nullptr, part, splits, maxabs, err, s);
+                                 int splits, const float* maxabs, unsigned* err, cudaStream_t s, bool pdl) {
+  return launch_tma<false>(R, m, n, Ut, ldu, w, nullptr, part, splits, maxabs, err, s, pdl);
 }
 
 cudaError_t launch_product_u_tma(const float* R, int m, int n, const __half* Vt, int ldv, int w, const float* h,
-                                 float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s) {
-  return launch_tma<true>(R, m, n, Vt, ldv, w, h, part, splits, maxabs, err, s);
+                                 float* part, int splits, const float* maxabs, unsigned* err, cudaStream_t s,
+                                 bool pdl) {
+  return launch_tma<true>(R, m, n, Vt, ldv, w, h, part, splits, maxabs, err, s, pdl);
 }
 
 }  // namespace externd

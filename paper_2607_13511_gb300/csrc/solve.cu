@@ -6,12 +6,19 @@
 // on an SPD matrix, no pivoting needed): one 1024-thread CTA holds the w x w matrix in registers, one row per
 // 1024/W_PAD threads, and sweeps the w pivots with one barrier per pivot. Sweeping every pivot of S = G turns S
 // into -G^-1.
+#include <cooperative_groups.h>
+
+#include <cstdlib>
+#include <cstring>
+
 #include "kernels.h"
 #include "umma.cuh"
 
 namespace externd {
 
 namespace {
+
+namespace cg = cooperative_groups;
 
 constexpr int GT = 32;     // Gram tile (a, b)
 constexpr int GY = 64;     // Gram depth slice
@@ -701,6 +708,796 @@ __global__ void __launch_bounds__(544) sweep32_kernel(const float* __restrict__ 
 
 }
 
+// Register-tiled sweep for w <= 128 on one CTA: RG x CG tile threads hold the WP x WP matrix as TR x TC
+// register tiles (8 x 4 over 16 warps at WP = 128, 4 x 2 over 16 warps at 64, 2 x 2 over 8 warps at 32), one
+// row group per warp at WP >= 64, so every shared-memory read of a pivot row is a broadcast and every read of a
+// W row covers contiguous bytes; one more warp inverts the next pivot block ahead. Thread t owns the rows
+// TR * (t / CG) + a and the columns TC * (t % CG) + c. With the published rows Rk = S[K,:] of pivot block K and
+// Q = S[K,K]^-1 (both ready at the start of a step):
+//   A. W = Q Rk (NB x WP) into shared memory; the owners of the next block K+ also save S[K+,K+]      barrier
+//   B. rows outside K: S[i,j] -= sum_d Rk[d][i] W[d][j] (S[i,K] = Rk[.,i] by symmetry; fma chains in d
+//      order on the paired FMA), then the columns of K take S[i,K] Q = W[.,i]; rows of K become
+//      Q S[K,J] = W[.,J] and -Q on the pivot block; the owners of K+ publish their updated rows.
+//      Pivot warp, meanwhile: the updated S[K+,K+] from the saved block with the same fma chains, and its
+//      inverse (warp_sweep)                                                                              barrier
+// Every S stays symmetric; after the last block S = -(G + eps I)^-1. About w^3 FMAs in all. The pivot warp's
+// shuffles and loads issue between the tile warps' paired FMAs, which keep the FMA pipes busy.
+template <int WP>
+struct InvShape {
+  static constexpr int NB = WP >= 64 ? 16 : 8;   // pivot block
+  static constexpr int TR = WP == 128 ? 8 : WP == 64 ? 4 : 2;
+  static constexpr int TC = WP == 128 ? 4 : 2;
+  static constexpr int RG = WP / TR, CG = WP / TC, NT = RG * CG;   // row groups, column groups, tile threads
+};
+
+template <int WP>
+constexpr int inv_threads() { return InvShape<WP>::NT + 32; }
+
+template <int WP, int MODE, bool IN_INT>
+__global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float* __restrict__ Gpart, int splits,
+                                                                   int w, const float* __restrict__ GVraw,
+                                                                   const float* __restrict__ r,
+                                                                   float* __restrict__ Graw, float* __restrict__ out,
+                                                                   int* Gint, uint8_t* __restrict__ op) {
+  using SH = InvShape<WP>;
+  constexpr int NB = SH::NB, TR = SH::TR, TC = SH::TC, CG = SH::CG, NT = SH::NT, NW = NT / 32;
+  constexpr int EPL = NB * NB / 32, LPR = NB / EPL;
+  static_assert(TR % 2 == 0 && TC % 2 == 0 && (TC == 2 || TC == 4) && NT % 32 == 0, "tile shape");
+  static_assert(NB % (TR * (32 / CG)) == 0, "a warp's rows lie in one pivot block");
+  __shared__ __align__(16) float Rk[2][NB][WP];   // published rows of the pivot block (two buffers)
+  __shared__ __align__(16) float Ws[NB][WP];      // W = Q Rk of the step
+  __shared__ __align__(16) float Qs[2][NB][NB];   // pivot-block inverses (two buffers)
+  __shared__ __align__(16) float Pn[NB][NB];      // next pivot block before this step's update
+  __shared__ float red[NW + 1];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const bool tile = tid < NT;
+  const int tr = tile ? tid / CG : 0, tc = tid % CG, i0 = tr * TR, jb = tc * TC;
+  const bool vec = (w & 3) == 0;   // rows of every w x w input and output start on 16-byte boundaries
+  // a run (i, jb .. jb + TC - 1) of a w x w matrix: one vector access where it is aligned and inside
+  const bool run_in = vec && jb + TC <= w;
+
+  float S[TR][TC];
+#pragma unroll
+  for (int a = 0; a < TR; ++a)
+#pragma unroll
+    for (int c = 0; c < TC; ++c) S[a][c] = 0.f;
+  if (IN_INT && tile) {
+    // The run of TC columns lies wholly above the diagonal (read along the rows), wholly below it (read the
+    // mirrored entries along the columns, where rows i0 .. i0 + TR - 1 are contiguous) or straddles it (entry by
+    // entry); every load is issued before the first use.
+    int g[TR][TC];
+    const bool upper = i0 + TR - 1 <= jb, lower = i0 > jb + TC - 1;
+    if (upper && run_in) {
+#pragma unroll
+      for (int a = 0; a < TR; ++a) {
+        const int* src = Gint + (long long)(i0 + a) * w + jb;
+        if (i0 + a >= w) {
+#pragma unroll
+          for (int c = 0; c < TC; ++c) g[a][c] = 0;
+        } else if constexpr (TC == 4) {
+          const int4 t = *reinterpret_cast<const int4*>(src);
+          g[a][0] = t.x; g[a][1] = t.y; g[a][2] = t.z; g[a][3] = t.w;
+        } else {
+          const int2 t = *reinterpret_cast<const int2*>(src);
+          g[a][0] = t.x; g[a][1] = t.y;
+        }
+      }
+    } else if (lower && vec && i0 + TR <= w) {
+#pragma unroll
+      for (int c = 0; c < TC; ++c) {
+        const int* src = Gint + (long long)(jb + c) * w + i0;
+        if (jb + c >= w) {
+#pragma unroll
+          for (int a = 0; a < TR; ++a) g[a][c] = 0;
+        } else if constexpr (TR % 4 == 0) {
+#pragma unroll
+          for (int a = 0; a < TR; a += 4) {
+            const int4 t = *reinterpret_cast<const int4*>(src + a);
+            g[a][c] = t.x; g[a + 1][c] = t.y; g[a + 2][c] = t.z; g[a + 3][c] = t.w;
+          }
+        } else {
+#pragma unroll
+          for (int a = 0; a < TR; a += 2) {
+            const int2 t = *reinterpret_cast<const int2*>(src + a);
+            g[a][c] = t.x; g[a + 1][c] = t.y;
+          }
+        }
+      }
+    } else {
+#pragma unroll
+      for (int a = 0; a < TR; ++a)
+#pragma unroll
+        for (int c = 0; c < TC; ++c) {
+          const int i = i0 + a, j = jb + c;
+          g[a][c] = (i < w && j < w) ? Gint[(long long)min(i, j) * w + max(i, j)] : 0;
+        }
+    }
+#pragma unroll
+    for (int a = 0; a < TR; ++a)
+#pragma unroll
+      for (int c = 0; c < TC; ++c) S[a][c] = (float)g[a][c];
+  } else if (tile) {
+    for (int sp = 0; sp < splits; ++sp) {
+      const float* G = Gpart + (long long)sp * w * w;
+#pragma unroll
+      for (int a = 0; a < TR; ++a)
+#pragma unroll
+        for (int c = 0; c < TC; ++c) {
+          const int i = i0 + a, j = jb + c;
+          if (i < w && j < w) S[a][c] += G[(long long)i * w + j];
+        }
+    }
+  }
+  // loads / stores of the thread's run of row i in a w x w float matrix
+  auto load_run = [&](const float* M, int i, float (&v)[TC]) {
+    const float* src = M + (long long)i * w + jb;
+    if (i < w && run_in) {
+      if constexpr (TC == 4) {
+        const float4 t = *reinterpret_cast<const float4*>(src);
+        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+      } else {
+        const float2 t = *reinterpret_cast<const float2*>(src);
+        v[0] = t.x; v[1] = t.y;
+      }
+    } else {
+#pragma unroll
+      for (int c = 0; c < TC; ++c) v[c] = (i < w && jb + c < w) ? src[c] : 0.f;
+    }
+  };
+  auto store_run = [&](float* M, int i, const float (&v)[TC]) {
+    float* dst = M + (long long)i * w + jb;
+    if (i < w && run_in) {
+      if constexpr (TC == 4) *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
+      else *reinterpret_cast<float2*>(dst) = make_float2(v[0], v[1]);
+    } else {
+#pragma unroll
+      for (int c = 0; c < TC; ++c)
+        if (i < w && jb + c < w) dst[c] = v[c];
+    }
+  };
+  float diag = 0.f;
+  if (tile) {
+    if (MODE == 1) {   // K = G_U .* G_V
+      float gv[TR][TC];
+#pragma unroll
+      for (int a = 0; a < TR; ++a) load_run(GVraw, i0 + a, gv[a]);
+#pragma unroll
+      for (int a = 0; a < TR; ++a)
+#pragma unroll
+        for (int c = 0; c < TC; ++c) S[a][c] *= gv[a][c];
+    }
+#pragma unroll
+    for (int a = 0; a < TR; ++a)
+#pragma unroll
+      for (int c = 0; c < TC; ++c) {
+        const int i = i0 + a, j = jb + c;
+        if (i < w && j < w) {
+          if (i == j) diag += S[a][c];
+        } else {
+          S[a][c] = (i == j) ? 1.f : 0.f;   // identity on the padding
+        }
+      }
+    if (Graw != nullptr) {   // the Gram (MODE 0) or K (MODE 1) before the ridge
+#pragma unroll
+      for (int a = 0; a < TR; ++a) store_run(Graw, i0 + a, S[a]);
+    }
+  }
+  diag = warp_sum(diag);
+  if (lane == 0) red[warp] = diag;
+  __syncthreads();
+  float trace = 0.f;
+#pragma unroll
+  for (int q = 0; q < NW; ++q) trace += red[q];
+  const float eps = ((MODE == 0) || (w > 1)) ? (float)kEpsRel * trace / (float)w : 0.f;
+  if (tile) {
+#pragma unroll
+    for (int a = 0; a < TR; ++a)
+#pragma unroll
+      for (int c = 0; c < TC; ++c)
+        if (i0 + a < w && i0 + a == jb + c) S[a][c] += eps;
+  }
+
+  auto publish_rows = [&](int kb, int buf) {   // rows [kb, kb + NB) of the register tiles into Rk[buf]
+    if (i0 >= kb && i0 < kb + NB) {
+#pragma unroll
+      for (int a = 0; a < TR; ++a) {
+        if constexpr (TC == 4)
+          *reinterpret_cast<float4*>(&Rk[buf][i0 + a - kb][jb]) = make_float4(S[a][0], S[a][1], S[a][2], S[a][3]);
+        else
+          *reinterpret_cast<float2*>(&Rk[buf][i0 + a - kb][jb]) = make_float2(S[a][0], S[a][1]);
+      }
+    }
+  };
+  const int pr = lane / LPR, pc = (lane % LPR) * EPL;   // pivot warp: its entries of an NB x NB block
+  if (tile) publish_rows(0, 0);
+  __syncthreads();
+  if (!tile) {
+    float A[EPL];
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) A[e] = Rk[0][pr][pc + e];
+    warp_sweep<NB>(A, lane);
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) Qs[0][pr][pc + e] = -A[e];
+  }
+  __syncthreads();
+
+  for (int k0 = 0, step = 0; k0 < w; k0 += NB, ++step) {
+    const int cur = step & 1, nxt = cur ^ 1, kn = k0 + NB;
+    const bool has_next = kn < w;
+    const bool rowsK = i0 >= k0 && i0 < k0 + NB;          // warp-uniform: a warp's rows lie in one block
+    const bool rowsN = has_next && i0 >= kn && i0 < kn + NB;
+    const bool colsK = jb + TC > k0 && jb < k0 + NB;      // TC divides NB: a run is wholly in or out of K
+    // A. W = Q Rk; the next pivot block as it stands
+    if (tile) {
+      for (int idx = tid; idx < NB * (WP / 4); idx += NT) {
+        const int c = idx / (WP / 4), q = (idx % (WP / 4)) * 4;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int d = 0; d < NB; ++d) {
+          const float qv = Qs[cur][c][d];
+          const float4 rv = *reinterpret_cast<const float4*>(&Rk[cur][d][q]);
+          acc.x = fmaf(qv, rv.x, acc.x);
+          acc.y = fmaf(qv, rv.y, acc.y);
+          acc.z = fmaf(qv, rv.z, acc.z);
+          acc.w = fmaf(qv, rv.w, acc.w);
+        }
+        *reinterpret_cast<float4*>(&Ws[c][q]) = acc;
+      }
+      if (rowsN && jb >= kn && jb < kn + NB) {
+#pragma unroll
+        for (int a = 0; a < TR; ++a)
+#pragma unroll
+          for (int c = 0; c < TC; ++c) Pn[i0 + a - kn][jb + c - kn] = S[a][c];
+      }
+    }
+    __syncthreads();
+    // B. the update (tile warps) beside the next pivot block's inverse (pivot warp)
+    if (tile) {
+      if (rowsK) {
+        if (colsK) {
+#pragma unroll
+          for (int a = 0; a < TR; ++a)
+#pragma unroll
+            for (int c = 0; c < TC; ++c) S[a][c] = -Qs[cur][i0 + a - k0][jb + c - k0];
+        } else {
+#pragma unroll
+          for (int a = 0; a < TR; ++a)
+#pragma unroll
+            for (int c = 0; c < TC; ++c) S[a][c] = Ws[i0 + a - k0][jb + c];
+        }
+      } else {
+#pragma unroll 4
+        for (int d = 0; d < NB; ++d) {
+          float rk[TR], wv[TC];
+#pragma unroll
+          for (int a = 0; a < TR; a += 2) {
+            const float2 t = *reinterpret_cast<const float2*>(&Rk[cur][d][i0 + a]);
+            rk[a] = t.x;
+            rk[a + 1] = t.y;
+          }
+          if constexpr (TC == 4) {
+            const float4 t = *reinterpret_cast<const float4*>(&Ws[d][jb]);
+            wv[0] = t.x; wv[1] = t.y; wv[2] = t.z; wv[3] = t.w;
+          } else {
+            const float2 t = *reinterpret_cast<const float2*>(&Ws[d][jb]);
+            wv[0] = t.x; wv[1] = t.y;
+          }
+#pragma unroll
+          for (int a = 0; a < TR; ++a)
+#pragma unroll
+            for (int c = 0; c < TC; c += 2) {   // lane-wise fma.rn, the same rounding as fmaf
+              const float2 s2 = __ffma2_rn(make_float2(-rk[a], -rk[a]), make_float2(wv[c], wv[c + 1]),
+                                           make_float2(S[a][c], S[a][c + 1]));
+              S[a][c] = s2.x;
+              S[a][c + 1] = s2.y;
+            }
+        }
+        if (colsK) {
+#pragma unroll
+          for (int c = 0; c < TC; ++c)
+#pragma unroll
+            for (int a = 0; a < TR; ++a) S[a][c] = Ws[jb + c - k0][i0 + a];
+        }
+      }
+      if (rowsN) publish_rows(kn, nxt);
+    } else if (has_next) {
+      float A[EPL];
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) A[e] = Pn[pr][pc + e];
+#pragma unroll
+      for (int d = 0; d < NB; ++d) {   // the fma chains of the tile owners, in the same order
+        const float rk = Rk[cur][d][kn + pr];
+        float wv[EPL];
+#pragma unroll
+        for (int e = 0; e < EPL; e += 2) {
+          const float2 t = *reinterpret_cast<const float2*>(&Ws[d][kn + pc + e]);
+          wv[e] = t.x;
+          wv[e + 1] = t.y;
+        }
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) A[e] = fmaf(-rk, wv[e], A[e]);
+      }
+      warp_sweep<NB>(A, lane);
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) Qs[nxt][pr][pc + e] = -A[e];
+    }
+    __syncthreads();
+  }
+
+  if (MODE == 0) {
+    if (op == nullptr) {   // Ginv in float32 (the tensor-core decorrelation reads only the operand image below)
+      if (tile) {
+#pragma unroll
+        for (int a = 0; a < TR; ++a) {
+          float v[TC];
+#pragma unroll
+          for (int c = 0; c < TC; ++c) v[c] = -S[a][c];
+          store_run(out, i0 + a, v);
+        }
+      }
+    } else if constexpr (WP == 128) {
+      // Ginv * 2^sg as hi / lo fp16 K-major operands (zero outside w x w) for the tensor-core decorrelation, with
+      // sg from the largest magnitude; sg (int) follows the two 32 KB images.
+      float mx = 0.f;
+      if (tile) {
+#pragma unroll
+        for (int a = 0; a < TR; ++a)
+#pragma unroll
+          for (int c = 0; c < TC; ++c)
+            if (i0 + a < w && jb + c < w) mx = fmaxf(mx, fabsf(S[a][c]));
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      if (lane == 0) red[warp] = mx;
+      __syncthreads();
+#pragma unroll
+      for (int q = 0; q < NW; ++q) mx = fmaxf(mx, red[q]);
+      const int sg = fp16_scale_exp(mx);
+      const float sc = ldexpf(1.f, sg);
+      if (tile) {   // the run of 4 columns (jb % 4 == 0) is 8 contiguous bytes of one row in the image
+#pragma unroll
+        for (int a = 0; a < TR; ++a) {
+          const int i = i0 + a;
+          __align__(8) __half hi[4];
+          __align__(8) __half lo[4];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) split_f16((i < w && jb + c < w) ? -S[a][c] * sc : 0.f, hi[c], lo[c]);
+          const uint32_t off = k_major_offset(128u, (uint32_t)i, (uint32_t)jb);
+          *reinterpret_cast<uint2*>(op + off) = *reinterpret_cast<const uint2*>(hi);
+          *reinterpret_cast<uint2*>(op + 2 * 16384u + off) = *reinterpret_cast<const uint2*>(lo);
+        }
+      }
+      if (tid == 0) *reinterpret_cast<int*>(op + 4 * 16384u) = sg;
+    }
+  } else if (tile) {
+    // d_i = sum_j (-S)[i][j] r_j, double-float, over the CG threads that share the row group
+    float rv[TC];
+#pragma unroll
+    for (int c = 0; c < TC; ++c) rv[c] = jb + c < w ? r[jb + c] : 0.f;
+#pragma unroll
+    for (int a = 0; a < TR; ++a) {
+      const int i = i0 + a;
+      F2 acc2;
+#pragma unroll
+      for (int c = 0; c < TC; ++c)
+        if (jb + c < w) acc2 = f2_add(acc2, -S[a][c] * rv[c]);
+#pragma unroll
+      for (int o = CG / 2; o > 0; o >>= 1) acc2 = f2_add(acc2, f2_shfl_xor(acc2, o));
+      if (tc == 0 && i < w) out[i] = acc2.hi + acc2.lo;
+    }
+  }
+  if (IN_INT) {   // every thread read the Gram before the first barrier: reset it for the next accumulation
+    const int ww = w * w;
+    if ((ww & 3) == 0) {
+      for (int idx = tid; idx < ww / 4; idx += NT + 32) reinterpret_cast<int4*>(Gint)[idx] = make_int4(0, 0, 0, 0);
+    } else {
+      for (int idx = tid; idx < ww; idx += NT + 32) Gint[idx] = 0;
+    }
+  }
+}
+
+// Cluster sweep for 16 < w <= 128: the CS = WP / 16 CTAs of one thread-block cluster each hold one pivot block's
+// 16 rows (CTA c: rows 16c .. 16c + 15) as 2 x TC register tiles; the pivot rows and inverse of each step reach
+// the other CTAs through distributed shared memory. Step s (K = the rows of CTA s):
+//   1. every CTA copies CTA s's published rows Rk = S[K,:] and Q = S[K,K]^-1 into its own shared memory
+//   2. W = Q Rk; the next owner (CTA s + 1) saves its diagonal block                                  CTA barrier
+//   3. rows outside K: S[i,j] -= sum_d Rk[d][i] W[d][j] (fma chains in d order), the columns of K take
+//      W[.,i]; CTA s's rows become W and -Q on the pivot block. Meanwhile the pivot warp of CTA s + 1 forms
+//      its updated diagonal block with the same fma chains and inverts it (warp_sweep); CTA s + 1 then
+//      publishes its rows and that inverse                                                          cluster barrier
+// The arithmetic per entry is that of inv_kernel (same operations in the same order); only the place where each
+// row lives differs. Every CTA reads only its own rows of the integer Gram's mirror image and of the outputs.
+// With pdl the CTAs let the next kernel of the stream launch as soon as they are all resident (programmatic
+// dependent launch): the residual product then runs beside them on the other SMs.
+template <int WP>
+struct InvClusterShape {
+  static constexpr int NB = 16, CS = WP / 16, TR = 2, TC = WP == 128 ? 4 : 2;
+  static constexpr int CG = WP / TC, NT = (NB / TR) * CG;   // column groups, tile threads
+};
+
+template <int WP>
+constexpr int inv_cluster_threads() { return InvClusterShape<WP>::NT + 32; }
+
+template <int WP, int MODE, bool IN_INT>
+__global__ void __launch_bounds__(InvClusterShape<WP>::NT + 32) inv_cluster_kernel(
+    const float* __restrict__ Gpart, int splits, int w, const float* __restrict__ GVraw, const float* __restrict__ r,
+    float* __restrict__ Graw, float* __restrict__ out, int* Gint, uint8_t* __restrict__ op, int pdl) {
+  using SH = InvClusterShape<WP>;
+  constexpr int NB = SH::NB, CS = SH::CS, TR = SH::TR, TC = SH::TC, CG = SH::CG, NT = SH::NT, NW = NT / 32;
+  constexpr int EPL = NB * NB / 32, LPR = NB / EPL;
+  static_assert(TC == 2 || TC == 4, "tile shape");
+  __shared__ __align__(16) float pubR[NB][WP];   // this CTA's rows when it owns the step's pivot block
+  __shared__ __align__(16) float pubQ[NB][NB];   // and the pivot block's inverse
+  __shared__ __align__(16) float Rk[NB][WP];     // the step's pivot rows (copied from their owner)
+  __shared__ __align__(16) float Qk[NB][NB];
+  __shared__ __align__(16) float Ws[NB][WP];     // W = Q Rk
+  __shared__ __align__(16) float Pn[NB][NB];     // own diagonal block before the update (next owner)
+  __shared__ float red[NW + 1];
+  __shared__ float cpart[2];                     // this CTA's trace part / max |Ginv| (read by the cluster)
+  cg::cluster_group cluster = cg::this_cluster();
+  const int c = (int)cluster.block_rank();
+  if (pdl) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const bool tile = tid < NT;
+  const int tr = tile ? tid / CG : 0, tc = tid % CG;
+  const int lr0 = tr * TR, i0 = NB * c + lr0, jb = tc * TC;
+  const bool vec = (w & 3) == 0;
+  const bool run_in = vec && jb + TC <= w;
+
+  float S[TR][TC];
+#pragma unroll
+  for (int a = 0; a < TR; ++a)
+#pragma unroll
+    for (int q = 0; q < TC; ++q) S[a][q] = 0.f;
+  if (IN_INT && tile) {
+    int g[TR][TC];
+    const bool upper = i0 + TR - 1 <= jb, lower = i0 > jb + TC - 1;
+    if (upper && run_in) {
+#pragma unroll
+      for (int a = 0; a < TR; ++a) {
+        const int* src = Gint + (long long)(i0 + a) * w + jb;
+        if (i0 + a >= w) {
+#pragma unroll
+          for (int q = 0; q < TC; ++q) g[a][q] = 0;
+        } else if constexpr (TC == 4) {
+          const int4 t = *reinterpret_cast<const int4*>(src);
+          g[a][0] = t.x; g[a][1] = t.y; g[a][2] = t.z; g[a][3] = t.w;
+        } else {
+          const int2 t = *reinterpret_cast<const int2*>(src);
+          g[a][0] = t.x; g[a][1] = t.y;
+        }
+      }
+    } else if (lower && vec && i0 + TR <= w) {
+#pragma unroll
+      for (int q = 0; q < TC; ++q) {
+        if (jb + q >= w) {
+          g[0][q] = g[1][q] = 0;
+        } else {
+          const int2 t = *reinterpret_cast<const int2*>(Gint + (long long)(jb + q) * w + i0);
+          g[0][q] = t.x;
+          g[1][q] = t.y;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int a = 0; a < TR; ++a)
+#pragma unroll
+        for (int q = 0; q < TC; ++q) {
+          const int i = i0 + a, j = jb + q;
+          g[a][q] = (i < w && j < w) ? Gint[(long long)min(i, j) * w + max(i, j)] : 0;
+        }
+    }
+#pragma unroll
+    for (int a = 0; a < TR; ++a)
+#pragma unroll
+      for (int q = 0; q < TC; ++q) S[a][q] = (float)g[a][q];
+  } else if (tile) {
+    for (int sp = 0; sp < splits; ++sp) {
+      const float* G = Gpart + (long long)sp * w * w;
+#pragma unroll
+      for (int a = 0; a < TR; ++a)
+#pragma unroll
+        for (int q = 0; q < TC; ++q) {
+          const int i = i0 + a, j = jb + q;
+          if (i < w && j < w) S[a][q] += G[(long long)i * w + j];
+        }
+    }
+  }
+  auto load_run = [&](const float* M, int i, float (&v)[TC]) {
+    const float* src = M + (long long)i * w + jb;
+    if (i < w && run_in) {
+      if constexpr (TC == 4) {
+        const float4 t = *reinterpret_cast<const float4*>(src);
+        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+      } else {
+        const float2 t = *reinterpret_cast<const float2*>(src);
+        v[0] = t.x; v[1] = t.y;
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < TC; ++q) v[q] = (i < w && jb + q < w) ? src[q] : 0.f;
+    }
+  };
+  auto store_run = [&](float* M, int i, const float (&v)[TC]) {
+    float* dst = M + (long long)i * w + jb;
+    if (i < w && run_in) {
+      if constexpr (TC == 4) *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
+      else *reinterpret_cast<float2*>(dst) = make_float2(v[0], v[1]);
+    } else {
+#pragma unroll
+      for (int q = 0; q < TC; ++q)
+        if (i < w && jb + q < w) dst[q] = v[q];
+    }
+  };
+  float diag = 0.f;
+  if (tile) {
+    if (MODE == 1) {   // K = G_U .* G_V
+      float gv[TR][TC];
+#pragma unroll
+      for (int a = 0; a < TR; ++a) load_run(GVraw, i0 + a, gv[a]);
+#pragma unroll
+      for (int a = 0; a < TR; ++a)
+#pragma unroll
+        for (int q = 0; q < TC; ++q) S[a][q] *= gv[a][q];
+    }
+#pragma unroll
+    for (int a = 0; a < TR; ++a)
+#pragma unroll
+      for (int q = 0; q < TC; ++q) {
+        const int i = i0 + a, j = jb + q;
+        if (i < w && j < w) {
+          if (i == j) diag += S[a][q];
+        } else {
+          S[a][q] = (i == j) ? 1.f : 0.f;   // identity on the padding
+        }
+      }
+    if (Graw != nullptr) {
+#pragma unroll
+      for (int a = 0; a < TR; ++a) store_run(Graw, i0 + a, S[a]);
+    }
+  }
+  diag = warp_sum(diag);
+  if (lane == 0) red[warp] = diag;
+  __syncthreads();
+  if (tid == 0) {
+    float t = 0.f;
+#pragma unroll
+    for (int q = 0; q < NW; ++q) t += red[q];
+    cpart[0] = t;
+  }
+  cluster.sync();
+  float trace = 0.f;
+#pragma unroll
+  for (int q = 0; q < CS; ++q) trace += *cluster.map_shared_rank(&cpart[0], q);   // the same order everywhere
+  const float eps = ((MODE == 0) || (w > 1)) ? (float)kEpsRel * trace / (float)w : 0.f;
+  if (tile) {
+#pragma unroll
+    for (int a = 0; a < TR; ++a)
+#pragma unroll
+      for (int q = 0; q < TC; ++q)
+        if (i0 + a < w && i0 + a == jb + q) S[a][q] += eps;
+  }
+  auto publish_rows = [&]() {
+#pragma unroll
+    for (int a = 0; a < TR; ++a) {
+      if constexpr (TC == 4)
+        *reinterpret_cast<float4*>(&pubR[lr0 + a][jb]) = make_float4(S[a][0], S[a][1], S[a][2], S[a][3]);
+      else
+        *reinterpret_cast<float2*>(&pubR[lr0 + a][jb]) = make_float2(S[a][0], S[a][1]);
+    }
+  };
+  const int pr = lane / LPR, pc = (lane % LPR) * EPL;   // pivot warp: its entries of the 16 x 16 block
+  const bool diagK = jb >= NB * c && jb < NB * c + NB;    // this thread's run lies in the own diagonal block
+  if (c == 0) {
+    if (tile) {
+      publish_rows();
+      if (diagK) {
+#pragma unroll
+        for (int a = 0; a < TR; ++a)
+#pragma unroll
+          for (int q = 0; q < TC; ++q) Pn[lr0 + a][jb + q] = S[a][q];
+      }
+    }
+    __syncthreads();
+    if (!tile) {
+      float A[EPL];
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) A[e] = Pn[pr][pc + e];
+      warp_sweep<NB>(A, lane);
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) pubQ[pr][pc + e] = -A[e];
+    }
+  }
+  cluster.sync();
+
+  const int nsteps = (int)cdiv(w, NB);
+  for (int s = 0; s < nsteps; ++s) {
+    const int k0 = NB * s, kn = k0 + NB;
+    const bool owner = c == s, next = c == s + 1 && s + 1 < nsteps;
+    const bool colsK = jb >= k0 && jb < k0 + NB;
+    // 1. the step's pivot rows and inverse from their owner
+    {
+      const float4* srcR = reinterpret_cast<const float4*>(cluster.map_shared_rank(&pubR[0][0], s));
+      const float4* srcQ = reinterpret_cast<const float4*>(cluster.map_shared_rank(&pubQ[0][0], s));
+      for (int idx = tid; idx < NB * WP / 4 + NB * NB / 4; idx += NT + 32) {
+        if (idx < NB * WP / 4) reinterpret_cast<float4*>(&Rk[0][0])[idx] = srcR[idx];
+        else reinterpret_cast<float4*>(&Qk[0][0])[idx - NB * WP / 4] = srcQ[idx - NB * WP / 4];
+      }
+    }
+    __syncthreads();
+    // 2. W = Q Rk; the next owner's diagonal block as it stands
+    if (tile) {
+      for (int idx = tid; idx < NB * (WP / 4); idx += NT) {
+        const int cc = idx / (WP / 4), q4 = (idx % (WP / 4)) * 4;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int d = 0; d < NB; ++d) {
+          const float qv = Qk[cc][d];
+          const float4 rv = *reinterpret_cast<const float4*>(&Rk[d][q4]);
+          acc.x = fmaf(qv, rv.x, acc.x);
+          acc.y = fmaf(qv, rv.y, acc.y);
+          acc.z = fmaf(qv, rv.z, acc.z);
+          acc.w = fmaf(qv, rv.w, acc.w);
+        }
+        *reinterpret_cast<float4*>(&Ws[cc][q4]) = acc;
+      }
+      if (next && diagK) {
+#pragma unroll
+        for (int a = 0; a < TR; ++a)
+#pragma unroll
+          for (int q = 0; q < TC; ++q) Pn[lr0 + a][jb + q - kn] = S[a][q];
+      }
+    }
+    __syncthreads();
+    // 3. the update beside the next pivot block's inverse
+    if (tile) {
+      if (owner) {
+        if (colsK) {
+#pragma unroll
+          for (int a = 0; a < TR; ++a)
+#pragma unroll
+            for (int q = 0; q < TC; ++q) S[a][q] = -Qk[lr0 + a][jb + q - k0];
+        } else {
+#pragma unroll
+          for (int a = 0; a < TR; ++a)
+#pragma unroll
+            for (int q = 0; q < TC; ++q) S[a][q] = Ws[lr0 + a][jb + q];
+        }
+      } else {
+#pragma unroll 4
+        for (int d = 0; d < NB; ++d) {
+          const float2 rk = *reinterpret_cast<const float2*>(&Rk[d][i0]);
+          float wv[TC];
+          if constexpr (TC == 4) {
+            const float4 t = *reinterpret_cast<const float4*>(&Ws[d][jb]);
+            wv[0] = t.x; wv[1] = t.y; wv[2] = t.z; wv[3] = t.w;
+          } else {
+            const float2 t = *reinterpret_cast<const float2*>(&Ws[d][jb]);
+            wv[0] = t.x; wv[1] = t.y;
+          }
+          const float rka[2] = {rk.x, rk.y};
+#pragma unroll
+          for (int a = 0; a < TR; ++a)
+#pragma unroll
+            for (int q = 0; q < TC; q += 2) {   // lane-wise fma.rn, the same rounding as fmaf
+              const float2 s2 = __ffma2_rn(make_float2(-rka[a], -rka[a]), make_float2(wv[q], wv[q + 1]),
+                                           make_float2(S[a][q], S[a][q + 1]));
+              S[a][q] = s2.x;
+              S[a][q + 1] = s2.y;
+            }
+        }
+        if (colsK) {
+#pragma unroll
+          for (int q = 0; q < TC; ++q)
+#pragma unroll
+            for (int a = 0; a < TR; ++a) S[a][q] = Ws[jb + q - k0][i0 + a];
+        }
+      }
+      if (next) publish_rows();
+    } else if (next) {
+      float A[EPL];
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) A[e] = Pn[pr][pc + e];
+#pragma unroll
+      for (int d = 0; d < NB; ++d) {   // the fma chains of the tile owners, in the same order
+        const float rk = Rk[d][kn + pr];
+        float wv[EPL];
+#pragma unroll
+        for (int e = 0; e < EPL; e += 2) {
+          const float2 t = *reinterpret_cast<const float2*>(&Ws[d][kn + pc + e]);
+          wv[e] = t.x;
+          wv[e + 1] = t.y;
+        }
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) A[e] = fmaf(-rk, wv[e], A[e]);
+      }
+      warp_sweep<NB>(A, lane);
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) pubQ[pr][pc + e] = -A[e];
+    }
+    cluster.sync();   // the next owner's rows and inverse are published; Rk, Qk, Ws may be overwritten
+  }
+
+  if (MODE == 0) {
+    if (op == nullptr) {
+      if (tile) {
+#pragma unroll
+        for (int a = 0; a < TR; ++a) {
+          float v[TC];
+#pragma unroll
+          for (int q = 0; q < TC; ++q) v[q] = -S[a][q];
+          store_run(out, i0 + a, v);
+        }
+      }
+    } else if constexpr (WP == 128) {
+      // Ginv * 2^sg as hi / lo fp16 K-major operands (zero outside w x w), sg from the cluster-wide max |Ginv|
+      float mx = 0.f;
+      if (tile) {
+#pragma unroll
+        for (int a = 0; a < TR; ++a)
+#pragma unroll
+          for (int q = 0; q < TC; ++q)
+            if (i0 + a < w && jb + q < w) mx = fmaxf(mx, fabsf(S[a][q]));
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      if (lane == 0) red[warp] = mx;
+      __syncthreads();
+      if (tid == 0) {
+        float t = 0.f;
+#pragma unroll
+        for (int q = 0; q < NW; ++q) t = fmaxf(t, red[q]);
+        cpart[1] = t;
+      }
+      cluster.sync();
+#pragma unroll
+      for (int q = 0; q < CS; ++q) mx = fmaxf(mx, *cluster.map_shared_rank(&cpart[1], q));
+      const int sg = fp16_scale_exp(mx);
+      const float sc = ldexpf(1.f, sg);
+      if (tile) {
+#pragma unroll
+        for (int a = 0; a < TR; ++a) {
+          const int i = i0 + a;
+          __align__(8) __half hi[4];
+          __align__(8) __half lo[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) split_f16((i < w && jb + q < w) ? -S[a][q] * sc : 0.f, hi[q], lo[q]);
+          const uint32_t off = k_major_offset(128u, (uint32_t)i, (uint32_t)jb);
+          *reinterpret_cast<uint2*>(op + off) = *reinterpret_cast<const uint2*>(hi);
+          *reinterpret_cast<uint2*>(op + 2 * 16384u + off) = *reinterpret_cast<const uint2*>(lo);
+        }
+      }
+      if (c == 0 && tid == 0) *reinterpret_cast<int*>(op + 4 * 16384u) = sg;
+    }
+  } else if (tile) {
+    float rv[TC];
+#pragma unroll
+    for (int q = 0; q < TC; ++q) rv[q] = jb + q < w ? r[jb + q] : 0.f;
+#pragma unroll
+    for (int a = 0; a < TR; ++a) {
+      const int i = i0 + a;
+      F2 acc2;
+#pragma unroll
+      for (int q = 0; q < TC; ++q)
+        if (jb + q < w) acc2 = f2_add(acc2, -S[a][q] * rv[q]);
+#pragma unroll
+      for (int o = CG / 2; o > 0; o >>= 1) acc2 = f2_add(acc2, f2_shfl_xor(acc2, o));
+      if (tc == 0 && i < w) out[i] = acc2.hi + acc2.lo;
+    }
+  }
+  if (IN_INT) {   // every CTA has read its entries (the cluster barriers since): reset the own rows
+    const int rows = min(NB, max(0, w - NB * c));
+    int* base = Gint + (long long)NB * c * w;
+    const int cnt = rows * w;
+    if (vec) {
+      for (int idx = tid; idx < cnt / 4; idx += NT + 32) reinterpret_cast<int4*>(base)[idx] = make_int4(0, 0, 0, 0);
+    } else {
+      for (int idx = tid; idx < cnt; idx += NT + 32) base[idx] = 0;
+    }
+  }
+  cluster.sync();   // no CTA leaves while another may still read its shared memory
+}
+
 int gram_chunk(int w, int L, int* splits) {
   int sms = 152, dev = 0;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -709,6 +1506,15 @@ int gram_chunk(int w, int L, int* splits) {
   const int chunk = (int)round_up(cdiv(L, s), GY);
   *splits = (int)cdiv(L, chunk);
   return chunk;
+}
+
+// The register-tiled inverse (inv_kernel); EXTERND_INV=0 keeps the earlier 16-warp sweep, for comparisons.
+bool tiled_inverse() {
+  static const bool enabled = [] {
+    const char* e = std::getenv("EXTERND_INV");
+    return !(e && std::strcmp(e, "0") == 0);
+  }();
+  return enabled;
 }
 
 template <int W_PAD, int NB, int MODE>
@@ -722,7 +1528,10 @@ cudaError_t launch_sweep_int_w(int* Gint, int w, const float* GVraw, const float
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  sweep32_kernel<W_PAD, NB, MODE, true><<<1, 544, smem, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint, op);
+  if (tiled_inverse())
+    inv_kernel<W_PAD, MODE, true><<<1, inv_threads<W_PAD>(), 0, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint, op);
+  else
+    sweep32_kernel<W_PAD, NB, MODE, true><<<1, 544, smem, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint, op);
   return cudaGetLastError();
 }
 
@@ -740,14 +1549,81 @@ cudaError_t launch_sweep(const float* Gpart, int splits, int w, const float* GVr
                          float* out, cudaStream_t s, uint8_t* op = nullptr) {
   // elements per lane RPW * CPL = W_PAD^2 / (32 * NWARP): 4 / 8 / 32 / 64
   // pivot-block sizes measured fastest on GB300: 8 up to w = 64, 16 at w = 128
-  if (w <= 32) sweep32_kernel<32, 8, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
+  const bool tiled = tiled_inverse();
+  if (w <= 32 && tiled) inv_kernel<32, MODE, false><<<1, inv_threads<32>(), 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
+  else if (w <= 64 && tiled) inv_kernel<64, MODE, false><<<1, inv_threads<64>(), 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
+  else if (w <= 128 && tiled) inv_kernel<128, MODE, false><<<1, inv_threads<128>(), 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, op);
+  else if (w <= 32) sweep32_kernel<32, 8, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
   else if (w <= 64) sweep32_kernel<64, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
   else if (w <= 128) sweep32_kernel<128, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, op);
   else sweep_kernel<256, 32, MODE><<<1, 32 * 32, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out);
   return cudaGetLastError();
 }
 
+// The cluster inverse and its launches (programmatic dependent launch of the next kernel when pdl). Off unless
+// EXTERND_CLUSTER_INV=1: on this GPU the pivot rows' broadcast through distributed shared memory costs about as
+// much per step as the single-CTA sweep's update, so the one-CTA inverse beside the product is faster overall.
+bool cluster_inverse_enabled() {
+  static const bool enabled = [] {
+    const char* e = std::getenv("EXTERND_CLUSTER_INV");
+    return e && std::strcmp(e, "1") == 0;
+  }();
+  return enabled;
+}
+
+template <int WP, int MODE, bool IN_INT>
+cudaError_t launch_cluster_w(const float* Gpart, int splits, int w, const float* GVraw, const float* r, float* Graw,
+                             float* out, int* Gint, uint8_t* op, bool pdl, cudaStream_t s) {
+  constexpr int CS = InvClusterShape<WP>::CS;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(CS, 1, 1);
+  cfg.blockDim = dim3(inv_cluster_threads<WP>(), 1, 1);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = CS;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, inv_cluster_kernel<WP, MODE, IN_INT>, Gpart, splits, w, GVraw, r, Graw, out, Gint,
+                            op, pdl ? 1 : 0);
+}
+
+template <int MODE, bool IN_INT>
+cudaError_t launch_cluster(const float* Gpart, int splits, int w, const float* GVraw, const float* r, float* Graw,
+                           float* out, int* Gint, uint8_t* op, bool pdl, cudaStream_t s) {
+  if (w <= 16 || w > 128) return cudaErrorInvalidValue;
+  if (w <= 32) return launch_cluster_w<32, MODE, IN_INT>(Gpart, splits, w, GVraw, r, Graw, out, Gint, nullptr, pdl, s);
+  if (w <= 64) return launch_cluster_w<64, MODE, IN_INT>(Gpart, splits, w, GVraw, r, Graw, out, Gint, nullptr, pdl, s);
+  return launch_cluster_w<128, MODE, IN_INT>(Gpart, splits, w, GVraw, r, Graw, out, Gint, op, pdl, s);
+}
+
 }  // namespace
+
+int inverse_cluster_size(int w) {
+  if (!cluster_inverse_enabled() || w <= 16 || w > 128) return 0;
+  return w <= 32 ? 2 : w <= 64 ? 4 : 8;
+}
+
+cudaError_t launch_inverse_cluster(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s,
+                                   void* op, bool pdl) {
+  if (op != nullptr && (w <= 64 || w > 128 || (reinterpret_cast<uintptr_t>(op) & 15) != 0)) return cudaErrorInvalidValue;
+  return launch_cluster<0, false>(Gpart, splits, w, nullptr, nullptr, Graw, Ginv, nullptr, static_cast<uint8_t*>(op),
+                                  pdl, s);
+}
+
+cudaError_t launch_inverse_cluster_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s, void* op, bool pdl) {
+  if (op != nullptr && (w <= 64 || w > 128 || (reinterpret_cast<uintptr_t>(op) & 15) != 0)) return cudaErrorInvalidValue;
+  return launch_cluster<0, true>(nullptr, 0, w, nullptr, nullptr, Graw, Ginv, Gint, static_cast<uint8_t*>(op), pdl,
+                                 s);
+}
+
+cudaError_t launch_scales_cluster_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s,
+                                      float* K) {
+  return launch_cluster<1, true>(nullptr, 0, w, GVraw, r, K, d, GUint, nullptr, false, s);
+}
 
 int gram_splits(int w, int L) {
   int s;

@@ -93,10 +93,13 @@ def test_block_width_one_first_components_match_exactly(X):
     assert np.allclose(res.D.cpu().numpy(), ref.D, rtol=1e-5)
 
 
-def test_first_block_matches_exactly(X):
-    A = W.student_t(128, 160, 5.0, 0.015, 6)
-    ref = O.block_als(A, 16 / 128, 0.7, 16, 2)    # one block of 16 components
-    res = X.decompose(cuda(A), 16 / 128, 0.7, 16, 2)
+@pytest.mark.parametrize("m,n,w", [(128, 160, 16), (256, 320, 24), (400, 416, 48), (640, 768, 80)])
+def test_first_block_matches_exactly(X, m, n, w):
+    # one block of w components: the FMA inverse beside the product (w = 16), the cluster inverse (w > 16), the
+    # tensor-core targets (w > 64)
+    A = W.student_t(m, n, 5.0, 0.015, 6)
+    ref = O.block_als(A, w / min(m, n), 0.7, w, 2)
+    res = X.decompose(cuda(A), w / min(m, n), 0.7, w, 2)
     assert (res.B.cpu().numpy() == ref.B).all() and (res.C.cpu().numpy() == ref.C).all()
     assert np.allclose(res.D.cpu().numpy(), ref.D, rtol=1e-4)
 
