@@ -6,16 +6,18 @@
 //
 // A CTA owns 128 output positions (MMA M) and all w components (N = w rounded up to 16), reducing over one
 // split of the other dimension in stages of 64. Roles, all hand-offs through mbarriers with bounded waits:
-//   producer (one thread)  TMA loads of the float32 R tile of a stage (128-byte swizzled boxes of 32 floats)
-//                          into a ring of S32 slots, and of the stage's fp16 ternary tile (the MMA's B operand,
-//                          128-byte swizzled K-major) into a ring of SB slots
-//   converters (8 warps)   read a staged R tile (lanes on consecutive positions: conflict-free), scale it by
-//                          2^s, split it into fp16 hi and lo, and write the two swizzled K-major A tiles into a
-//                          ring of S16 slots; the same warps run the epilogue (TMEM -> split-K partials)
-//   MMA (one thread)       two kind::f16 MMAs per 16-deep K step (hi and lo against the same B), commits that
-//                          free the A and B slots
-// R never passes through registers on its way into shared memory, so the loads of several stages are in flight
-// per SM without any register cost.
+//   R producer (1 thread)  TMA loads of the float32 R tile of a stage (128-byte swizzled boxes of 32 floats)
+//                          into a ring of S32 slots; the stage's fp16 ternary tile (the MMA's B operand,
+//                          128-byte swizzled K-major) goes into a ring of SB slots
+//   converters (16 warps)  read a staged R tile into registers (lanes on consecutive positions) and free its
+//                          slot at once, scale it by 2^s, split it into fp16 hi and lo and store the two A tiles
+//                          into tensor memory (one position per lane, a ring of S16 stages); the same warps run
+//                          the epilogue (TMEM -> split-K partials)
+//   B producer (1 thread)  TMA loads of the ternary tiles, so that a B slot the MMAs still hold never delays R
+//   MMA (one thread)       two kind::f16 MMAs per 16-deep K step (hi and lo from tensor memory against the same
+//                          B in shared memory), commits that free the A stages and B slots
+// R never passes through registers on its way into shared memory, and with A in tensor memory the shared memory
+// holds six R stages: about 190 KB of copies in flight per SM, enough to keep the HBM queue full.
 //
 // Work is a sequence of units (128 positions x 64 reduction rows), tile-major. Classic plan: CTA (tile, split)
 // takes one tile's units of its split, and writes partial slot `split`. Stream plan, used when tiles x splits
@@ -43,7 +45,7 @@ static_assert(kConv % 128 == 0 && kItems >= 1, "a converter thread keeps one pos
 constexpr int kProducerWarp = kConvWarps, kMmaWarp = kConvWarps + 1, kBWarp = kConvWarps + 2;
 constexpr int kThreads = (kConvWarps + 3) * 32;
 constexpr int kStageK = 64;
-constexpr uint32_t kTileA = 128u * 128u;      // 128 rows x 64 fp16
+constexpr uint32_t kAcols = 64u;               // TMEM columns of one stage's A operand: 64 fp16 hi + 64 lo per row
 constexpr uint32_t kStage32 = 128u * 64u * 4u;   // float32 R tile of one stage
 
 struct TmaArgs {
@@ -54,6 +56,7 @@ struct TmaArgs {
   unsigned* err;
   int s32, sb, s16;
   uint32_t tmem_cols;
+  uint32_t acol;       // first TMEM column of the A stages (after the accumulators)
   int nkt;             // units per tile: cdiv(Ly, 64)
   int cu;              // classic: units per split
   long long U;         // stream: all units (tiles x nkt)
@@ -97,8 +100,7 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
   const uint32_t tileB = (uint32_t)p.wpad * 128u;
   const uint32_t r32 = sbase;                                   // S32 x 32 KB
   const uint32_t rb = r32 + (uint32_t)p.s32 * kStage32;         // SB x tileB (1024-aligned: tileB = wpad * 128)
-  const uint32_t ra = rb + (uint32_t)round_up((long long)p.sb * tileB, 1024);   // S16 x (2 x 16 KB)
-  const uint32_t bars = ra + (uint32_t)p.s16 * 2u * kTileA;
+  const uint32_t bars = rb + (uint32_t)round_up((long long)p.sb * tileB, 1024);
   const uint32_t full32 = bars, empty32 = full32 + 8u * p.s32;
   const uint32_t fullB = empty32 + 8u * p.s32, emptyB = fullB + 8u * p.sb;
   const uint32_t full16 = emptyB + 8u * p.sb, empty16 = full16 + 8u * p.s16;
@@ -281,12 +283,14 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
         }
         tc_fence_after();
         const uint32_t d = tmem + (uint32_t)((seg & 1) * p.wpad);
-        const uint32_t a_hi = ra + (uint32_t)s * 2u * kTileA, a_lo = a_hi + kTileA, bt = rb + (uint32_t)sb * tileB;
+        // A from tensor memory: stage s holds hi in columns acol + 64 s .. + 31 and lo in the next 32, two fp16
+        // (consecutive K) per column, one position per lane
+        const uint32_t a_hi = tmem + p.acol + (uint32_t)s * kAcols, a_lo = a_hi + kAcols / 2, bt = rb + (uint32_t)sb * tileB;
 #pragma unroll
         for (int kk = 0; kk < kStageK / 16; ++kk) {
           const uint64_t bd = sw128_desc(bt + 32u * kk);
-          mma_f16(d, sw128_desc(a_hi + 32u * kk), bd, idesc, (!first || kk > 0) ? 1u : 0u);
-          mma_f16(d, sw128_desc(a_lo + 32u * kk), bd, idesc, 1u);
+          mma_f16_ts(d, a_hi + 8u * kk, bd, idesc, (!first || kk > 0) ? 1u : 0u);
+          mma_f16_ts(d, a_lo + 8u * kk, bd, idesc, 1u);
         }
         mma_commit(empty16 + 8u * s);
         mma_commit(emptyB + 8u * sb);
@@ -348,8 +352,10 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
       got = k < p.s16 || mbar_wait(empty16 + 8u * s16, (uint32_t)(k / p.s16 - 1) & 1u, p.err);
       ok = __all_sync(0xffffffffu, got) != 0;
       if (!ok) break;
-      uint8_t* a_hi = gbase + (ra - sbase) + (size_t)s16 * 2u * kTileA;
-      uint8_t* a_lo = a_hi + kTileA;
+      tc_fence_after();   // the MMAs that read this A stage are complete: its columns may be rewritten
+      // this warp's lanes (positions 32 (warp % 4) .. + 31) of stage s16's A columns in tensor memory
+      const uint32_t a_hi = tmem + ((uint32_t)(quad * 32) << 16) + p.acol + (uint32_t)s16 * kAcols;
+      const uint32_t a_lo = a_hi + kAcols / 2;
 #pragma unroll
       for (int q = 0; q < kItems; ++q) {
         const int o = o0 + (kConv / 128) * q;
@@ -371,11 +377,12 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
             split_pair(x0v, x1v, hi[e], lo[e]);
           }
         }
-        const uint32_t off = sw128_offset((uint32_t)x, (uint32_t)o);
-        *reinterpret_cast<uint4*>(a_hi + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-        *reinterpret_cast<uint4*>(a_lo + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        // K chunk o (warp-uniform) is columns 4 o .. 4 o + 3: two fp16 of consecutive K per 32-bit column
+        tmem_st4(a_hi + 4u * (uint32_t)o, hi[0], hi[1], hi[2], hi[3]);
+        tmem_st4(a_lo + 4u * (uint32_t)o, lo[0], lo[1], lo[2], lo[3]);
       }
-      fence_async_shared();
+      tmem_wait_st();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(full16 + 8u * s16);
       // the previous segment's partials, once this segment is fully converted (its MMAs are then queued)
@@ -426,13 +433,17 @@ TmaPlan tma_plan(int w) {
   TmaPlan t;
   t.wpad = (int)round_up(w, 16);
   const size_t tileB = (size_t)t.wpad * 128;
-  t.s16 = 2;
-  t.sb = 2;   // the ternary tiles come from L2: two slots keep the MMAs fed; the rest of the space holds R in flight
-  const size_t budget = 227 * 1024 - 1024 - 512 - (size_t)t.s16 * 2 * kTileA - round_up((long long)t.sb * tileB, 1024);
+  // A stages live in tensor memory (4 x 64 columns beside up to 256 accumulator columns). The ternary tiles come
+  // from L2 but under a saturated HBM queue still take a microsecond or more: four B slots let them be requested
+  // well ahead of the MMAs, so that neither the MMAs nor (through the A stages) the converters wait for them; the
+  // rest of the space holds R in flight.
+  t.s16 = 4;
+  t.sb = 4;
+  const size_t budget = 227 * 1024 - 1024 - 512 - round_up((long long)t.sb * tileB, 1024);
   int s = 6;
   while (s > 1 && (size_t)s * kStage32 > budget) --s;
   t.s32 = s;
-  t.smem = 1024 + (size_t)s * kStage32 + round_up((long long)t.sb * tileB, 1024) + (size_t)t.s16 * 2 * kTileA + 512;
+  t.smem = 1024 + (size_t)s * kStage32 + round_up((long long)t.sb * tileB, 1024) + 512;
   return t;
 }
 
@@ -508,9 +519,11 @@ cudaError_t launch_tma(const float* R, int m, int n, const __half* T, int ldt, i
     if (e != cudaSuccess) return e;
     configured[USTEP] = true;
   }
+  // accumulators (the stream plan alternates two), then the A stages
+  const uint32_t acol = (uint32_t)((wk.stream ? 2 : 1) * t.wpad);
   uint32_t cols = 32;
-  while ((int)cols < (wk.stream ? 2 : 1) * t.wpad) cols <<= 1;   // the stream plan alternates two accumulators
-  TmaArgs a{m, n, w, t.wpad, h, part, maxabs, err, t.s32, t.sb, t.s16, cols, wk.nkt, wk.cu, wk.U, wk.slots};
+  while (cols < acol + (uint32_t)t.s16 * kAcols) cols <<= 1;
+  TmaArgs a{m, n, w, t.wpad, h, part, maxabs, err, t.s32, t.sb, t.s16, cols, acol, wk.nkt, wk.cu, wk.U, wk.slots};
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)wk.grid_x, 1, (unsigned)wk.grid_z);
   cfg.blockDim = dim3(kThreads, 1, 1);
