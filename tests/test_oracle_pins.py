@@ -56,6 +56,13 @@ def test_ternarize_hand_cases():
     assert (O.ternarize(x, 0.7) == -O.ternarize(-x, 0.7)).all()
 
 
+def test_ternarize_mean_counts_zeros():
+    # Eq. 2's mean runs over the vector's whole length, zeros included: |x| = (3, 1.2, 0, 0) has mean 4.2 / 4 =
+    # 1.05, so 1.2 passes at tau = 1 (over the nonzeros, or over L - 1 = 3 entries, it would not).
+    assert O.ternarize([3.0, -1.2, 0.0, 0.0], 1.0).tolist() == [1, -1, 0, 0]
+    assert O.ternarize([0.0, 0.0, 1.2, -3.0], 1.0).tolist() == [0, 0, 1, -1]
+
+
 def test_ternarize_strict_threshold_boundary():
     # mean |x| = 1 exactly; at tau = 2 the entry equal to the threshold (2.0) must not pass.
     x = np.array([2.0, 0.5, 0.5, 1.0])
@@ -318,3 +325,85 @@ def test_weighted_vstep_correction_beats_naive_weighted_vstep():
     naive = _naive_block(A, 1.5, 0.7, 12, 4, h, naive_w=True)
     # §2.5: the naive weighted V-step loses 0.3-1.8 points of weighted energy.
     assert corrected > naive
+
+
+# ---------------------------------------------------------------------------------------------- a block step by hand
+def test_hand_computed_two_component_block_step():
+    """One block of w = 2 (§2.4, Eq. 3 and Eq. 4) worked out by hand on a 4 x 4 residual, tau = 0.7.
+
+    Start (largest column energies 32 and 18: columns 0 and 1): U = [e0 + e1, e2 + e3].
+    V-step: U^T U = 2 I, eps = 1e-4 * 4 / 2, so X = (R[0] + R[1], R[2] + R[3]) / 2.0002 = ([8,0,0,0], [0,6,0,1])
+    / 2.0002; means of |x| 2 and 1.75 (times 1 / 2.0002) give thresholds 1.4 and 1.225 (same scale): V = e0, e1.
+    U-step: V^T V = I, eps = 1e-4, Y = R V / 1.0001 = ([4,4,0,0], [0,0,3,3]) / 1.0001: U stays [e0 + e1, e2 + e3].
+    Eq. 4: K = (U^T U) .* (V^T V) = 2 I, eps = 1e-4 * 4 / 2 = 2e-4, r = (8, 6): d = (8, 6) / 2.0002.
+    Deflation leaves 4 - d0 in R[0:2, 0], 3 - d1 in R[2:4, 1] and the three unit entries."""
+    R = np.array([[4.0, 0.0, 1.0, 0.0],
+                  [4.0, 0.0, -1.0, 0.0],
+                  [0.0, 3.0, 0.0, 0.0],
+                  [0.0, 3.0, 0.0, 1.0]])
+    U0 = np.array([[1, 0], [1, 0], [0, 1], [0, 1]], dtype=np.int8)
+    assert O.initial_columns(R, 2, np.ones(4)).tolist() == [0, 1]
+    assert (O.ternarize_cols(R[:, [0, 1]], 0.7) == U0).all()
+    X = O.vstep_target(R, U0)
+    assert np.allclose(X, np.array([[8.0, 0, 0, 0], [0, 6.0, 0, 1.0]]) / 2.0002, rtol=1e-14, atol=0)
+    Cb = O.ternarize_rows(X, 0.7)
+    assert (Cb == np.array([[1, 0, 0, 0], [0, 1, 0, 0]])).all()
+    PU = O.ustep_product(R, Cb)
+    assert np.array_equal(PU, np.array([[4.0, 0], [4.0, 0], [0, 3.0], [0, 3.0]]))
+    Y = O.ustep_solve(PU, Cb)
+    assert np.allclose(Y, PU / 1.0001, rtol=1e-14, atol=0)
+    U1 = O.ternarize_cols(Y, 0.7)
+    assert (U1 == U0).all()
+    d = O.block_scales(U1, Cb, PU)
+    assert np.allclose(d, [8 / 2.0002, 6 / 2.0002], rtol=1e-14, atol=0)
+    R1 = O.deflate(R, U1, d, Cb)
+    expect = R.copy()
+    expect[0:2, 0] = 4 - 8 / 2.0002
+    expect[2:4, 1] = 3 - 6 / 2.0002
+    assert np.allclose(R1, expect, rtol=0, atol=1e-14)
+
+
+# ---------------------------------------------------------------------------------------------- block loop properties
+def _block_residuals(A, res, b):
+    """The residual each block of a block_als result was fitted to, rebuilt from the returned factors alone."""
+    R = np.asarray(A, dtype=np.float64).copy()
+    out = []
+    for j0 in range(0, res.D.size, b):
+        j1 = min(res.D.size, j0 + b)
+        out.append((R.copy(), j0, j1))
+        R = R - (res.B[:, j0:j1] * res.D[j0:j1]) @ res.C[j0:j1].astype(np.float64)
+    return out
+
+
+@pytest.mark.parametrize("weighted", [False, True])
+def test_block_loop_scales_are_ridge_least_squares_for_each_block(weighted):
+    # Eq. 4 for the factors block_als returns: each block's D is the ridge least-squares scale of its own U and V
+    # against the residual it was fitted to (lstsq on the vectorised problem, independent of the oracle's solver).
+    A = W.student_t(40, 48, 5.0, 0.015, 21)
+    h = W.importance(48, 21).astype(float) if weighted else None
+    hh = np.ones(48) if h is None else h
+    res = O.block_als(A, 0.6, 0.7, 8, 3, h)
+    for R, j0, j1 in _block_residuals(A, res, 5):
+        U, Cb = res.B[:, j0:j1].astype(float), res.C[j0:j1].astype(float)
+        K = (U.T @ U) * (Cb @ (hh[:, None] * Cb.T))
+        eps = O.EPS_REL * np.trace(K) / (j1 - j0) if j1 - j0 > 1 else 0.0
+        d_ls, _ = _lstsq_scales(R, U, Cb, hh, eps)
+        assert np.allclose(res.D[j0:j1], d_ls, rtol=1e-9, atol=1e-12), (j0, j1)
+
+
+@pytest.mark.parametrize("weighted", [False, True])
+def test_block_loop_final_u_is_the_ustep_of_the_final_v(weighted):
+    # The last step of every block is the U-step (Eq. 3 right, §2.5): U = T_tau of the weighted ridge
+    # least-squares target of the block's final V against the residual it was fitted to (lstsq, column-weighted).
+    A = W.gaussian(40, 48, 0.02, 22)
+    h = W.importance(48, 22).astype(float) if weighted else None
+    hh = np.ones(48) if h is None else h
+    res = O.block_als(A, 0.6, 0.7, 8, 3, h)
+    for R, j0, j1 in _block_residuals(A, res, 5):
+        V = res.C[j0:j1].astype(float).T
+        w = j1 - j0
+        eps = O.EPS_REL * np.sum(hh[:, None] * V * V) / w
+        sh = np.sqrt(hh)[:, None]
+        Yt = np.linalg.lstsq(np.vstack([sh * V, math.sqrt(eps) * np.eye(w)]),
+                             np.vstack([sh * R.T, np.zeros((w, R.shape[0]))]), rcond=None)[0]
+        assert (O.ternarize_cols(Yt.T, 0.7) == res.B[:, j0:j1]).all(), (j0, j1)
