@@ -250,7 +250,21 @@ def algorithmic_bytes(kind, wl):
         return (algorithmic_bytes("vstep", wl) + algorithmic_bytes("ustep", wl)) / 2
     if kind == "deflate":    # read and write R, read U, V, d
         return 8 * m * n + (m + n) * b + 4 * b + hbytes
+    if kind == "sequential":   # the one-launch b = 1 fit: R in shared memory, per component the start's column
+        # energies and column, 2 iters products and the deflation's read and write: (2 iters + 3) 4mn bytes
+        return inner_rank(wl) * (2 * wl.iters + 3) * 4 * m * n
     raise ValueError(kind)
+
+
+# Shared-memory roofline of the one-launch sequential kernel: its cluster's 8 SMs, 128 bytes per SM per clock
+# (32 banks x 4 bytes) at the 2070 MHz maximum SM clock.
+SEQ_SMEM_GBS = 8 * 128 * 2.07
+
+
+def sequential_workload(wl):
+    """Block width 1 and a residual that fits the cluster kernel's shared memory (8 CTAs, <= 200 KB each)."""
+    rpc = -(-wl.m // 8)
+    return block_width(wl) == 1 and wl.n <= 4096 and (rpc * wl.n + 5 * wl.n + 2 * rpc) * 4 <= 200 * 1024
 
 
 def decomposition_bytes(wl):
@@ -368,7 +382,10 @@ def run_gpu(args):
 
     # ---- live roofline of the dominant kernel class: event pairs inside the graph, over a second timed pass
     kind = args.roofline_kind
-    X.profile(kind)
+    seq = all(sequential_workload(wl) for wl in wls)
+    if seq:   # the whole fit is one kernel (profiled as the solve class)
+        kind = "sequential"
+    X.profile("solve" if seq else kind)
     for _ in range(2):
         flush.fill_(0.0)
         step()
@@ -384,8 +401,11 @@ def run_gpu(args):
     X.profile("off")
     per_launch_s = prof_ms / 1e3 / max(prof_n, 1)
     bytes_per_launch = prof_bytes / max(prof_n, 1)
-    achieved = bytes_per_launch / per_launch_s / 1e9
+    achieved = bytes_per_launch / per_launch_s / 1e9 if per_launch_s > 0 else 0.0
     peak, peak_src = peaks()
+    bound = "hbm"
+    if seq:
+        bound, peak, peak_src = "smem", SEQ_SMEM_GBS, "derived: 8 SMs x 128 B/clock x 2070 MHz"
     traffic = None
     src = os.path.join(ROOT, "paper_2607_13511_gb300", "csrc", NCU_TRAFFIC.get("file", "gemm.cu"))
     if NCU_TRAFFIC.get("kind") == kind and os.path.exists(src) and NCU_TRAFFIC.get("sha") == source_sha(src) \
@@ -421,12 +441,13 @@ def run_gpu(args):
     line["e2e"] = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                    "path": "externd_decompose_host (pinned host buffers)"}
     line["gpu_launches"] = launches
-    line["roofline"] = {"bound": "hbm", "kernel": kind, "achieved": achieved, "peak": peak, "unit": "GB/s",
+    line["roofline"] = {"bound": bound, "kernel": kind, "achieved": achieved, "peak": peak, "unit": "GB/s",
                         "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
                         "bytes_per_launch": bytes_per_launch, "launches": prof_n,
                         "us_per_launch": per_launch_s * 1e6}
-    line["step_roofline"] = {"algorithmic_bytes": step_bytes, "lower_bound_ms": step_bytes / (peak * 1e6),
-                             "frac": step_bytes / (peak * 1e6) / ms_step}
+    if not seq:   # the HBM model of the whole step: 2 iters passes over R and the deflation per block
+        line["step_roofline"] = {"algorithmic_bytes": step_bytes, "lower_bound_ms": step_bytes / (peak * 1e6),
+                                 "frac": step_bytes / (peak * 1e6) / ms_step}
     cs = clocks.summary()
     if cs is not None:
         line["clocks"] = cs
@@ -523,6 +544,31 @@ def run_row(args):
                          "cpu_baseline": {"value": kk / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                                           "sample": f"one sweep over the first {kk} components of {wl.name}, "
                                                     f"{dt:.1f} s"}})
+    elif args.row == "sequential":
+        # §2.3 against §2.4 on the same matrices: the sequential algorithm (block width 1) and the block algorithm
+        # at the cap, the same number of components; the paper reports about 16x for block over sequential (§3.1)
+        cases = []
+        for wl_s, block, mu in ((W.SEQUENTIAL_256, 32, None), (W.MLP_UP_2560x9728, 128, 256 / 2560)):
+            A = torch.from_numpy(wl_s.matrix()).to(dev)
+            mu_c = wl_s.mu if mu is None else mu
+            kk = X.rank(wl_s.m, wl_s.n, mu_c)
+            res = {}
+            for b in (1, block):
+                fn = lambda b=b: X.decompose(A, mu_c, wl_s.tau, b, wl_s.iters)
+                for _ in range(max(1, args.warmup)):
+                    fn()
+                reps = 3 if (b == 1 and wl_s.m * wl_s.n > 1 << 20) else args.steps
+                ms, dec = time_steps(torch, stream, reps, fn)
+                res[b] = {"ms": ms, "components_per_s": kk / (ms / 1e3), "energy": dec.energy,
+                          "launches": X.kernel_launches()}
+            cases.append({"matrix": wl_s.name, "m": wl_s.m, "n": wl_s.n, "k": kk, "tau": wl_s.tau,
+                          "iters": wl_s.iters, "sequential_b1": res[1], f"block_b{block}": res[block],
+                          "block_over_sequential": res[block]["components_per_s"] / res[1]["components_per_s"]})
+        line.update({"metric": "ternary components fitted/sec, sequential (§2.3) and block (§2.4) on the same matrix",
+                     "unit": UNIT, "value": cases[0]["sequential_b1"]["components_per_s"],
+                     "ms_per_step": cases[0]["sequential_b1"]["ms"], "higher_is_better": True, "dtype": "f32",
+                     "cases": cases,
+                     "paper_context": "about 16x block over sequential on one AMD MI50 (torch), §3.1 / Table 1"})
     else:   # packed inference product
         m, n = wl.m, wl.n
         layer_bytes = (m * k + k * n) / 4.0                    # 2 bits per ternary entry
@@ -582,7 +628,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-blocks", type=int, default=16, help="blocks of the workload the CPU baseline times")
     ap.add_argument("--reference-blocks", type=int, default=2, help="blocks per step of the reference arm")
-    ap.add_argument("--row", default="decompose", choices=["decompose", "safeguard", "refine", "packed"],
+    ap.add_argument("--row", default="decompose", choices=["decompose", "safeguard", "refine", "packed", "sequential"],
                     help="an extension row instead of the headline decomposition (one GPU)")
     args = ap.parse_args()
     if args.row != "decompose":

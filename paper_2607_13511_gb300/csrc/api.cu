@@ -72,14 +72,16 @@ struct Profile {
 };
 Profile g_prof;
 
-cudaError_t prof_mark(cudaStream_t s) {
+cudaError_t prof_mark(cudaStream_t s, bool captured = true) {
   if (g_prof.used == g_prof.events.size()) {
     cudaEvent_t e;
     cudaError_t err = cudaEventCreate(&e);
     if (err != cudaSuccess) return err;
     g_prof.events.push_back(e);
   }
-  return cudaEventRecordWithFlags(g_prof.events[g_prof.used++], s, cudaEventRecordExternal);
+  // inside a stream capture the event becomes a node of the graph (external record); otherwise a plain record
+  return captured ? cudaEventRecordWithFlags(g_prof.events[g_prof.used++], s, cudaEventRecordExternal)
+                  : cudaEventRecord(g_prof.events[g_prof.used++], s);
 }
 
 template <typename T>
@@ -786,6 +788,53 @@ int run_plan(const Plan& p, const float* A, const float* h, int8_t* Bout, float*
   return EXTERND_OK;
 }
 
+// The one-launch cluster kernel for block width 1 where the residual fits its shared memory;
+// EXTERND_SEQ=0 keeps the kernel-by-kernel schedule, for comparisons.
+bool sequential_cluster_enabled() {
+  static const bool enabled = [] {
+    const char* e = std::getenv("EXTERND_SEQ");
+    return !(e && std::strcmp(e, "0") == 0);
+  }();
+  return enabled;
+}
+
+// §2.3 in one cluster launch (sequential.cu): the components, the energy after each, the final energy.
+int run_sequential(const Plan& p, const float* A, const float* h, int8_t* Bout, float* Dout, int8_t* Cout,
+                   double* energy, double* trace, long long* activations) {
+  Workspace* ws;
+  TRY(current_ws(&ws));
+  double *tr, *en;
+  long long* act = nullptr;
+  TRY(need(*ws, "trace", (size_t)p.k, &tr));
+  TRY(need(*ws, "seq.energy", 1, &en));
+  cudaStream_t s = g_stream;
+  if (activations != nullptr) {
+    TRY(need(*ws, "seq.act", 1, &act));
+    LK(cudaMemsetAsync(act, 0, sizeof(long long), s));
+  }
+  g_prof.used = 0;
+  const bool prof = g_prof.kind == kSolve;   // the whole fit is one kernel: timed as the solve class
+  if (prof) LK(prof_mark(s, false));
+  LK(launch_sequential_cluster(A, p.m, p.n, p.k, p.iters, p.tau, h, Bout, Dout, Cout, tr, en, act, s));
+  if (prof) LK(prof_mark(s, false));
+  g_prof.last_used = g_prof.used;
+  g_prof.last_launches = 1;
+  if (energy != nullptr || trace != nullptr || activations != nullptr) {
+    const size_t tb = sizeof(double) * (size_t)(trace != nullptr ? p.k : 0);
+    void* hbuf;
+    TRY(need_host(*ws, tb + 16, &hbuf));
+    CK(cudaMemcpyAsync(hbuf, en, sizeof(double), cudaMemcpyDeviceToHost, s));
+    if (act) CK(cudaMemcpyAsync(static_cast<char*>(hbuf) + 8, act, sizeof(long long), cudaMemcpyDeviceToHost, s));
+    if (tb > 0) CK(cudaMemcpyAsync(static_cast<char*>(hbuf) + 16, tr, tb, cudaMemcpyDeviceToHost, s));
+    CK(cudaStreamSynchronize(s));
+    if (energy) *energy = *static_cast<const double*>(hbuf);
+    if (activations) *activations = *reinterpret_cast<const long long*>(static_cast<char*>(hbuf) + 8);
+    if (tb > 0) std::memcpy(trace, static_cast<char*>(hbuf) + 16, tb);
+  }
+  CK(cudaGetLastError());
+  return EXTERND_OK;
+}
+
 int run_decompose(const float* A, long long m, long long n, double mu, double tau, int block, int iters,
                   const float* h, int8_t* Bout, float* Dout, int8_t* Cout, double* energy, double* trace,
                   long long* activations = nullptr) {
@@ -793,6 +842,8 @@ int run_decompose(const float* A, long long m, long long n, double mu, double ta
   TRY(externd_rank(m, n, mu, &k));
   Plan p = make_plan(m, n, k, block, iters, tau);
   p.mode = activations != nullptr ? kSafeguard : kPlain;
+  if (p.b == 1 && sequential_cluster_enabled() && sequential_cluster_fits(m, n))
+    return run_sequential(p, A, h, Bout, Dout, Cout, energy, trace, activations);
   return run_plan(p, A, h, Bout, Dout, Cout, energy, trace, p.nblocks, activations, activations ? 1 : 0);
 }
 

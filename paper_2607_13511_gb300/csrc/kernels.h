@@ -314,6 +314,14 @@ cudaError_t launch_scales_int(int* GUint, const float* GVraw, const float* r, in
                               float* K = nullptr);
 
 
+// ---- the sequential algorithm (§2.3, block width 1) in one launch of one thread-block cluster (sequential.cu),
+// for residuals that fit the cluster's shared memory. trace (k doubles) may be nullptr; energy: one double;
+// activations (one zeroed long long, or nullptr): Prop. 2's safeguard on, counting the components it replaced.
+bool sequential_cluster_fits(long long m, long long n);
+cudaError_t launch_sequential_cluster(const float* A, int m, int n, long long k, int iters, double tau, const float* h,
+                                      int8_t* B, float* D, int8_t* C, double* trace, double* energy,
+                                      long long* activations, cudaStream_t s);
+
 // ---- extensions of the block loop (extend.cu): Prop. 2 safeguard and §2.4 refinement sweeps
 struct __align__(16) EntryBest {   // a CTA's best single entry: score (|R_ij| or h_j R_ij^2), R_ij, row-major index
   float score, rij;
