@@ -32,10 +32,11 @@ constexpr uint32_t kOpCopy = 16384;                         // bytes per bulk co
 template <int NPOS>
 struct TcDecor {
   static constexpr uint32_t kAtomB = (uint32_t)NPOS * 128u;   // one K atom of B: NPOS rows x 128 B
-  static constexpr size_t kSmem = 1024 + kOpBytes + 2 * (2 * kAtomB);
+  static constexpr uint32_t kSlot = (uint32_t)kWp * NPOS * 4u;  // one split-K slot of the P tile, float32
+  static constexpr int kStage = NPOS == 64 ? 3 : (NPOS == 32 ? 7 : 14);   // slots staged at once (96-112 KB)
+  static constexpr size_t kSmem = 1024 + kOpBytes + 2 * (2 * kAtomB) + kStage * kSlot;
   static constexpr int kPairs = NPOS / 2;                     // position pairs: the threads of one b group
   static constexpr int kBper = 128 / (256 / kPairs);          // components b per thread: 16, 8 or 4
-  static constexpr int kSlotUnroll = 32 / kBper;              // slots loaded per round: 32 loads in flight
   static constexpr uint32_t kTmemCols = NPOS < 32 ? 32u : (uint32_t)NPOS;
 };
 
@@ -84,13 +85,16 @@ struct ApplyOut {
 // MODE 1 (cooperative; bar: 2 zero words, left zero): every CTA finalizes its share of the thresholds after a
 //   grid barrier, as in the FMA decorrelation.
 // MODE 2 (cooperative; bar: 4 zero words, left zero): no X; after a second grid barrier every CTA ternarizes its
-//   tile from TMEM (Eq. 2 with the finalized thresholds) and writes the factor layouts of `out`. With out.gram,
-//   the tile's Gram T T^T is one more MMA (M = N = 128, K = NPOS) on the fp16 trits in shared memory, stored to
-//   out.gsc as int8 (|count| <= NPOS); after a third barrier the warps of the grid sum the tiles' Grams, one warp
-//   per 16 entries of the upper triangle (8 lane groups over the tiles, 4 entries per lane, then shuffles), and
-//   add them to out.gram. Integer sums: the order does not matter. With out.h (the weighted V^T H V of §2.5) the
-//   B operand is t_b(x) h(x) as a scaled fp16 hi + lo pair (two MMAs per K step), the tile Grams are float32 and
-//   the sums, in a fixed order, are written to both triangles of out.gramf.
+//   tile from TMEM (Eq. 2 with the finalized thresholds) into a K-major fp16 image in shared memory, from which
+//   the warps write whole rows of T and T16 (the K-major copy Tk goes out position by position). With out.gram,
+//   the tile's Gram T T^T is one more MMA (M = N = 128, K = NPOS) on that image, read back as int8
+//   (|count| <= NPOS) and written to out.gsc in whole rows; after a third barrier CTA c adds rows c, c + G, ...
+//   of all the tiles' Grams (warps over the tiles, lanes over the row, then the warps' sums in shared memory) to
+//   out.gram's upper triangle (integer sums: the order does not matter). With out.h (the weighted V^T H V of
+//   §2.5) the B operand is t_b(x) h(x) as a scaled fp16 hi + lo pair (two MMAs per K step), the tile Grams go to
+//   out.gsc as float32, and after the third barrier the warps of the grid sum them in a fixed order (one warp per
+//   16 entries of the upper triangle: 8 lane groups over the tiles, 4 entries per lane, then shuffles) into both
+//   triangles of out.gramf.
 template <int NPOS, int MODE>
 __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* __restrict__ op, int w,
                                                                 const float* __restrict__ part, int splits, int L,
@@ -115,54 +119,69 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int x0 = blockIdx.x * NPOS;
-  if (tid == 0) {
-    mbar_init(smem_addr(&op_bar), 1);
-    mbar_init(smem_addr(&done_bar), 1);
-    fence_barrier_init();
-    mbar_expect_tx(smem_addr(&op_bar), kOpBytes);
-#pragma unroll
-    for (uint32_t c = 0; c < kOpBytes / kOpCopy; ++c) bulk_copy(a_hi + c * kOpCopy, op + c * kOpCopy, kOpCopy, smem_addr(&op_bar));
-  }
-  if (warp == 0) {
-    tmem_alloc(smem_addr(&tmem_slot), kCols);
-    tmem_relinquish();
-  }
-  const int sg = __ldg(reinterpret_cast<const int*>(op + kOpBytes));
 
-  // ---- P tile: thread (pair xp, group bq) sums, slot by slot in order, P[kBper bq + j][x0 + 2 xp + c]
+  // ---- P tile: the slots go to shared memory by cp.async, kStage slots in flight at once (16, 8 or 4 bytes a
+  //      copy, as L's alignment allows; positions past L zero-filled); then thread (pair xp, group bq) sums,
+  //      slot by slot in order, P[kBper bq + j][x0 + 2 xp + c]
+  const int sg = __ldg(reinterpret_cast<const int*>(op + kOpBytes));
   const int xp = tid % C::kPairs, bq = tid / C::kPairs;
-  const int xa = x0 + 2 * xp;
   float pv[C::kBper][2];
 #pragma unroll
   for (int j = 0; j < C::kBper; ++j) pv[j][0] = pv[j][1] = 0.f;
   {
-    const bool vec2 = (L & 1) == 0 && xa + 1 < L;
+    const uint32_t pst = sbase + kOpBytes + 4 * C::kAtomB;
+    const float* const pstg = reinterpret_cast<const float*>(gbase + kOpBytes + 4 * C::kAtomB);
+    const int vw = (L & 3) == 0 ? 4 : ((L & 1) == 0 ? 2 : 1);
+    const int per_row = NPOS / vw, step = 256 / per_row;
+    const int q = tid % per_row, r0 = tid / per_row;
+    const int xq = x0 + q * vw;
+    const bool xin = xq < L;
+    const uint32_t nbytes = xin ? 4u * (uint32_t)vw : 0u;
     const long long sstride = (long long)w * L;
-    for (int s0 = 0; s0 < splits; s0 += C::kSlotUnroll) {
-      float2 v[C::kSlotUnroll][C::kBper];
+    auto stage = [&](int s0, int ns) {
+      for (int u = 0; u < ns; ++u)
+        for (int b = r0; b < w; b += step) {
+          const float* src = part + (s0 + u) * sstride + (long long)b * L + (xin ? xq : 0);
+          const uint32_t dst = pst + 4u * (uint32_t)((u * kWp + b) * NPOS + q * vw);
+          if (vw == 4)
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(nbytes) : "memory");
+          else if (vw == 2)
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src), "r"(nbytes) : "memory");
+          else
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(nbytes) : "memory");
+        }
+    };
+    stage(0, min(C::kStage, splits));
+    // the operand image, the barriers and the tensor memory while the first group is in flight
+    if (tid == 0) {
+      mbar_init(smem_addr(&op_bar), 1);
+      mbar_init(smem_addr(&done_bar), 1);
+      fence_barrier_init();
+      mbar_expect_tx(smem_addr(&op_bar), kOpBytes);
 #pragma unroll
-      for (int u = 0; u < C::kSlotUnroll; ++u)
+      for (uint32_t c = 0; c < kOpBytes / kOpCopy; ++c)
+        bulk_copy(a_hi + c * kOpCopy, op + c * kOpCopy, kOpCopy, smem_addr(&op_bar));
+    }
+    if (warp == 0) {
+      tmem_alloc(smem_addr(&tmem_slot), kCols);
+      tmem_relinquish();
+    }
+    for (int s0 = 0; s0 < splits; s0 += C::kStage) {
+      const int ns = min(C::kStage, splits - s0);
+      if (s0 > 0) stage(s0, ns);
+      asm volatile("cp.async.wait_all;" ::: "memory");
+      __syncthreads();
+      for (int u = 0; u < ns; ++u)
 #pragma unroll
         for (int j = 0; j < C::kBper; ++j) {
           const int b = C::kBper * bq + j;
-          v[u][j] = make_float2(0.f, 0.f);
-          if (b < w && s0 + u < splits) {
-            const float* src = part + (s0 + u) * sstride + (long long)b * L + xa;
-            if (vec2) {
-              v[u][j] = __ldg(reinterpret_cast<const float2*>(src));
-            } else {
-              v[u][j].x = xa < L ? __ldg(src) : 0.f;
-              v[u][j].y = xa + 1 < L ? __ldg(src + 1) : 0.f;
-            }
+          if (b < w) {
+            const float2 v = *reinterpret_cast<const float2*>(pstg + (u * kWp + b) * NPOS + 2 * xp);
+            pv[j][0] += v.x;
+            pv[j][1] += v.y;
           }
         }
-#pragma unroll
-      for (int u = 0; u < C::kSlotUnroll; ++u)
-#pragma unroll
-        for (int j = 0; j < C::kBper; ++j) {
-          pv[j][0] += v[u][j].x;
-          pv[j][1] += v[u][j].y;
-        }
+      __syncthreads();   // the stage is free for the next group
     }
   }
   // ---- 2^sp from max |P| of the tile; B row 2 xp + c, 8-byte quarter-chunk groups of 4 b
@@ -314,6 +333,8 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
     uint8_t* const ts = gbase;   // the tile's trits as a K-major fp16 operand (rows a): the free A region
     uint8_t* const th_hi = gbase + 16384u;   // weighted: t h 2^sh as fp16 hi / lo, the same layout
     uint8_t* const th_lo = gbase + 32768u;
+    uint8_t* const gst = gbase + 16384u;     // unweighted: the tile's int8 Gram, 128 rows x 128 B
+    uint8_t* const tks = gbase + 49152u;     // Tk's position rows for the tile, NPOS x 128 fp16
     const bool wgram = out.h != nullptr, anyg = wgram || out.gram != nullptr;
     int sh = 0;
     if (wgram) {   // 2^sh from the tile's largest weight
@@ -351,37 +372,13 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
       for (int e = 0; e < 4; ++e)
         h[e] = (uint32_t)__half_as_ushort(__short2half_rn(t[2 * e])) |
                ((uint32_t)__half_as_ushort(__short2half_rn(t[2 * e + 1])) << 16);
-      if (a < w) {
-        int8_t* Tr = out.T + (long long)a * out.ldt + xb;
-        __half* Hr = out.T16 != nullptr ? out.T16 + (long long)a * out.ldt16 + xb : nullptr;
-        if (xb + 7 < L) {
-          uint32_t b0 = 0u, b1 = 0u;
+      if (out.Tk != nullptr) {   // the K-major copy: position rows of 128 components, staged
+        __half* const tr = reinterpret_cast<__half*>(tks) + col * kWp + a;
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            b0 |= (uint32_t)(uint8_t)t[i] << (8 * i);
-            b1 |= (uint32_t)(uint8_t)t[4 + i] << (8 * i);
-          }
-          *reinterpret_cast<uint2*>(Tr) = make_uint2(b0, b1);
-          if (Hr != nullptr) *reinterpret_cast<uint4*>(Hr) = make_uint4(h[0], h[1], h[2], h[3]);
-        } else {
-#pragma unroll
-          for (int i = 0; i < 8; ++i)
-            if (xb + i < L) {
-              Tr[i] = (int8_t)t[i];
-              if (Hr != nullptr) Hr[i] = __short2half_rn(t[i]);
-            }
-        }
+        for (int i = 0; i < 8; ++i) tr[i * kWp] = __short2half_rn(t[i]);
       }
-      // position rows of the K-major copy (the warp's 32 components are 64 contiguous bytes), with zeros up to the
-      // next multiple of 8 components
-      if (out.Tk != nullptr && a < ((w + 7) & ~7) && a < out.ldk) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          if (xb + i < L) out.Tk[(long long)(xb + i) * out.ldk + a] = __short2half_rn(t[i]);
-      }
-      if (anyg)
-        *reinterpret_cast<uint4*>(ts + k_major_offset(128u, (uint32_t)a, (uint32_t)col)) =
-            make_uint4(h[0], h[1], h[2], h[3]);
+      *reinterpret_cast<uint4*>(ts + k_major_offset(128u, (uint32_t)a, (uint32_t)col)) =
+          make_uint4(h[0], h[1], h[2], h[3]);
       if (wgram) {
         float v[8];
 #pragma unroll
@@ -393,12 +390,11 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
         *reinterpret_cast<uint4*>(th_lo + off) = make_uint4(hl[0], hl[1], hl[2], hl[3]);
       }
     }
-    if (anyg) {
-      fence_async_shared();
-      tc_fence_before();
-      __syncthreads();
-      tc_fence_after();
-      if (tid == 0) {
+    fence_async_shared();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (anyg && tid == 0) {
         const uint32_t idesc = f16_idesc((uint32_t)kWp, (uint32_t)kWp);
 #pragma unroll
         for (int kk = 0; kk < NPOS / 16; ++kk) {
@@ -411,8 +407,56 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
           }
         }
         mma_commit(smem_addr(&done_bar));
+    }
+    __syncwarp();
+    {   // T and T16 rows from the staged trits, NPOS / 8 lanes per row (16 bytes of fp16 trits each): full rows
+      constexpr int kCh = NPOS / 8, kRows = 32 / kCh;
+      const int c = lane % kCh, xb = x0 + 8 * c;
+      for (int r = warp * kRows + lane / kCh; r - lane / kCh < w; r += 8 * kRows) {
+        if (r >= w || xb >= L) continue;
+        const uint4 hv = *reinterpret_cast<const uint4*>(ts + k_major_offset(128u, (uint32_t)r, 8u * (uint32_t)c));
+        const uint32_t hw4[4] = {hv.x, hv.y, hv.z, hv.w};
+        uint32_t b[2] = {0u, 0u};
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int v = (int)__half2short_rz(__ushort_as_half((unsigned short)(hw4[i >> 1] >> (16 * (i & 1)))));
+          b[i >> 2] |= (uint32_t)(uint8_t)(int8_t)v << (8 * (i & 3));
+        }
+        int8_t* Tr = out.T + (long long)r * out.ldt + xb;
+        __half* Hr = out.T16 != nullptr ? out.T16 + (long long)r * out.ldt16 + xb : nullptr;
+        if (xb + 7 < L) {
+          *reinterpret_cast<uint2*>(Tr) = make_uint2(b[0], b[1]);
+          if (Hr != nullptr) *reinterpret_cast<uint4*>(Hr) = hv;
+        } else {
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (xb + i < L) {
+              Tr[i] = (int8_t)(b[i >> 2] >> (8 * (i & 3)));
+              if (Hr != nullptr) Hr[i] = __ushort_as_half((unsigned short)(hw4[i >> 1] >> (16 * (i & 1))));
+            }
+        }
       }
-      __syncwarp();
+    }
+    if (out.Tk != nullptr) {   // Tk rows x (components up to the next multiple of 8, zeros past w), 16 lanes a row
+      const int lim = min((w + 7) & ~7, (int)min(out.ldk, (long long)kWp));
+      const bool vec = (out.ldk & 7) == 0 && (reinterpret_cast<uintptr_t>(out.Tk) & 15) == 0;
+      const int c8 = lane & 15;
+      for (int pr = 2 * warp + (lane >> 4); pr - (lane >> 4) < NPOS; pr += 16) {
+        const int x = x0 + pr;
+        if (x >= L || 8 * c8 >= lim) continue;
+        const uint4 v = *reinterpret_cast<const uint4*>(tks + pr * (2 * kWp) + 16 * c8);
+        __half* dst = out.Tk + (long long)x * out.ldk + 8 * c8;
+        if (vec && 8 * c8 + 8 <= lim) {
+          *reinterpret_cast<uint4*>(dst) = v;
+        } else {
+          const uint32_t vv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (8 * c8 + i < lim) dst[i] = __ushort_as_half((unsigned short)(vv[i >> 1] >> (16 * (i & 1))));
+        }
+      }
+    }
+    if (anyg) {
       const bool gok = mbar_wait(smem_addr(&done_bar), 1u, err);
       const bool have = __all_sync(0xffffffffu, gok) != 0;
       tc_fence_after();
@@ -432,8 +476,8 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
                               __uint_as_float(g[i + 2]) * ih, __uint_as_float(g[i + 3]) * ih);
           }
         }
-      } else if (have) {   // row a, columns 64 hpos .. + 63 of the tile's Gram (the loads are warp-collective)
-        int8_t* dst = out.gsc + ((long long)blockIdx.x * kWp + a) * kWp + 64 * hpos;
+      } else if (have) {   // row a, columns 64 hpos .. + 63 of the tile's Gram as int8 in shared memory, 16-byte
+        // chunks swizzled by row (the loads are warp-collective)
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           uint32_t g[16];
@@ -446,25 +490,66 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
 #pragma unroll
             for (int i = 0; i < 4; ++i) pk[e] |= ((uint32_t)(int)__uint_as_float(g[4 * e + i]) & 0xffu) << (8 * i);
           }
-          if (a < w) *reinterpret_cast<uint4*>(dst + 16 * c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          *reinterpret_cast<uint4*>(gst + a * 128 + (((4 * hpos + c) ^ (a & 7)) << 4)) =
+              make_uint4(pk[0], pk[1], pk[2], pk[3]);
         }
       }
-      ok = grid_barrier(bar + 2, G, err);
-      if (ok) {
-        if (blockIdx.x == 0 && tid == 0) bar[1] = 0u;   // everyone has left barrier 2
-        // tasks: (row a, 16 columns from 16 u) for u = a / 16 .. cdiv(w, 16) - 1, rows in order; lane (q, j)
-        // sums entries (a, 16 u + 4 j .. + 3) of the tiles q, q + 8, ...
-        const int ng = (w + 15) >> 4, w16 = w >> 4, q = lane >> 2, j = lane & 3;
-        const int ntask = ng * w - 16 * (w16 * (w16 - 1) / 2) - (w & 15) * w16;
-        for (int task = (int)blockIdx.x * 8 + warp; task < ntask; task += (int)G * 8) {
-          int ra = 0, t = task;
-          for (; ra < w; ++ra) {
-            const int n = ng - (ra >> 4);
-            if (t < n) break;
-            t -= n;
+      if (!wgram) {   // integer: the tile's Gram to out.gsc in whole rows; after a third barrier CTA c adds up rows
+        // c, c + G, ... of all tiles (warp q takes tiles q, q + 8, ..., lane j entries 4j .. 4j + 3) into out.gram
+        __syncthreads();
+        int8_t* const gt = out.gsc + (long long)blockIdx.x * (kWp * kWp);
+#pragma unroll
+        for (int it = 0; it < 4; ++it) {
+          const int r = 32 * it + (tid >> 3), c16 = tid & 7;
+          *reinterpret_cast<uint4*>(gt + r * kWp + 16 * c16) =
+              *reinterpret_cast<const uint4*>(gst + r * 128 + ((c16 ^ (r & 7)) << 4));
+        }
+        ok = grid_barrier(bar + 2, G, err);
+        if (ok) {
+          if (blockIdx.x == 0 && tid == 0) bar[1] = 0u;   // everyone has left barrier 2
+          int* const rsum = reinterpret_cast<int*>(gst);   // 8 warps x 128 entries
+          for (int ra = (int)blockIdx.x; ra < w; ra += (int)G) {
+            int acc[4] = {0, 0, 0, 0};
+            const int8_t* src = out.gsc + (long long)ra * kWp + 4 * lane;
+            for (int c0 = warp; c0 < (int)G; c0 += 8 * 16) {
+              unsigned v[16];
+#pragma unroll
+              for (int k = 0; k < 16; ++k) {
+                const int c = c0 + 8 * k;
+                v[k] = c < (int)G ? __ldcg(reinterpret_cast<const unsigned*>(src + (long long)c * (kWp * kWp))) : 0u;
+              }
+#pragma unroll
+              for (int k = 0; k < 16; ++k)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc[i] += (int)(int8_t)(v[k] >> (8 * i));
+            }
+            *reinterpret_cast<int4*>(rsum + warp * kWp + 4 * lane) = make_int4(acc[0], acc[1], acc[2], acc[3]);
+            __syncthreads();
+            if (tid < w && tid >= ra) {
+              int tot = 0;
+#pragma unroll
+              for (int q = 0; q < 8; ++q) tot += rsum[q * kWp + tid];
+              if (tot != 0) out.gram[(long long)ra * w + tid] += tot;
+            }
+            __syncthreads();
           }
-          const int b0 = 16 * ((ra >> 4) + t) + 4 * j;
-          if (wgram) {   // float32 tiles, 12 loads of 16 bytes in flight per lane
+        }
+      } else {   // weighted: float32 tile Grams, summed in a fixed order after a third barrier
+        ok = grid_barrier(bar + 2, G, err);
+        if (ok) {
+          if (blockIdx.x == 0 && tid == 0) bar[1] = 0u;   // everyone has left barrier 2
+          // tasks: (row a, 16 columns from 16 u) for u = a / 16 .. cdiv(w, 16) - 1, rows in order; lane (q, j)
+          // sums entries (a, 16 u + 4 j .. + 3) of the tiles q, q + 8, ..., 12 loads of 16 bytes in flight
+          const int ng = (w + 15) >> 4, w16 = w >> 4, q = lane >> 2, j = lane & 3;
+          const int ntask = ng * w - 16 * (w16 * (w16 - 1) / 2) - (w & 15) * w16;
+          for (int task = (int)blockIdx.x * 8 + warp; task < ntask; task += (int)G * 8) {
+            int ra = 0, t = task;
+            for (; ra < w; ++ra) {
+              const int n = ng - (ra >> 4);
+              if (t < n) break;
+              t -= n;
+            }
+            const int b0 = 16 * ((ra >> 4) + t) + 4 * j;
             const float* srcf = reinterpret_cast<const float*>(out.gsc) + (long long)ra * kWp + b0;
             float facc[4] = {0.f, 0.f, 0.f, 0.f};
             for (int c0 = q; c0 < (int)G; c0 += 8 * 12) {
@@ -499,34 +584,6 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
                 }
               }
             }
-            continue;
-          }
-          const int8_t* src = out.gsc + (long long)ra * kWp + b0;
-          int acc[4] = {0, 0, 0, 0};
-          for (int c0 = q; c0 < (int)G; c0 += 8 * 24) {
-            unsigned v[24];
-#pragma unroll
-            for (int k = 0; k < 24; ++k) {
-              const int c = c0 + 8 * k;
-              v[k] = c < (int)G ? __ldcg(reinterpret_cast<const unsigned*>(src + (long long)c * kWp * kWp)) : 0u;
-            }
-#pragma unroll
-            for (int k = 0; k < 24; ++k)
-#pragma unroll
-              for (int i = 0; i < 4; ++i) acc[i] += (int)(int8_t)(v[k] >> (8 * i));
-          }
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], 4);
-            acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], 8);
-            acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], 16);
-          }
-          if (q == 0) {
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const int b = b0 + i;
-              if (b >= ra && b < w && acc[i] != 0) atomicAdd(out.gram + (long long)ra * w + b, acc[i]);
-            }
           }
         }
       }
@@ -539,7 +596,7 @@ __global__ void __launch_bounds__(256, 1) decorrelate_tc_kernel(const uint8_t* _
     tmem_dealloc(tmem, kCols);
   }
   if (!ok) return;
-  if (tid == 0) {   // exit ticket: the last CTA resets the words still set (barrier 2 without a Gram)
+  if (tid == 0) {   // exit ticket: the last CTA resets the words still set (barrier 2 without the weighted Gram)
     unsigned old;
     asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(bar + 3) : "memory");
     if (old == G - 1u) {
@@ -645,7 +702,7 @@ cudaError_t launch_decorrelate_apply_tc(const void* op, int w, const float* part
   if ((h == nullptr) != (gramf == nullptr) || (h != nullptr && (gram != nullptr || gsc == nullptr)))
     return cudaErrorInvalidValue;
   if (!decorrelate_apply_tc_fits(w, L) || st.nchunk != (int)cdiv(L, npos) || op == nullptr || err == nullptr ||
-      (gram != nullptr && (gsc == nullptr || (reinterpret_cast<uintptr_t>(gsc) & 15) != 0)) ||
+      ((gram != nullptr || h != nullptr) && (gsc == nullptr || (reinterpret_cast<uintptr_t>(gsc) & 15) != 0)) ||
       bar == nullptr || T == nullptr || (reinterpret_cast<uintptr_t>(op) & 15) != 0 || (ldt & 7) != 0 ||
       (reinterpret_cast<uintptr_t>(T) & 7) != 0 ||
       (T16 != nullptr && ((ldt16 & 7) != 0 || (reinterpret_cast<uintptr_t>(T16) & 15) != 0)) ||

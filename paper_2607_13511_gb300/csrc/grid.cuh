@@ -14,12 +14,12 @@ __device__ __forceinline__ unsigned long long grid_ns() {
 }
 
 // Grid barrier on ctr: every CTA adds one (release) and polls until the count reaches target (acquire);
-// false after a timeout (then err holds 1).
+// false after a timeout (then err holds 1). The CTA barrier before the release and after the acquire carries the
+// ordering to the other threads of the CTA (release and acquire are cumulative), so no separate fences.
 __device__ __forceinline__ bool grid_barrier(unsigned* ctr, unsigned target, unsigned* err) {
   __shared__ int s_ok;
   __syncthreads();
   if (threadIdx.x == 0) {
-    __threadfence();
     asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
     int ok = 1;
     const unsigned long long t0 = grid_ns();
@@ -33,7 +33,6 @@ __device__ __forceinline__ bool grid_barrier(unsigned* ctr, unsigned target, uns
         break;
       }
     }
-    __threadfence();
     s_ok = ok;
   }
   __syncthreads();
