@@ -331,22 +331,51 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
   }
 }
 
-__global__ void norm_kernel(const F2* __restrict__ part, int count, double* out, const double* norm_a, double* trace,
-                            const float* __restrict__ maxpart, float* maxout) {
+// One CTA of 1024 threads: thread t adds the partials t, t + 1024, ... (all its loads issued before the first
+// addition), then the warps' sums combine by shuffles and the 32 warp sums in warp order: a fixed order, so the
+// result is the same on every run.
+__global__ void __launch_bounds__(1024) norm_kernel(const F2* __restrict__ part, int count, double* out,
+                                                    const double* norm_a, double* trace,
+                                                    const float* __restrict__ maxpart, float* maxout) {
+  constexpr int kBatch = 8;
+  __shared__ F2 red_s[32];
+  __shared__ float red_m[32];
   F2 s;
   float mx = 0.f;
-  for (int i = threadIdx.x; i < count; i += 32) {
-    s = f2_add(s, part[i]);
-    if (maxpart != nullptr) mx = fmaxf(mx, maxpart[i]);
+  for (int i0 = threadIdx.x; i0 < count; i0 += 1024 * kBatch) {
+    F2 v[kBatch];
+    float m[kBatch];
+#pragma unroll
+    for (int b = 0; b < kBatch; ++b) {
+      const int i = i0 + 1024 * b;
+      v[b] = i < count ? part[i] : F2{};
+      m[b] = (maxpart != nullptr && i < count) ? maxpart[i] : 0.f;
+    }
+#pragma unroll
+    for (int b = 0; b < kBatch; ++b) {
+      s = f2_add(s, v[b]);
+      mx = fmaxf(mx, m[b]);
+    }
   }
   s = warp_sum(s);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  if ((threadIdx.x & 31) == 0) {
+    red_s[threadIdx.x >> 5] = s;
+    red_m[threadIdx.x >> 5] = mx;
+  }
+  __syncthreads();
   if (threadIdx.x == 0) {
-    const double v = f2_value(s);
+    F2 t = red_s[0];
+    float tm = red_m[0];
+    for (int q = 1; q < 32; ++q) {
+      t = f2_add(t, red_s[q]);
+      tm = fmaxf(tm, red_m[q]);
+    }
+    const double v = f2_value(t);
     out[0] = v;
     if (trace != nullptr) trace[0] = 1.0 - v / norm_a[0];
-    if (maxout != nullptr) maxout[0] = mx;
+    if (maxout != nullptr) maxout[0] = tm;
   }
 }
 
@@ -514,7 +543,7 @@ cudaError_t launch_select_with(const float* colpart, int nrt, int n, const float
 
 cudaError_t launch_norm(const F2* normpart, int count, double* out, const double* norm_a, double* trace,
                         cudaStream_t s, const float* maxpart, float* maxout) {
-  norm_kernel<<<1, 32, 0, s>>>(normpart, count, out, norm_a, trace, maxpart, maxout);
+  norm_kernel<<<1, 1024, 0, s>>>(normpart, count, out, norm_a, trace, maxpart, maxout);
   return cudaGetLastError();
 }
 
