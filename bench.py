@@ -50,7 +50,7 @@ JOBS["decoder36"] = list(W.decoder_conversion())
 # dram__bytes_read.sum + dram__bytes_write.sum per launch of the profiled kernel, from one ncu capture, valid
 # only while the kernel's source is unchanged (sha256 of the file that holds it).
 NCU_TRAFFIC: dict = {
-    # profiles/residual_products_up2560x9728.md: V-step 100.39 + 3.43 MB, U-step 102.15 + 3.15 MB per launch
+    # ncu --set full of product_tma_kernel on this workload: V-step 100.39 + 3.43 MB, U-step 102.15 + 3.15 MB
     "kind": "products", "file": "product_tma.cu", "sha": "7746e0aa82c2a97b", "workload": "up2560x9728_t5_mu3_tau1_b128",
     "bytes_per_launch": (100.387840e6 + 3.434752e6 + 102.153216e6 + 3.150336e6) / 2,
 }
