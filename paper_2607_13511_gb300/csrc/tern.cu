@@ -13,26 +13,15 @@ namespace externd {
 
 namespace {
 
-// Per-chunk statistics of vector a over positions [x0, x0 + 128): optionally gathering x = R[r][J[a]].
-template <bool GATHER>
-__global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X, int L, long long ldx, int ncols,
-                                                    const int* __restrict__ J, float* __restrict__ Y, long long ldy,
-                                                    Stats st) {
+// Per-chunk statistics of vector a over positions [x0, x0 + 128).
+__global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X, int L, long long ldx, Stats st) {
   __shared__ F2 ssum[4];
   __shared__ u64 skey[4];
   const int a = blockIdx.y;
   const int x = blockIdx.x * kStatChunk + threadIdx.x;
   float v = 0.f;
   bool valid = x < L;
-  if (valid) {
-    if (GATHER) {
-      const int j = min(max(__ldg(J + a), 0), ncols - 1);   // J comes from select_kernel; never read outside R
-      v = __ldg(X + (long long)x * ncols + j);
-      Y[(long long)a * ldy + x] = v;
-    } else {
-      v = __ldg(X + (long long)a * ldx + x);
-    }
-  }
+  if (valid) v = __ldg(X + (long long)a * ldx + x);
   F2 s;
   s.hi = valid ? fabsf(v) : 0.f;
   u64 key = valid ? mag_key(v, (uint32_t)x) : 0ull;
@@ -55,6 +44,45 @@ __global__ void __launch_bounds__(128) stats_kernel(const float* __restrict__ X,
     put_stat(st, a, blockIdx.x, t, k);
   }
   stats_done(st, gridDim.y);
+}
+
+// The block start's gather with the per-chunk statistics: Y[a][x] = R[x][J[a]] for one 128-position chunk per
+// warp (lanes take positions x0 + lane + 32k, k < 4, the four gathers in flight together), 8 warps per CTA over
+// the nv * cdiv(L, 128) (vector, chunk) items, so that few CTAs take the finalize ticket.
+__global__ void __launch_bounds__(256) gather_stats_kernel(const float* __restrict__ R, int L, int ncols,
+                                                           const int* __restrict__ J, float* __restrict__ Y,
+                                                           long long ldy, int nv, Stats st) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nchunk = (L + kStatChunk - 1) / kStatChunk;
+  const long long items = (long long)nv * nchunk;
+  for (long long it = (long long)blockIdx.x * 8 + warp; it < items; it += (long long)gridDim.x * 8) {
+    const int a = (int)(it / nchunk), ch = (int)(it - (long long)a * nchunk);
+    const int j = min(max(__ldg(J + a), 0), ncols - 1);   // J comes from select_kernel; never read outside R
+    float v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int x = ch * kStatChunk + lane + 32 * k;
+      v[k] = x < L ? __ldg(R + (long long)x * ncols + j) : 0.f;
+    }
+    F2 s;
+    u64 key = 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int x = ch * kStatChunk + lane + 32 * k;
+      if (x < L) {
+        Y[(long long)a * ldy + x] = v[k];
+        F2 t;
+        t.hi = fabsf(v[k]);
+        s = f2_add(s, t);
+        const u64 kk = mag_key(v[k], (uint32_t)x);
+        key = kk > key ? kk : key;
+      }
+    }
+    s = warp_sum(s);
+    key = warp_max(key);
+    if (lane == 0) put_stat(st, a, ch, s, key);
+  }
+  stats_done(st, nv);
 }
 
 // T = T_tau(X) for up to 256 vectors per CTA over positions [x0, x0 + P), in 64-position chunks. Each warp
@@ -264,13 +292,25 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
   const int tid = threadIdx.x;
   const int per = (int)cdiv(n, 1024);
   const int cb = min(n, tid * per), ce = min(n, cb + per);
+  // the thread's keys stay in registers across the passes when they number at most kKeep (n <= 16384)
+  constexpr int kKeep = 16;
+  const bool keep = per <= kKeep;
+  unsigned kr[kKeep];
+#pragma unroll
+  for (int i = 0; i < kKeep; ++i) kr[i] = (keep && cb + i < ce) ? __float_as_uint(e[cb + i]) : 0u;
   unsigned prefix = 0, mask = 0, remaining = (unsigned)w;
   for (int shift = 24; shift >= 0; shift -= 8) {
     for (int i = tid; i < 256; i += 1024) hist[i] = 0;
     __syncthreads();
-    for (int c = cb; c < ce; ++c) {
-      const unsigned key = __float_as_uint(e[c]);
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    if (keep) {
+#pragma unroll
+      for (int i = 0; i < kKeep; ++i)
+        if (cb + i < ce && (kr[i] & mask) == prefix) atomicAdd(&hist[(kr[i] >> shift) & 255u], 1u);
+    } else {
+      for (int c = cb; c < ce; ++c) {
+        const unsigned key = __float_as_uint(e[c]);
+        if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+      }
     }
     __syncthreads();
     if (tid < 32) {
@@ -309,26 +349,34 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
     __syncthreads();
   }
   // prefix = key of the w-th largest; take every key above it and the first `remaining` keys equal to it.
+  // visit(f) calls f(c, key) for the thread's columns in order (keys from registers when kept)
+  auto visit = [&](auto&& f) {
+    if (keep) {
+#pragma unroll
+      for (int i = 0; i < kKeep; ++i)
+        if (cb + i < ce) f(cb + i, kr[i]);
+    } else {
+      for (int c = cb; c < ce; ++c) f(c, __float_as_uint(e[c]));
+    }
+  };
   int eq = 0;
-  for (int c = cb; c < ce; ++c) eq += (__float_as_uint(e[c]) == prefix);
+  visit([&](int, unsigned key) { eq += key == prefix; });
   int eq_before = block_scan_incl(eq, scan_sh) - eq;
   int sel = 0;
   {
     int e_seen = eq_before;
-    for (int c = cb; c < ce; ++c) {
-      const unsigned key = __float_as_uint(e[c]);
+    visit([&](int, unsigned key) {
       if (key > prefix) ++sel;
       else if (key == prefix) sel += (unsigned)(e_seen++) < remaining;
-    }
+    });
   }
   int pos = block_scan_incl(sel, scan_sh) - sel;
   int e_seen = eq_before;
-  for (int c = cb; c < ce; ++c) {
-    const unsigned key = __float_as_uint(e[c]);
+  visit([&](int c, unsigned key) {
     bool take = key > prefix;
     if (key == prefix) take = (unsigned)(e_seen++) < remaining;
     if (take) J[pos++] = c;
-  }
+  });
 }
 
 // One CTA of 1024 threads: thread t adds the partials t, t + 1024, ... (all its loads issued before the first
@@ -457,14 +505,22 @@ __global__ void sum_splits_kernel(const float* __restrict__ part, int splits, in
 
 cudaError_t launch_stats(const float* X, int nv, int L, int ldx, Stats st, cudaStream_t s) {
   dim3 grid((unsigned)cdiv(L, kStatChunk), (unsigned)nv);
-  stats_kernel<false><<<grid, kStatChunk, 0, s>>>(X, L, ldx, 0, nullptr, nullptr, 0, st);
+  stats_kernel<<<grid, kStatChunk, 0, s>>>(X, L, ldx, st);
   return cudaGetLastError();
 }
 
 cudaError_t launch_gather(const float* R, int m, int n, const int* J, int w, float* Y, int ldy, Stats st,
                           cudaStream_t s) {
-  dim3 grid((unsigned)cdiv(m, kStatChunk), (unsigned)w);
-  stats_kernel<true><<<grid, kStatChunk, 0, s>>>(R, m, 0, n, J, Y, ldy, st);
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0, v = 0;
+    sms = (cudaGetDevice(&dev) == cudaSuccess &&
+           cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && v > 0) ? v : 148;
+    cudaGetLastError();
+  }
+  const long long items = (long long)w * cdiv(m, kStatChunk);
+  const long long grid = std::max<long long>(1, std::min<long long>(cdiv(items, 8), 2LL * sms));
+  gather_stats_kernel<<<(unsigned)grid, 256, 0, s>>>(R, m, n, J, Y, ldy, w, st);
   return cudaGetLastError();
 }
 
