@@ -31,6 +31,9 @@
 
 #include <algorithm>
 
+#include <cstdlib>
+#include <cstring>
+
 #include "kernels.h"
 #include "umma.cuh"
 
@@ -326,8 +329,8 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
       bool got = mbar_wait(full32 + 8u * s, (uint32_t)(k / p.s32) & 1u, p.err);
       ok = __all_sync(0xffffffffu, got) != 0;
       if (!ok) break;
-      // read the stage into registers and hand its slot back to the producer at once (the split below then
-      // overlaps the next copies), then wait for the A slot the split writes into
+      // read the stage into registers and hand its slot back to the producer (the split below then overlaps the
+      // next copies), then wait for the A slot the split writes into
       const uint8_t* st = gbase + (r32 - sbase) + (size_t)s * kStage32;
       const int y0 = (STREAM ? kc : kc + k) * kStageK;
       float v[kItems][8];
@@ -347,6 +350,10 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
           v[q][4] = b.x; v[q][5] = b.y; v[q][6] = b.z; v[q][7] = b.w;
         }
       }
+      // hand the stage back: the next copy into it is an async-proxy write, so this thread's generic loads from
+      // it are ordered before that write by a proxy fence (without it a lane's loads could still be in flight
+      // when the copy landed, and one row of the partials took values of a later stage)
+      fence_async_shared();
       __syncwarp();
       if (lane == 0) mbar_arrive(empty32 + 8u * s);
       got = k < p.s16 || mbar_wait(empty16 + 8u * s16, (uint32_t)(k / p.s16 - 1) & 1u, p.err);
@@ -462,7 +469,11 @@ TmaWork tma_work(int w, int Lx, int Ly) {
   TmaWork t{0, nkt, chunk / kStageK, sp, tiles, sp, (long long)tiles * nkt};
   // SMs left to the product: the w x w inverse of the same half-step holds one (single CTA) or a cluster's worth
   const long long G = sms - std::max(1, inverse_cluster_size(w));
-  if ((long long)tiles * sp > G && G >= 1 && t.U >= G) {
+  static const bool stream_ok = [] {
+    const char* e = std::getenv("EXTERND_STREAMK");
+    return !(e && std::strcmp(e, "0") == 0);
+  }();
+  if (stream_ok && (long long)tiles * sp > G && G >= 1 && t.U >= G) {
     int S = 0;
     for (long long tt = 0; tt < tiles; ++tt) {
       const long long a = tt * nkt, b = a + nkt - 1;

@@ -66,7 +66,8 @@ __device__ __forceinline__ void fence_barrier_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
 
-// Makes this thread's generic-proxy shared-memory writes visible to the tensor core's async proxy.
+// Orders this thread's generic-proxy shared-memory accesses before later async-proxy ones: its writes become
+// visible to the tensor core, and its reads of a buffer complete before a bulk copy refills the buffer.
 __device__ __forceinline__ void fence_async_shared() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 // ---- tensor memory

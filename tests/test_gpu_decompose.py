@@ -112,6 +112,18 @@ def test_repeatable_and_graph_replay(X):
     assert torch.equal(r1.B, r2.B) and torch.equal(r1.C, r2.C) and torch.equal(r1.D, r2.D)
 
 
+def test_repeatable_at_full_size_tensor_core_path(X):
+    # 2560 x 9728, blocks of 128: the TMA products (stream-K, A in tensor memory) and the fused targets grid run
+    # every half-step. Every decision is taken in a fixed order, so repeated runs agree bit for bit.
+    wl = W.WORKLOADS["up2560x9728_t5_mu3_tau1_b128"]
+    A = cuda(wl.matrix())
+    ref = X.decompose_traced(A, wl.mu, wl.tau, wl.block, wl.iters)
+    for _ in range(3):
+        r = X.decompose_traced(A, wl.mu, wl.tau, wl.block, wl.iters)
+        assert r.trace == ref.trace
+        assert torch.equal(r.B, ref.B) and torch.equal(r.C, ref.C) and torch.equal(r.D, ref.D)
+
+
 def test_host_entry_point_matches_device(X):
     A = W.gaussian(200, 180, 0.02, 8)
     h = W.importance(180, 8)
