@@ -48,6 +48,7 @@ static_assert(kConv % 128 == 0 && kItems >= 1, "a converter thread keeps one pos
 constexpr int kProducerWarp = kConvWarps, kMmaWarp = kConvWarps + 1, kBWarp = kConvWarps + 2;
 constexpr int kThreads = (kConvWarps + 3) * 32;
 constexpr int kStageK = 64;
+constexpr int kS16 = 4, kSB = 4;   // A stages in tensor memory, ternary-tile slots (powers of two)
 constexpr uint32_t kAcols = 64u;               // TMEM columns of one stage's A operand: 64 fp16 hi + 64 lo per row
 constexpr uint32_t kStage32 = 128u * 64u * 4u;   // float32 R tile of one stage
 
@@ -103,11 +104,11 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
   const uint32_t tileB = (uint32_t)p.wpad * 128u;
   const uint32_t r32 = sbase;                                   // S32 x 32 KB
   const uint32_t rb = r32 + (uint32_t)p.s32 * kStage32;         // SB x tileB (1024-aligned: tileB = wpad * 128)
-  const uint32_t bars = rb + (uint32_t)round_up((long long)p.sb * tileB, 1024);
+  const uint32_t bars = rb + (uint32_t)round_up((long long)kSB * tileB, 1024);
   const uint32_t full32 = bars, empty32 = full32 + 8u * p.s32;
-  const uint32_t fullB = empty32 + 8u * p.s32, emptyB = fullB + 8u * p.sb;
-  const uint32_t full16 = emptyB + 8u * p.sb, empty16 = full16 + 8u * p.s16;
-  const uint32_t accfull = empty16 + 8u * p.s16, accempty = accfull + 16u;   // two TMEM accumulators
+  const uint32_t fullB = empty32 + 8u * p.s32, emptyB = fullB + 8u * kSB;
+  const uint32_t full16 = emptyB + 8u * kSB, empty16 = full16 + 8u * kS16;
+  const uint32_t accfull = empty16 + 8u * kS16, accempty = accfull + 16u;   // two TMEM accumulators
   const uint32_t tmem_slot = accempty + 16u;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -147,11 +148,11 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
       mbar_init(full32 + 8u * s, 1);
       mbar_init(empty32 + 8u * s, kConvWarps);
     }
-    for (int s = 0; s < p.sb; ++s) {
+    for (int s = 0; s < kSB; ++s) {
       mbar_init(fullB + 8u * s, 1);
       mbar_init(emptyB + 8u * s, 1);
     }
-    for (int s = 0; s < p.s16; ++s) {
+    for (int s = 0; s < kS16; ++s) {
       mbar_init(full16 + 8u * s, kConvWarps);
       mbar_init(empty16 + 8u * s, 1);
     }
@@ -224,14 +225,14 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
     if (lane == 0) {
       int k = 0;   // stages whose R copies were issued
       int t = (int)(u0 / p.nkt), kc = (int)(u0 - (long long)t * p.nkt);   // advanced without divisions
+      int s = 0, r = 0;                                                   // slot and round of stage k
       for (; k < nk; ++k) {
         if (STREAM && k > 0 && ++kc == p.nkt) {
           kc = 0;
           ++t;
         }
         const int x0 = t * 128, y0 = (STREAM ? kc : kc + k) * kStageK;   // a classic run stays in its tile
-        const int s = k % p.s32;
-        if (k >= p.s32 && !mbar_wait(empty32 + 8u * s, (uint32_t)(k / p.s32 - 1) & 1u, p.err)) break;
+        if (r > 0 && !mbar_wait(empty32 + 8u * s, (uint32_t)(r - 1) & 1u, p.err)) break;
         mbar_expect_tx(full32 + 8u * s, kStage32);
         if (!USTEP) {
 #pragma unroll
@@ -239,6 +240,10 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
         } else {
 #pragma unroll
           for (int b = 0; b < 2; ++b) tma_load_2d(r32 + s * kStage32 + b * 16384u, &mapR, y0 + 32 * b, x0, full32 + 8u * s);
+        }
+        if (++s == p.s32) {
+          s = 0;
+          ++r;
         }
       }
       // every copy this thread issued lands before the CTA can exit (bounded waits)
@@ -253,12 +258,12 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
       for (; k < nk; ++k) {
         if (STREAM && k > 0 && ++kc == p.nkt) kc = 0;
         const int y0 = (STREAM ? kc : kc + k) * kStageK;
-        const int sb = k % p.sb;
-        if (k >= p.sb && !mbar_wait(emptyB + 8u * sb, (uint32_t)(k / p.sb - 1) & 1u, p.err)) break;
+        const int sb = k & (kSB - 1);
+        if (k >= kSB && !mbar_wait(emptyB + 8u * sb, (uint32_t)(k / kSB - 1) & 1u, p.err)) break;
         mbar_expect_tx(fullB + 8u * sb, tileB);
         tma_load_2d(rb + sb * tileB, &mapT, y0, 0, fullB + 8u * sb);
       }
-      for (int j = max(0, k - p.sb); j < k; ++j) mbar_wait(fullB + 8u * (j % p.sb), (uint32_t)(j / p.sb) & 1u, p.err);
+      for (int j = max(0, k - kSB); j < k; ++j) mbar_wait(fullB + 8u * (j % kSB), (uint32_t)(j / kSB) & 1u, p.err);
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------------ MMA issuer
@@ -278,9 +283,9 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
             break;
           }
         }
-        const int s = k % p.s16, sb = k % p.sb;
-        if (!mbar_wait(full16 + 8u * s, (uint32_t)(k / p.s16) & 1u, p.err) ||
-            !mbar_wait(fullB + 8u * sb, (uint32_t)(k / p.sb) & 1u, p.err)) {
+        const int s = k & (kS16 - 1), sb = k & (kSB - 1);
+        if (!mbar_wait(full16 + 8u * s, (uint32_t)(k / kS16) & 1u, p.err) ||
+            !mbar_wait(fullB + 8u * sb, (uint32_t)(k / kSB) & 1u, p.err)) {
           ok = false;
           break;
         }
@@ -313,20 +318,30 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
     for (int j = 0; j < 8; ++j)
       voff[j] = (uint32_t)(x >> 5) * 8192u + (uint32_t)j * 128u + ((((uint32_t)(x & 31) >> 2) ^ (uint32_t)j) << 4) +
                 ((uint32_t)(x & 3) << 2);
-    int prev_tile = -1;
+    // a finished segment whose partials are still to be written (stream plan), and its tile
+    int pend = -1, pend_tile = -1;
     int t = (int)(u0 / p.nkt), kc = (int)(u0 - (long long)t * p.nkt);   // advanced without divisions
-    for (int k = 0; k < nk && ok; ++k) {
+    int s = 0, r = 0;                                                   // R slot and round of stage k
+    for (int k = 0; k < nk && ok; ++k, s = (s + 1 == p.s32) ? 0 : s + 1, r += (s == 0) ? 1 : 0) {
       if (STREAM && k > 0 && ++kc == p.nkt) {
         kc = 0;
         ++t;
       }
       if (k == 0 || (STREAM && kc == 0)) {
+        if (pend >= 0) {   // (only with segments shorter than the accumulator turnaround)
+          ok = epilogue(pend, pend_tile);
+          pend = -1;
+          if (!ok) break;
+        }
+        if (seg >= 0) {
+          pend = seg;
+          pend_tile = seg_tile;
+        }
         ++seg;
-        prev_tile = seg_tile;
         seg_tile = t;
       }
-      const int s = k % p.s32, s16 = k % p.s16;
-      bool got = mbar_wait(full32 + 8u * s, (uint32_t)(k / p.s32) & 1u, p.err);
+      const int s16 = k & (kS16 - 1);
+      bool got = mbar_wait(full32 + 8u * s, (uint32_t)r & 1u, p.err);
       ok = __all_sync(0xffffffffu, got) != 0;
       if (!ok) break;
       // read the stage into registers and hand its slot back to the producer (the split below then overlaps the
@@ -356,7 +371,7 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
       fence_async_shared();
       __syncwarp();
       if (lane == 0) mbar_arrive(empty32 + 8u * s);
-      got = k < p.s16 || mbar_wait(empty16 + 8u * s16, (uint32_t)(k / p.s16 - 1) & 1u, p.err);
+      got = k < kS16 || mbar_wait(empty16 + 8u * s16, (uint32_t)(k / kS16 - 1) & 1u, p.err);
       ok = __all_sync(0xffffffffu, got) != 0;
       if (!ok) break;
       tc_fence_after();   // the MMAs that read this A stage are complete: its columns may be rewritten
@@ -392,9 +407,16 @@ __global__ void __launch_bounds__(kThreads, 1) product_tma_kernel(const __grid_c
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(full16 + 8u * s16);
-      // the previous segment's partials, once this segment is fully converted (its MMAs are then queued)
-      const bool seg_end = k == nk - 1 || kc == p.nkt - 1;
-      if (STREAM && seg_end && seg >= 1) ok = epilogue(seg - 1, prev_tile);
+      // the previous segment's partials as soon as its MMAs have completed (checked without waiting after each
+      // stage, so that the copies keep streaming meanwhile), at the latest when this segment is converted
+      if (STREAM && pend >= 0) {
+        const bool seg_end = k == nk - 1 || kc == p.nkt - 1;
+        const bool done = __shfl_sync(0xffffffffu, lane == 0 && mbar_try_wait(accfull + 8u * (pend & 1), (uint32_t)(pend / 2) & 1u), 0);
+        if (done || seg_end) {
+          ok = epilogue(pend, pend_tile);
+          pend = -1;
+        }
+      }
     }
   }
   // the last segment (or zeros after a failure, so every partial slot is written), once every role is done
@@ -444,8 +466,8 @@ TmaPlan tma_plan(int w) {
   // from L2 but under a saturated HBM queue still take a microsecond or more: four B slots let them be requested
   // well ahead of the MMAs, so that neither the MMAs nor (through the A stages) the converters wait for them; the
   // rest of the space holds R in flight.
-  t.s16 = 4;
-  t.sb = 4;
+  t.s16 = kS16;
+  t.sb = kSB;
   const size_t budget = 227 * 1024 - 1024 - 512 - round_up((long long)t.sb * tileB, 1024);
   int s = 6;
   while (s > 1 && (size_t)s * kStage32 > budget) --s;
