@@ -50,9 +50,12 @@ JOBS["decoder36"] = list(W.decoder_conversion())
 # dram__bytes_read.sum + dram__bytes_write.sum per launch of the profiled kernel, from one ncu capture, valid
 # only while the kernel's source is unchanged (sha256 of the file that holds it).
 NCU_TRAFFIC: dict = {
-    # ncu --set full of product_tma_kernel on this workload: V-step 100.39 + 3.43 MB, U-step 102.15 + 3.15 MB
-    "kind": "products", "file": "product_tma.cu", "sha": "7746e0aa82c2a97b", "workload": "up2560x9728_t5_mu3_tau1_b128",
-    "bytes_per_launch": (100.387840e6 + 3.434752e6 + 102.153216e6 + 3.150336e6) / 2,
+    # ncu --cache-control none (L2 kept across launches, as in the timed graph) of four product_tma_kernel launches
+    # in one decomposition of this workload: V-step 45.40 + 37.16 and 44.61 + 13.60 MB, U-step 56.64 + 25.68 and
+    # 51.04 + 16.25 MB (read + write); part of the 99.6 MB residual is served from L2
+    "kind": "products", "file": "product_tma.cu", "sha": "59887d1810844a9e", "workload": "up2560x9728_t5_mu3_tau1_b128",
+    "bytes_per_launch": (45.396992e6 + 37.157376e6 + 44.608256e6 + 13.601536e6 + 56.641280e6 + 25.675008e6 +
+                         51.037696e6 + 16.249856e6) / 4,
 }
 
 
@@ -356,6 +359,15 @@ def run_gpu(args):
     ms_max = max_over_ranks(ev0.elapsed_time(ev1), dev, world)
     value = job_rate(world, comps * args.steps, ms_max)
 
+    if args.steps_only:
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                              "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "gpu_launches": launches,
+                              "config": config_of(args.workload), "steps_only": True}), flush=True)
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
     # ---- end to end through the host entry point: H2D of A (and h), decomposition, D2H of B, D, C, energy
     A_pin = [a.pin_memory() for a in host_A]
     h_pin = [None if h is None else h.pin_memory() for h in host_h]
@@ -630,6 +642,8 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(JOBS))
     ap.add_argument("--roofline-kind", default=ROOFLINE_KIND, choices=["products", "vstep", "ustep", "deflate"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--steps-only", action="store_true",
+                    help="time the steps and print the line without the e2e, roofline and CPU passes (profiler runs)")
     ap.add_argument("--cpu-blocks", type=int, default=16, help="blocks of the workload the CPU baseline times")
     ap.add_argument("--reference-blocks", type=int, default=2, help="blocks per step of the reference arm")
     ap.add_argument("--row", default="decompose", choices=["decompose", "safeguard", "refine", "packed", "sequential"],

@@ -188,6 +188,28 @@ bool use_tc(int w) {
   }();
   return enabled && w >= 16;
 }
+// The Gram inverse and the Eq. 4 solve: on the tensor cores for 65 to 128 components (when the products are),
+// else the register-tiled sweep on one CTA.
+bool tc_inverse(int w, const unsigned* err) { return err != nullptr && use_tc(w) && inverse_tc_enabled(w); }
+cudaError_t inverse_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s, void* op, unsigned* err) {
+  return tc_inverse(w, err) ? launch_inverse_tc_int(Gint, w, Graw, Ginv, s, op, err)
+                            : launch_inverse_int(Gint, w, Graw, Ginv, s, op);
+}
+cudaError_t inverse_f(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s, void* op,
+                      unsigned* err) {
+  return tc_inverse(w, err) ? launch_inverse_tc(Gpart, splits, w, Graw, Ginv, s, op, err)
+                            : launch_inverse(Gpart, splits, w, Graw, Ginv, s, op);
+}
+cudaError_t scales_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s, float* K,
+                       unsigned* err) {
+  return tc_inverse(w, err) ? launch_scales_tc_int(GUint, GVraw, r, w, d, s, K, err)
+                            : launch_scales_int(GUint, GVraw, r, w, d, s, K);
+}
+cudaError_t scales_f(const float* GUpart, int splits, const float* GVraw, const float* r, int w, float* d,
+                     cudaStream_t s, float* K, unsigned* err) {
+  return tc_inverse(w, err) ? launch_scales_tc(GUpart, splits, GVraw, r, w, d, s, K, err)
+                            : launch_scales(GUpart, splits, GVraw, r, w, d, s, K);
+}
 // The TMA-fed tensor-core products where the layout allows them; EXTERND_TMA=0 keeps the register-fed ones.
 bool use_tma() {
   static const bool enabled = [] {
@@ -517,10 +539,10 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
     } else if (w > 1) {
       FORK();
       if (fusedU && !(staged && it == 0)) {
-        KLS(kSolve, 1, side, launch_inverse_int(B.GintU, w, B.GrawU, B.Ginv, side, gop));
+        KLS(kSolve, 1, side, inverse_int(B.GintU, w, B.GrawU, B.Ginv, side, gop, B.err));
       } else {
         KLS(kGram, 1, side, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, side));
-        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side, gop));
+        KLS(kSolve, 1, side, inverse_f(B.Gpart, p.gm, w, B.GrawU, B.Ginv, side, gop, B.err));
       }
     }
     KL(kVstep, 1, product_v(B.R, m, n, B.Ut, U16, (int)p.ldm, w, B.part, sv, B.maxabs, B.err, s, clusterV));
@@ -537,12 +559,12 @@ int fit_block(Workspace& ws, const Plan& p, const Bufs& B, Eq2& q, const float* 
     } else {
       FORK();
       if (fusedV) {
-        KLS(kSolve, 1, side, launch_inverse_int(B.GintV, w, B.GrawV, B.Ginv, side, gop));
+        KLS(kSolve, 1, side, inverse_int(B.GintV, w, B.GrawV, B.Ginv, side, gop, B.err));
       } else if (fusedVw) {
-        KLS(kSolve, 1, side, launch_inverse(B.Gpart, 1, w, B.GrawV, B.Ginv, side, gop));
+        KLS(kSolve, 1, side, inverse_f(B.Gpart, 1, w, B.GrawV, B.Ginv, side, gop, B.err));
       } else {
         KLS(kGram, 1, side, launch_gram(B.Vt, (int)p.ldn, w, n, h, B.Gpart, p.gn, side));
-        KLS(kSolve, 1, side, launch_inverse(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side, gop));
+        KLS(kSolve, 1, side, inverse_f(B.Gpart, p.gn, w, B.GrawV, B.Ginv, side, gop, B.err));
       }
     }
     KL(kUstep, 1, product_u(B.R, m, n, B.Vt, V16, (int)p.ldn, w, h, B.part, su, B.maxabs, B.err, s, clusterU));
@@ -565,10 +587,10 @@ int block_scales_step(const Plan& p, const Bufs& B, int w, float* K, cudaStream_
   if (inverse_cluster_size(w) > 0) {
     KL(kSolve, 1, launch_scales_cluster_int(B.GintU, B.GrawV, B.r, w, B.d, s, K));
   } else if (w <= 128) {
-    KL(kSolve, 1, launch_scales_int(B.GintU, B.GrawV, B.r, w, B.d, s, K));
+    KL(kSolve, 1, scales_int(B.GintU, B.GrawV, B.r, w, B.d, s, K, B.err));
   } else {
     KL(kGram, 1, launch_gram(B.Ut, (int)p.ldm, w, m, nullptr, B.Gpart, p.gm, s));
-    KL(kSolve, 1, launch_scales(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s, K));
+    KL(kSolve, 1, scales_f(B.Gpart, p.gm, B.GrawV, B.r, w, B.d, s, K, B.err));
   }
   return EXTERND_OK;
 }
@@ -1231,7 +1253,7 @@ int step_target(bool vstep, const float* R, long long m, long long n, const int8
   if (decorrelate_needs_operand(w)) TRY(need(*ws, "gop", ginv_operand_bytes() / sizeof(unsigned), &gop));
   if (w > 1) {
     LK(launch_gram(T, (int)ldt, w, (int)Lred, vstep ? nullptr : h, Gpart, gs, g_stream));
-    LK(launch_inverse(Gpart, gs, w, Graw, Ginv, g_stream, gop));
+    LK(inverse_f(Gpart, gs, w, Graw, Ginv, g_stream, gop, err));
   }
   float* theta;
   int* fb;
@@ -1296,10 +1318,10 @@ int externd_block_scales(const float* R, int64_t m, int64_t n, const int8_t* U, 
   TRY(need(*ws, "r", (size_t)w, &r));
   LK(product_u(R, (int)m, (int)n, Vt, V16, (int)ld16(n), (int)w, weights, part, su, mx, err, g_stream));
   LK(launch_gram(Vt, (int)ld16(n), (int)w, (int)n, weights, Gpart, gn, g_stream));
-  LK(launch_inverse(Gpart, gn, (int)w, GrawV, Ginv, g_stream));
+  LK(inverse_f(Gpart, gn, (int)w, GrawV, Ginv, g_stream, nullptr, err));
   LK(launch_gram(Ut, (int)ld16(m), (int)w, (int)m, nullptr, Gpart, gm, g_stream));
   LK(launch_rvec(Ut, (int)ld16(m), (int)w, (int)m, part, su, r, g_stream));
-  LK(launch_scales(Gpart, gm, GrawV, r, (int)w, d, g_stream));
+  LK(scales_f(Gpart, gm, GrawV, r, (int)w, d, g_stream, nullptr, err));
   return check_device_error(*ws, err, g_stream);
 }
 

@@ -312,6 +312,19 @@ cudaError_t launch_scales(const float* GUpart, int splits, const float* GVraw, c
 // Same with G_U from an integer upper-triangle Gram, reset to zero after reading.
 cudaError_t launch_scales_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s,
                               float* K = nullptr);
+// ---- the same on the tensor cores (inverse_tc.cu), for 65 to 128 components: one CTA, S in tensor memory, the
+// rank-16 update of each pivot step as one tf32 MMA (split operands, ~22 significant bits per product); err is
+// the device error word (a bounded wait on the MMA sets it). inverse_tc_enabled: only with EXTERND_TCINV=1 (the
+// register-tiled sweep is faster on GB300).
+bool inverse_tc_enabled(int w);
+cudaError_t launch_inverse_tc(const float* Gpart, int splits, int w, float* Graw, float* Ginv, cudaStream_t s,
+                              void* op, unsigned* err);
+cudaError_t launch_inverse_tc_int(int* Gint, int w, float* Graw, float* Ginv, cudaStream_t s, void* op,
+                                  unsigned* err);
+cudaError_t launch_scales_tc(const float* GUpart, int splits, const float* GVraw, const float* r, int w, float* d,
+                             cudaStream_t s, float* K, unsigned* err);
+cudaError_t launch_scales_tc_int(int* GUint, const float* GVraw, const float* r, int w, float* d, cudaStream_t s,
+                                 float* K, unsigned* err);
 
 
 // ---- the sequential algorithm (§2.3, block width 1) in one launch of one thread-block cluster (sequential.cu),

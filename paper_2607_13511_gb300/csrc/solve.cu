@@ -12,6 +12,7 @@
 #include <cstring>
 
 #include "kernels.h"
+#include "sweep.cuh"
 #include "umma.cuh"
 
 namespace externd {
@@ -342,35 +343,6 @@ __global__ void __launch_bounds__(512) rvec_kernel(const int8_t* __restrict__ Ut
     F2 s;
     for (int q = 0; q < NT / 32; ++q) s = f2_add(s, red[q]);
     r[a] = s.hi + s.lo;
-  }
-}
-
-// One warp inverts an NB x NB SPD block by the symmetric sweep: lane l holds EPL = NB^2/32 entries of row
-// l / LPR (LPR = NB / EPL lanes per row), columns (l % LPR) * EPL + e. Per pivot kk every lane fetches with
-// shuffles the pivot-row entries of its columns (from the lane of row kk with the same column group), the pivot,
-// and its row's pivot-column entry (by symmetry the entry of row r in column kk sits at a register index that is
-// the same for every lane), then updates its entries. On return A holds -P^-1.
-template <int NB>
-__device__ __forceinline__ void warp_sweep(float (&A)[NB * NB / 32], int lane) {
-  constexpr int EPL = NB * NB / 32, LPR = NB / EPL;
-  const int r = lane / LPR, cg = lane % LPR, cb = cg * EPL;
-#pragma unroll
-  for (int kk = 0; kk < NB; ++kk) {
-    float akc[EPL];
-#pragma unroll
-    for (int e = 0; e < EPL; ++e) akc[e] = __shfl_sync(0xffffffffu, A[e], kk * LPR + cg);
-    const float p = __shfl_sync(0xffffffffu, A[kk % EPL], kk * LPR + kk / EPL);
-    const float ark0 = __shfl_sync(0xffffffffu, A[kk % EPL], r * LPR + kk / EPL);
-    const float ip = __fdividef(1.f, p);
-    const float ark = ark0 * ip;   // P[r][kk] / p
-#pragma unroll
-    for (int e = 0; e < EPL; ++e) {
-      const int c = cb + e;
-      float v = fmaf(-ark, akc[e], A[e]);
-      v = (c == kk) ? ark : v;
-      v = (r == kk) ? ((c == kk) ? -ip : akc[e] * ip) : v;
-      A[e] = v;
-    }
   }
 }
 
@@ -728,29 +700,74 @@ struct InvShape {
   static constexpr int TR = WP == 128 ? 8 : WP == 64 ? 4 : 2;
   static constexpr int TC = WP == 128 ? 4 : 2;
   static constexpr int RG = WP / TR, CG = WP / TC, NT = RG * CG;   // row groups, column groups, tile threads
+  // tile warps; warps launched (at WP = 128 with the sub-partition layout of inv_role, else the tile warps then
+  // the pivot warp)
+  static constexpr bool REMAP = WP == 128;
+  static constexpr int NW = NT / 32, NWALL = REMAP ? NW + 4 : NW + 1;
 };
 
 template <int WP>
-constexpr int inv_threads() { return InvShape<WP>::NT + 32; }
+constexpr int inv_threads() { return InvShape<WP>::NWALL * 32; }
+
+// Warp roles of inv_kernel. Warp w runs on SM sub-partition w % 4. Warp 0 is the pivot warp; sub-partition 0
+// holds only p0 tile warps beside it (warps 4, 8, ...), so the pivot warp's serial chain of shuffles and
+// reciprocals is not starved of issue slots by the tile warps' FMA streams; the other tile warps fill
+// sub-partitions 1-3 evenly. Returns the tile-warp index, -2 for the pivot warp, -1 for an idle warp.
+template <int NW>
+__device__ __forceinline__ int inv_role(int warp, int p0) {
+  if (warp == 0) return -2;
+  if ((warp & 3) != 0) {
+    const int t = (warp >> 2) * 3 + (warp & 3) - 1;
+    return t < NW - p0 ? t : -1;
+  }
+  const int j = warp >> 2;   // 1 .. NWALL / 4 - 1
+  return j <= p0 ? NW - p0 + j - 1 : -1;
+}
+
+// The barrier of the pivot and tile warps (idle warps leave at the start).
+template <int N>
+__device__ __forceinline__ void inv_bar() {
+  asm volatile("bar.sync 1, %0;" ::"n"(N) : "memory");
+}
+
+// Tile warps on sub-partition 0 beside the pivot warp (1 .. 4; 4 puts four tile warps on every sub-partition).
+int inv_p0() {
+  static const int p0 = [] {
+    const char* e = std::getenv("EXTERND_INV_P0");
+    const int v = e ? std::atoi(e) : 2;
+    return v < 1 ? 1 : v > 4 ? 4 : v;
+  }();
+  return p0;
+}
+
+template <int WP>
+int inv_p0_for() {   // at most the warps 4, 8, ... that the launch has on sub-partition 0
+  return InvShape<WP>::REMAP ? (inv_p0() < InvShape<WP>::NWALL / 4 - 1 ? inv_p0() : InvShape<WP>::NWALL / 4 - 1) : 0;
+}
 
 template <int WP, int MODE, bool IN_INT>
-__global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float* __restrict__ Gpart, int splits,
-                                                                   int w, const float* __restrict__ GVraw,
-                                                                   const float* __restrict__ r,
-                                                                   float* __restrict__ Graw, float* __restrict__ out,
-                                                                   int* Gint, uint8_t* __restrict__ op) {
+__global__ void __launch_bounds__(InvShape<WP>::NWALL * 32) inv_kernel(const float* __restrict__ Gpart, int splits,
+                                                                     int w, const float* __restrict__ GVraw,
+                                                                     const float* __restrict__ r,
+                                                                     float* __restrict__ Graw,
+                                                                     float* __restrict__ out, int* Gint,
+                                                                     uint8_t* __restrict__ op, int p0) {
   using SH = InvShape<WP>;
-  constexpr int NB = SH::NB, TR = SH::TR, TC = SH::TC, CG = SH::CG, NT = SH::NT, NW = NT / 32;
+  constexpr int NB = SH::NB, TR = SH::TR, TC = SH::TC, CG = SH::CG, NT = SH::NT, NW = SH::NW;
   constexpr int EPL = NB * NB / 32, LPR = NB / EPL;
   static_assert(TR % 2 == 0 && TC % 2 == 0 && (TC == 2 || TC == 4) && NT % 32 == 0, "tile shape");
   static_assert(NB % (TR * (32 / CG)) == 0, "a warp's rows lie in one pivot block");
-  __shared__ __align__(16) float Rk[2][NB][WP];   // published rows of the pivot block (two buffers)
+  __shared__ __align__(16) float Rk[2 * NB * WP];   // published rows of the pivot block (two buffers)
   __shared__ __align__(16) float Ws[NB][WP];      // W = Q Rk of the step
   __shared__ __align__(16) float Qs[2][NB][NB];   // pivot-block inverses (two buffers)
+  __shared__ __align__(16) float Qt[2][NB][NB];   // the same, transposed (Qt[d][c] = Qs[c][d], bit for bit)
   __shared__ __align__(16) float Pn[NB][NB];      // next pivot block before this step's update
-  __shared__ float red[NW + 1];
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const bool tile = tid < NT;
+  __shared__ float red[NW];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tw = SH::REMAP ? inv_role<NW>(warp, p0) : warp < NW ? warp : -2;
+  if (tw == -1) return;   // idle warp (never takes part in the barrier)
+  const bool tile = tw >= 0;
+  const int tid = tile ? tw * 32 + lane : NT + lane;   // tile threads 0 .. NT - 1, then the pivot warp
   const int tr = tile ? tid / CG : 0, tc = tid % CG, i0 = tr * TR, jb = tc * TC;
   const bool vec = (w & 3) == 0;   // rows of every w x w input and output start on 16-byte boundaries
   // a run (i, jb .. jb + TC - 1) of a w x w matrix: one vector access where it is aligned and inside
@@ -883,8 +900,16 @@ __global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float*
     }
   }
   diag = warp_sum(diag);
-  if (lane == 0) red[warp] = diag;
-  __syncthreads();
+  if (lane == 0 && tile) red[tw] = diag;
+  inv_bar<NT + 32>();
+  if (IN_INT) {   // every tile thread has read its entries of the Gram: reset it for the next accumulation
+    const int ww = w * w;
+    if ((ww & 3) == 0) {
+      for (int idx = tid; idx < ww / 4; idx += NT + 32) reinterpret_cast<int4*>(Gint)[idx] = make_int4(0, 0, 0, 0);
+    } else {
+      for (int idx = tid; idx < ww; idx += NT + 32) Gint[idx] = 0;
+    }
+  }
   float trace = 0.f;
 #pragma unroll
   for (int q = 0; q < NW; ++q) trace += red[q];
@@ -897,29 +922,36 @@ __global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float*
         if (i0 + a < w && i0 + a == jb + c) S[a][c] += eps;
   }
 
+  // the published entry (buf, row d of the pivot block, column i)
+  auto rk_at = [&](int buf, int d, int i) -> float* { return &Rk[(buf * NB + d) * WP + i]; };
+  auto rk_val = [&](int buf, int d, int i) -> float { return *rk_at(buf, d, i); };
   auto publish_rows = [&](int kb, int buf) {   // rows [kb, kb + NB) of the register tiles into Rk[buf]
     if (i0 >= kb && i0 < kb + NB) {
 #pragma unroll
       for (int a = 0; a < TR; ++a) {
-        if constexpr (TC == 4)
-          *reinterpret_cast<float4*>(&Rk[buf][i0 + a - kb][jb]) = make_float4(S[a][0], S[a][1], S[a][2], S[a][3]);
-        else
-          *reinterpret_cast<float2*>(&Rk[buf][i0 + a - kb][jb]) = make_float2(S[a][0], S[a][1]);
+        if constexpr (TC == 4) {
+          *reinterpret_cast<float4*>(rk_at(buf, i0 + a - kb, jb)) = make_float4(S[a][0], S[a][1], S[a][2], S[a][3]);
+        } else {
+          *reinterpret_cast<float2*>(rk_at(buf, i0 + a - kb, jb)) = make_float2(S[a][0], S[a][1]);
+        }
       }
     }
   };
   const int pr = lane / LPR, pc = (lane % LPR) * EPL;   // pivot warp: its entries of an NB x NB block
   if (tile) publish_rows(0, 0);
-  __syncthreads();
+  inv_bar<NT + 32>();
   if (!tile) {
     float A[EPL];
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) A[e] = Rk[0][pr][pc + e];
+    for (int e = 0; e < EPL; ++e) A[e] = rk_val(0, pr, pc + e);
     warp_sweep<NB>(A, lane);
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) Qs[0][pr][pc + e] = -A[e];
+    for (int e = 0; e < EPL; ++e) {
+      Qs[0][pr][pc + e] = -A[e];
+      Qt[0][pc + e][pr] = -A[e];
+    }
   }
-  __syncthreads();
+  inv_bar<NT + 32>();
 
   for (int k0 = 0, step = 0; k0 < w; k0 += NB, ++step) {
     const int cur = step & 1, nxt = cur ^ 1, kn = k0 + NB;
@@ -927,15 +959,41 @@ __global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float*
     const bool rowsK = i0 >= k0 && i0 < k0 + NB;          // warp-uniform: a warp's rows lie in one block
     const bool rowsN = has_next && i0 >= kn && i0 < kn + NB;
     const bool colsK = jb + TC > k0 && jb < k0 + NB;      // TC divides NB: a run is wholly in or out of K
-    // A. W = Q Rk; the next pivot block as it stands
+    // A. W = Q Rk; the next pivot block as it stands. At WP = 128 four tile warps, one per sub-partition
+    //    (warps 1 .. 4), form W: lane (cg, qg) of warp 1 + a the rows 4cg .. 4cg + 3 and the columns
+    //    32a + 4qg .. + 3, so a warp reads each Rk row once (128 bytes) and Q as 16-byte rows of Qt; the same
+    //    fma chains in d order as one output per thread.
+    if constexpr (WP == 128) {
+      if (warp >= 1 && warp <= 4) {
+        const int c0 = 4 * (lane >> 3), q0 = 32 * (warp - 1) + 4 * (lane & 7);
+        float4 acc[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int d = 0; d < NB; ++d) {
+          const float4 rv = *reinterpret_cast<const float4*>(rk_at(cur, d, q0));
+          const float4 qv = *reinterpret_cast<const float4*>(&Qt[cur][d][c0]);
+          const float qc[4] = {qv.x, qv.y, qv.z, qv.w};
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            acc[c].x = fmaf(qc[c], rv.x, acc[c].x);
+            acc[c].y = fmaf(qc[c], rv.y, acc[c].y);
+            acc[c].z = fmaf(qc[c], rv.z, acc[c].z);
+            acc[c].w = fmaf(qc[c], rv.w, acc[c].w);
+          }
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) *reinterpret_cast<float4*>(&Ws[c0 + c][q0]) = acc[c];
+      }
+    }
     if (tile) {
-      for (int idx = tid; idx < NB * (WP / 4); idx += NT) {
+      for (int idx = WP == 128 ? NB * (WP / 4) : tid; idx < NB * (WP / 4); idx += NT) {
         const int c = idx / (WP / 4), q = (idx % (WP / 4)) * 4;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
         for (int d = 0; d < NB; ++d) {
           const float qv = Qs[cur][c][d];
-          const float4 rv = *reinterpret_cast<const float4*>(&Rk[cur][d][q]);
+          const float4 rv = *reinterpret_cast<const float4*>(rk_at(cur, d, q));
           acc.x = fmaf(qv, rv.x, acc.x);
           acc.y = fmaf(qv, rv.y, acc.y);
           acc.z = fmaf(qv, rv.z, acc.z);
@@ -950,7 +1008,7 @@ __global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float*
           for (int c = 0; c < TC; ++c) Pn[i0 + a - kn][jb + c - kn] = S[a][c];
       }
     }
-    __syncthreads();
+    inv_bar<NT + 32>();
     // B. the update (tile warps) beside the next pivot block's inverse (pivot warp)
     if (tile) {
       if (rowsK) {
@@ -971,7 +1029,7 @@ __global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float*
           float rk[TR], wv[TC];
 #pragma unroll
           for (int a = 0; a < TR; a += 2) {
-            const float2 t = *reinterpret_cast<const float2*>(&Rk[cur][d][i0 + a]);
+            const float2 t = *reinterpret_cast<const float2*>(rk_at(cur, d, i0 + a));
             rk[a] = t.x;
             rk[a + 1] = t.y;
           }
@@ -1006,7 +1064,7 @@ __global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float*
       for (int e = 0; e < EPL; ++e) A[e] = Pn[pr][pc + e];
 #pragma unroll
       for (int d = 0; d < NB; ++d) {   // the fma chains of the tile owners, in the same order
-        const float rk = Rk[cur][d][kn + pr];
+        const float rk = rk_val(cur, d, kn + pr);
         float wv[EPL];
 #pragma unroll
         for (int e = 0; e < EPL; e += 2) {
@@ -1019,9 +1077,12 @@ __global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float*
       }
       warp_sweep<NB>(A, lane);
 #pragma unroll
-      for (int e = 0; e < EPL; ++e) Qs[nxt][pr][pc + e] = -A[e];
+      for (int e = 0; e < EPL; ++e) {
+        Qs[nxt][pr][pc + e] = -A[e];
+        Qt[nxt][pc + e][pr] = -A[e];
+      }
     }
-    __syncthreads();
+    inv_bar<NT + 32>();
   }
 
   if (MODE == 0) {
@@ -1048,8 +1109,8 @@ __global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float*
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      if (lane == 0) red[warp] = mx;
-      __syncthreads();
+      if (lane == 0 && tile) red[tw] = mx;
+      inv_bar<NT + 32>();
 #pragma unroll
       for (int q = 0; q < NW; ++q) mx = fmaxf(mx, red[q]);
       const int sg = fp16_scale_exp(mx);
@@ -1084,14 +1145,6 @@ __global__ void __launch_bounds__(InvShape<WP>::NT + 32) inv_kernel(const float*
 #pragma unroll
       for (int o = CG / 2; o > 0; o >>= 1) acc2 = f2_add(acc2, f2_shfl_xor(acc2, o));
       if (tc == 0 && i < w) out[i] = acc2.hi + acc2.lo;
-    }
-  }
-  if (IN_INT) {   // every thread read the Gram before the first barrier: reset it for the next accumulation
-    const int ww = w * w;
-    if ((ww & 3) == 0) {
-      for (int idx = tid; idx < ww / 4; idx += NT + 32) reinterpret_cast<int4*>(Gint)[idx] = make_int4(0, 0, 0, 0);
-    } else {
-      for (int idx = tid; idx < ww; idx += NT + 32) Gint[idx] = 0;
     }
   }
 }
@@ -1529,7 +1582,8 @@ cudaError_t launch_sweep_int_w(int* Gint, int w, const float* GVraw, const float
     configured = true;
   }
   if (tiled_inverse())
-    inv_kernel<W_PAD, MODE, true><<<1, inv_threads<W_PAD>(), 0, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint, op);
+    inv_kernel<W_PAD, MODE, true><<<1, inv_threads<W_PAD>(), 0, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint, op,
+                                                                      inv_p0_for<W_PAD>());
   else
     sweep32_kernel<W_PAD, NB, MODE, true><<<1, 544, smem, s>>>(nullptr, 0, w, GVraw, r, Graw, out, Gint, op);
   return cudaGetLastError();
@@ -1550,9 +1604,9 @@ cudaError_t launch_sweep(const float* Gpart, int splits, int w, const float* GVr
   // elements per lane RPW * CPL = W_PAD^2 / (32 * NWARP): 4 / 8 / 32 / 64
   // pivot-block sizes measured fastest on GB300: 8 up to w = 64, 16 at w = 128
   const bool tiled = tiled_inverse();
-  if (w <= 32 && tiled) inv_kernel<32, MODE, false><<<1, inv_threads<32>(), 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
-  else if (w <= 64 && tiled) inv_kernel<64, MODE, false><<<1, inv_threads<64>(), 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
-  else if (w <= 128 && tiled) inv_kernel<128, MODE, false><<<1, inv_threads<128>(), 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, op);
+  if (w <= 32 && tiled) inv_kernel<32, MODE, false><<<1, inv_threads<32>(), 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr, inv_p0_for<32>());
+  else if (w <= 64 && tiled) inv_kernel<64, MODE, false><<<1, inv_threads<64>(), 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr, inv_p0_for<64>());
+  else if (w <= 128 && tiled) inv_kernel<128, MODE, false><<<1, inv_threads<128>(), 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, op, inv_p0_for<128>());
   else if (w <= 32) sweep32_kernel<32, 8, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
   else if (w <= 64) sweep32_kernel<64, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, nullptr);
   else if (w <= 128) sweep32_kernel<128, 16, MODE, false><<<1, 544, 0, s>>>(Gpart, splits, w, GVraw, r, Graw, out, nullptr, op);
