@@ -428,6 +428,22 @@ def run_gpu(args):
             and NCU_TRAFFIC.get("workload") == args.workload:
         traffic = NCU_TRAFFIC["bytes_per_launch"]
 
+    # ---- what this GPU's HBM delivers to a plain read stream (context for the products' fraction, not the peak):
+    # torch's float32 sum over 2 GB, best of 5, CUDA events
+    rbuf = torch.ones(512 * 1024 * 1024, dtype=torch.float32, device=dev)
+    for _ in range(2):
+        rbuf.sum()
+    best = float("inf")
+    for _ in range(5):
+        r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        r0.record(stream)
+        rbuf.sum()
+        r1.record(stream)
+        r1.synchronize()
+        best = min(best, r0.elapsed_time(r1))
+    read_gbs = rbuf.numel() * 4 / (best / 1e3) / 1e9
+    del rbuf
+
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
@@ -461,6 +477,10 @@ def run_gpu(args):
                         "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
                         "bytes_per_launch": bytes_per_launch, "launches": prof_n,
                         "us_per_launch": per_launch_s * 1e6}
+    if not seq:
+        line["read_ceiling"] = {"gbs": read_gbs, "frac_of_peak": read_gbs / peak,
+                                "roofline_frac_of_it": achieved / read_gbs,
+                                "how": "torch float32 sum over 2 GB on this GPU, best of 5 (a read-only stream)"}
     if not seq:   # the HBM model of the whole step: 2 iters passes over R and the deflation per block
         line["step_roofline"] = {"algorithmic_bytes": step_bytes, "lower_bound_ms": step_bytes / (peak * 1e6),
                                  "frac": step_bytes / (peak * 1e6) / ms_step}

@@ -2,19 +2,21 @@
 // components.
 //
 // The symmetric sweep of inv_kernel (Gauss-Jordan on an SPD matrix without pivoting, pivot blocks K of 16),
-// with the 128 x 128 float32 matrix S in tensor memory (row i in lane i) instead of registers. Per step, with
-// the pivot rows Rk = S[K,:] and Q = S[K,K]^-1:
-//   1. W = Q Rk (16 x 128) on the CUDA cores, thread j computing column j;
-//   2. S[i][j] -= sum_d Rk[d][i] W[d][j] for all i, j as ONE 128 x 128 x 16 MMA of kind::tf32: A = -Rk^T and
-//      B = W, both split into tf32 hi + lo parts (hi.hi + hi.lo + lo.hi, about 22 significant bits per
-//      product), accumulated in float32 in tensor memory;
-//   3. the pivot rows and columns take their exact sweep values: column K_d of row i is W[d][i] (= S[i,K] Q),
-//      row K_d is W[d][.] and -Q[d][.] on the pivot block. The warp of K's lane quadrant reads its 32 lanes
-//      back and rewrites them; every other warp rewrites only the 16 columns of K. The rows of the next pivot
-//      block go to shared memory on the way;
-//   4. the pivot warp inverts the next pivot block (warp_sweep).
-// After the last step S = -(G + eps I)^-1. The O(w^3) update runs on the tensor cores; what stays serial is the
-// 16-pivot sweep per step. Every wait on the MMA is bounded (2 s, then the error word and an early exit).
+// with the 128 x 128 float32 matrix S in tensor memory (row i in lane i) instead of registers. Per step s, with
+// the pivot rows Rk = S[K,:] and Q = S[K,K]^-1 in shared memory:
+//   1. W = Q Rk (16 x 128) on the CUDA cores, thread j computing column j; the MMA operands A = -Rk^T and B = W,
+//      split into tf32 hi + lo parts;
+//   2. S[i][j] -= sum_d Rk[d][i] W[d][j] for all i, j as ONE 128 x 128 x 16 MMA of kind::tf32 (hi.hi + hi.lo +
+//      lo.hi, about 22 significant bits per product, float32 accumulation in tensor memory). Meanwhile the
+//      rows of the next pivot block are updated in float32 on the CUDA cores (the same fma chains as inv_kernel)
+//      and the pivot warp inverts the next pivot block (warp_sweep), so neither waits for the MMA;
+//   3. once the MMA is done the pivot rows and columns take their exact sweep values (column K_d of row i is
+//      W[d][i] = (S[i,K] Q)_d, row K_d is W[d][.] and -Q[d][.] on the pivot block: the warp of K's lane quadrant
+//      reads its 32 lanes back and rewrites them), and the rows two blocks ahead are read from tensor memory.
+// After the last step S = -(G + eps I)^-1. The tensor-memory copies of a pivot block's rows before its own step
+// are never used (the step rewrites them), so the pivot blocks and their inverses are float32-exact as in
+// inv_kernel; the rest of S carries the MMA's ~22-bit products. Every wait on the MMA is bounded (2 s, then the
+// error word and an early exit).
 #include <cuda_fp16.h>
 
 #include <cstdlib>
@@ -32,19 +34,24 @@ constexpr int kTiN = 128;        // matrix side in tensor memory (padded with th
 constexpr int kTiNB = 16;        // pivot block
 constexpr int kTiRows = 128;     // row threads (warps 0-3, thread i = lane i)
 constexpr int kTiThreads = 192;  // + warp 4 (tensor memory, MMA issue) + warp 5 (pivot warp)
-// shared memory: A hi, A lo, B hi, B lo (K-major, 128-byte swizzle, 128 rows of which 64 B are used), then
-// Ws (16 x 128), Rk (16 x 128), Q (16 x 16), and with MODE 1 the staged G_V. The Gram is staged first over the
-// operands (and the start of Ws), rows of kTiP floats: entry (a, b) of both triangles sits in bank (a + b) % 32.
-constexpr int kTiP = 129;
+// shared memory: the MMA operands A hi, A lo, B hi, B lo (K-major, 128-byte swizzle, 128 rows of which 64 B are
+// used), over which the Gram is staged first (rows of kTiP floats, 16-byte aligned: a row read as float4 runs and
+// a column read as scalars both spread over all banks); then W (16 x 128), the current and next pivot rows, the
+// rows two blocks ahead, Q and its transpose (two buffers each), and with MODE 1 the staged G_V.
+constexpr int kTiP = 132;
 constexpr uint32_t kTiOp = 16384;
-constexpr uint32_t kTiWs = 4 * kTiOp, kTiRk = kTiWs + kTiNB * kTiN * 4, kTiQ = kTiRk + kTiNB * kTiN * 4;
-constexpr uint32_t kTiGV = kTiQ + kTiNB * kTiNB * 4;
-constexpr size_t kTiStage = (size_t)kTiN * kTiP * 4;
-static_assert(kTiStage <= kTiRk, "the staged Gram ends before Rk");
+constexpr uint32_t kTiStage = (uint32_t)kTiN * kTiP * 4;   // 67,584 B >= the operands' 65,536 B
+constexpr uint32_t kTiRowBlk = kTiNB * kTiN * 4;           // 16 rows of 128 floats
+constexpr uint32_t kTiWs = kTiStage, kTiRkA = kTiWs + kTiRowBlk, kTiRkB = kTiRkA + kTiRowBlk,
+                   kTiRn = kTiRkB + kTiRowBlk, kTiQ = kTiRn + kTiRowBlk, kTiQt = kTiQ + 2 * kTiNB * kTiNB * 4,
+                   kTiGV = kTiQt + 2 * kTiNB * kTiNB * 4;
 constexpr size_t tc_inv_smem(int mode) { return 1024 + kTiGV + (mode == 1 ? kTiStage : 0); }
 
 __device__ __forceinline__ void cp_async4(uint32_t dst, const void* src) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
 }
 
 // Instruction descriptor of kind::tf32: tf32 A and B, fp32 D, both K-major, M x N.
@@ -117,9 +124,14 @@ __global__ void __launch_bounds__(kTiThreads, 1) inv_tc_kernel(const float* __re
   const uint32_t sbase = (raw + 1023u) & ~1023u;
   uint8_t* const gbase = smem_raw + (sbase - raw);
   const uint32_t opA = sbase, opB = sbase + 2 * kTiOp;
-  float* const Rk = reinterpret_cast<float*>(gbase + kTiRk);   // [16][128]
-  float* const Ws = reinterpret_cast<float*>(gbase + kTiWs);   // [16][128]
-  float* const Qs = reinterpret_cast<float*>(gbase + kTiQ);    // [16][16]
+  uint32_t* const Gs = reinterpret_cast<uint32_t*>(gbase);                 // staged Gram, rows of kTiP
+  const float* const GVs = reinterpret_cast<const float*>(gbase + kTiGV);  // staged G_V (MODE 1)
+  float* const Ws = reinterpret_cast<float*>(gbase + kTiWs);               // [16][128]
+  float* RkA = reinterpret_cast<float*>(gbase + kTiRkA);                   // pivot rows of this step
+  float* RkB = reinterpret_cast<float*>(gbase + kTiRkB);                   // pivot rows of the next step
+  float* const Rn = reinterpret_cast<float*>(gbase + kTiRn);               // rows two blocks ahead
+  float* const Qb = reinterpret_cast<float*>(gbase + kTiQ);                // [2][16][16]
+  float* const Qtb = reinterpret_cast<float*>(gbase + kTiQt);              // [2][16][16], transposed
   __shared__ uint64_t mma_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ float red[4];
@@ -135,44 +147,60 @@ __global__ void __launch_bounds__(kTiThreads, 1) inv_tc_kernel(const float* __re
       fence_barrier_init();
     }
   }
-  // Stage the Gram (the integer upper triangle, or the float partials) and, for Eq. 4, G_V: asynchronous 4-byte
-  // copies, all in flight at once, rows of kTiP floats.
-  uint32_t* const Graw_s = reinterpret_cast<uint32_t*>(gbase);
-  const float* const GVs = reinterpret_cast<const float*>(gbase + kTiGV);
+  // ---- stage the Gram (the integer upper triangle, or the float partials) and, for Eq. 4, G_V
+  const bool vec = (w & 3) == 0;   // rows start on 16-byte boundaries in global memory
+  auto stage = [&](uint32_t* dst, const uint32_t* src) {
+    if (vec) {
+      const int q4 = w >> 2;
+      for (int a = warp; a < w; a += kTiThreads / 32)
+        for (int c = lane; c < q4; c += 32) cp_async16(smem_addr(dst + a * kTiP + 4 * c), src + (long long)a * w + 4 * c);
+    } else {
+      for (int a = warp; a < w; a += kTiThreads / 32)
+        for (int b = lane; b < w; b += 32) cp_async4(smem_addr(dst + a * kTiP + b), src + (long long)a * w + b);
+    }
+  };
   if (IN_INT || splits == 1) {
-    const uint32_t* src = IN_INT ? reinterpret_cast<const uint32_t*>(Gint) : reinterpret_cast<const uint32_t*>(Gpart);
-    for (int a = warp; a < w; a += kTiThreads / 32)
-      for (int b = lane; b < w; b += 32) cp_async4(smem_addr(Graw_s + a * kTiP + b), src + (long long)a * w + b);
+    stage(Gs, IN_INT ? reinterpret_cast<const uint32_t*>(Gint) : reinterpret_cast<const uint32_t*>(Gpart));
   } else {
     for (int a = warp; a < w; a += kTiThreads / 32)
       for (int b = lane; b < w; b += 32) {
         float g = 0.f;
         for (int sp = 0; sp < splits; ++sp) g += Gpart[(long long)sp * w * w + (long long)a * w + b];
-        Graw_s[a * kTiP + b] = __float_as_uint(g);
+        Gs[a * kTiP + b] = __float_as_uint(g);
       }
   }
-  if (MODE == 1) {
-    for (int a = warp; a < w; a += kTiThreads / 32)
-      for (int b = lane; b < w; b += 32) cp_async4(smem_addr(GVs + a * kTiP + b), GVraw + (long long)a * w + b);
-  }
+  if (MODE == 1) stage(reinterpret_cast<uint32_t*>(gbase + kTiGV), reinterpret_cast<const uint32_t*>(GVraw));
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
   __syncthreads();
-  // the Gram's (or K's) entry (a, b), a, b < w
-  auto entry = [&](int a, int b) -> float {
-    float g = IN_INT ? (float)(int)Graw_s[min(a, b) * kTiP + max(a, b)] : __uint_as_float(Graw_s[a * kTiP + b]);
-    if (MODE == 1) g *= GVs[a * kTiP + b];   // K = G_U .* G_V
-    return g;
-  };
-  if (IN_INT) {   // every entry is staged: reset the Gram for the next accumulation
+  if (IN_INT) {
+    // the lower triangle from the upper one, as float; then the Gram can be reset for the next accumulation
+    for (int a = warp; a < w; a += kTiThreads / 32)
+      for (int b = lane; b < w; b += 32) {
+        const uint32_t g = Gs[min(a, b) * kTiP + max(a, b)];
+        if (b < a) Gs[a * kTiP + b] = __float_as_uint((float)(int)g);
+      }
+    __syncthreads();
+    for (int a = warp; a < w; a += kTiThreads / 32)
+      for (int b = lane; b <= a; b += 32) Gs[b * kTiP + a] = __float_as_uint((float)(int)Gs[b * kTiP + a]);
     for (int idx = tid; idx < w * w; idx += kTiThreads) Gint[idx] = 0;
+    __syncthreads();
   }
+  if (MODE == 1) {   // K = G_U .* G_V
+    for (int a = warp; a < w; a += kTiThreads / 32)
+      for (int b = lane; b < w; b += 32) {
+        float* g = reinterpret_cast<float*>(Gs + a * kTiP + b);
+        *g *= GVs[a * kTiP + b];
+      }
+    __syncthreads();
+  }
+  const float* const Gf = reinterpret_cast<const float*>(Gs);
   if (Graw != nullptr) {   // G (or K) before the ridge
     for (int a = warp; a < w; a += kTiThreads / 32)
-      for (int b = lane; b < w; b += 32) Graw[(long long)a * w + b] = entry(a, b);
+      for (int b = lane; b < w; b += 32) Graw[(long long)a * w + b] = Gf[a * kTiP + b];
   }
   if (row_thread) {
-    const float s = warp_sum(i < w ? entry(i, i) : 0.f);
-    if (lane == 0) red[warp] = s;
+    const float sd = warp_sum(i < w ? Gf[i * kTiP + i] : 0.f);
+    if (lane == 0) red[warp] = sd;
   }
   tc_fence_before();
   __syncthreads();
@@ -181,23 +209,30 @@ __global__ void __launch_bounds__(kTiThreads, 1) inv_tc_kernel(const float* __re
   const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);   // this warp's lane quadrant
   const float eps = ((MODE == 0) || (w > 1)) ? (float)kEpsRel * (red[0] + red[1] + red[2] + red[3]) / (float)w : 0.f;
 
-  // S = G + eps I (identity on the padding) into tensor memory, 16 columns at a time; rows 0..15 also to Rk
+  // ---- S = G + eps I (identity on the padding) into tensor memory; rows 0..15 to RkA, rows 16..31 to Rn
   if (row_thread) {
 #pragma unroll 1
     for (int c = 0; c < kTiN / 16; ++c) {
       uint32_t v[16];
 #pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        const int j = 16 * c + e;
-        float x;
-        if (i < w && j < w) {
-          x = entry(i, j);
-          if (i == j) x += eps;
-        } else {
-          x = i == j ? 1.f : 0.f;
+      for (int e4 = 0; e4 < 4; ++e4) {
+        const int j = 16 * c + 4 * e4;
+        float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i < w) g = *reinterpret_cast<const float4*>(Gf + i * kTiP + j);   // columns >= w are masked below
+        const float gv[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          float x = (i < w && j + e < w) ? gv[e] : 0.f;
+          if (i == j + e) x = i < w ? x + eps : 1.f;
+          v[4 * e4 + e] = __float_as_uint(x);
         }
-        if (i < kTiNB) Rk[i * kTiN + j] = x;
-        v[e] = __float_as_uint(x);
+      }
+      if (i < kTiNB) {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) RkA[i * kTiN + 16 * c + e] = __uint_as_float(v[e]);
+      } else if (i < 2 * kTiNB) {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) Rn[(i - kTiNB) * kTiN + 16 * c + e] = __uint_as_float(v[e]);
       }
       tmem_st16(trow + (uint32_t)(16 * c), v);
     }
@@ -207,43 +242,50 @@ __global__ void __launch_bounds__(kTiThreads, 1) inv_tc_kernel(const float* __re
   __syncthreads();
   tc_fence_after();
   const int pr = lane / 2, pc = (lane % 2) * 8;   // pivot warp: its 8 entries of the 16 x 16 block
-  if (warp == 5) {
+  auto sweep_block = [&](const float* rows, int col0, int buf) {   // Q of rows[.][col0 .. col0 + 15]
     float A[8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) A[e] = Rk[pr * kTiN + pc + e];
+    for (int e = 0; e < 8; ++e) A[e] = rows[pr * kTiN + col0 + pc + e];
     warp_sweep<kTiNB>(A, lane);
 #pragma unroll
-    for (int e = 0; e < 8; ++e) Qs[pr * kTiNB + pc + e] = -A[e];
-  }
+    for (int e = 0; e < 8; ++e) {
+      Qb[buf * 256 + pr * kTiNB + pc + e] = -A[e];
+      Qtb[buf * 256 + (pc + e) * kTiNB + pr] = -A[e];
+    }
+  };
+  if (warp == 5) sweep_block(RkA, 0, 0);
   __syncthreads();
 
   constexpr uint32_t idesc = tf32_idesc(kTiN, kTiN);
   bool ok = true;
   int step = 0;
   for (int k0 = 0; k0 < w; k0 += kTiNB, ++step) {
-    const int kn = k0 + kTiNB, qK = k0 >> 5;
-    const bool has_next = kn < w;
+    const int kn = k0 + kTiNB, kn2 = kn + kTiNB, qK = k0 >> 5, cur = step & 1;
+    const bool has_next = kn < w, has_next2 = kn2 < w;
+    const float* const Q = Qb + cur * 256;
+    const float* const Qt = Qtb + cur * 256;
     float wj[kTiNB];   // row threads: W[.][i]
-    // 1. W = Q Rk (column i per row thread); the operands A = -Rk^T and B = W
+    // 1. W = Q Rk, column i per row thread (fma chains over e in order, as inv_kernel); the MMA operands
     if (row_thread) {
       float rk[kTiNB];
 #pragma unroll
-      for (int e = 0; e < kTiNB; ++e) rk[e] = Rk[e * kTiN + i];
+      for (int e = 0; e < kTiNB; ++e) rk[e] = RkA[e * kTiN + i];
 #pragma unroll
-      for (int d = 0; d < kTiNB; ++d) {
-        const float4* qrow = reinterpret_cast<const float4*>(Qs + d * kTiNB);
-        float acc = 0.f;
+      for (int d = 0; d < kTiNB; ++d) wj[d] = 0.f;
 #pragma unroll
-        for (int e4 = 0; e4 < kTiNB / 4; ++e4) {
-          const float4 q = qrow[e4];
-          acc = fmaf(q.x, rk[4 * e4], acc);
-          acc = fmaf(q.y, rk[4 * e4 + 1], acc);
-          acc = fmaf(q.z, rk[4 * e4 + 2], acc);
-          acc = fmaf(q.w, rk[4 * e4 + 3], acc);
+      for (int e = 0; e < kTiNB; ++e) {
+        const float4* qc = reinterpret_cast<const float4*>(Qt + e * kTiNB);   // Q[.][e]
+#pragma unroll
+        for (int d4 = 0; d4 < kTiNB / 4; ++d4) {
+          const float4 q = qc[d4];
+          wj[4 * d4] = fmaf(q.x, rk[e], wj[4 * d4]);
+          wj[4 * d4 + 1] = fmaf(q.y, rk[e], wj[4 * d4 + 1]);
+          wj[4 * d4 + 2] = fmaf(q.z, rk[e], wj[4 * d4 + 2]);
+          wj[4 * d4 + 3] = fmaf(q.w, rk[e], wj[4 * d4 + 3]);
         }
-        wj[d] = acc;
-        Ws[d * kTiN + i] = acc;
       }
+#pragma unroll
+      for (int d = 0; d < kTiNB; ++d) Ws[d * kTiN + i] = wj[d];
       float na[kTiNB];
 #pragma unroll
       for (int e = 0; e < kTiNB; ++e) na[e] = -rk[e];
@@ -253,7 +295,7 @@ __global__ void __launch_bounds__(kTiThreads, 1) inv_tc_kernel(const float* __re
     }
     tc_fence_before();
     __syncthreads();
-    // 2. the rank-16 update
+    // 2. the rank-16 update on the tensor cores; meanwhile the next pivot rows in float32
     if (warp == 4 && lane == 0) {
       tc_fence_after();
 #pragma unroll
@@ -266,40 +308,60 @@ __global__ void __launch_bounds__(kTiThreads, 1) inv_tc_kernel(const float* __re
       }
       mma_commit(smem_addr(&mma_bar));
     }
-    // 3. the exact pivot rows and columns; the next pivot rows into Rk
+    const bool inK = i >= k0 && i < kn;
+    if (row_thread && has_next) {
+      // rows kn + e after this step: column j in K is W[j - k0][kn + e] (written by thread kn + e), any other
+      // column S[kn + e][j] - sum_d Rk[d][kn + e] W[d][j]
+      if (!inK) {
+#pragma unroll 4
+        for (int e = 0; e < kTiNB; ++e) {
+          float acc = Rn[e * kTiN + i];
+#pragma unroll
+          for (int d = 0; d < kTiNB; ++d) acc = fmaf(-RkA[d * kTiN + kn + e], wj[d], acc);
+          RkB[e * kTiN + i] = acc;
+        }
+      }
+      if (i >= kn && i < kn2) {
+#pragma unroll
+        for (int d = 0; d < kTiNB; ++d) RkB[(i - kn) * kTiN + k0 + d] = wj[d];
+      }
+    }
+    __syncthreads();
+    // 3. pivot warp: the next pivot block's inverse. Row threads: the exact pivot rows and columns once the MMA
+    //    is done, and the rows two blocks ahead
+    if (warp == 5 && has_next) sweep_block(RkB, kn, cur ^ 1);
     if (row_thread) {
       ok = mbar_wait(smem_addr(&mma_bar), (uint32_t)(step & 1), err);
       tc_fence_after();
       if (ok) {
-        const bool inK = i >= k0 && i < kn;
         const int dK = i - k0;
         uint32_t colK[16];   // columns K: W[.][i], or -Q on the pivot block
 #pragma unroll
-        for (int e = 0; e < 16; ++e) colK[e] = __float_as_uint(inK ? -Qs[dK * kTiNB + e] : wj[e]);
+        for (int e = 0; e < 16; ++e) colK[e] = __float_as_uint(inK ? -Q[dK * kTiNB + e] : wj[e]);
         tmem_st16(trow + (uint32_t)k0, colK);
-        const bool nextHere = has_next && (kn >> 5) == warp;   // this quadrant holds the next pivot rows
-        const bool inN = has_next && i >= kn && i < kn + kTiNB;
-        if (nextHere && inN) {
+        const bool aheadHere = has_next2 && (kn2 >> 5) == warp;
+        if (warp == qK || aheadHere) {
+          uint32_t v[kTiN / 16][16];
 #pragma unroll
-          for (int e = 0; e < 16; ++e) Rk[(i - kn) * kTiN + k0 + e] = __uint_as_float(colK[e]);
-        }
-        if (warp == qK || nextHere) {
-#pragma unroll 1
-          for (int c = 0; c < kTiN / 16; ++c) {
-            if (16 * c == k0) continue;
-            uint32_t v[16];
-            tmem_ld16(trow + (uint32_t)(16 * c), v);
-            tmem_wait_ld();
-            if (warp == qK) {
+          for (int c = 0; c < kTiN / 16; ++c)
+            if (16 * c != k0) tmem_ld16(trow + (uint32_t)(16 * c), v[c]);
+          tmem_wait_ld();
+          if (warp == qK) {
+#pragma unroll
+            for (int c = 0; c < kTiN / 16; ++c) {
+              if (16 * c == k0) continue;
               if (inK) {
 #pragma unroll
-                for (int e = 0; e < 16; ++e) v[e] = __float_as_uint(Ws[dK * kTiN + 16 * c + e]);
+                for (int e = 0; e < 16; ++e) v[c][e] = __float_as_uint(Ws[dK * kTiN + 16 * c + e]);
               }
-              tmem_st16(trow + (uint32_t)(16 * c), v);
+              tmem_st16(trow + (uint32_t)(16 * c), v[c]);
             }
-            if (inN) {
+          } else if (i >= kn2 && i < kn2 + kTiNB) {
 #pragma unroll
-              for (int e = 0; e < 16; ++e) Rk[(i - kn) * kTiN + 16 * c + e] = __uint_as_float(v[e]);
+            for (int c = 0; c < kTiN / 16; ++c) {
+#pragma unroll
+              for (int e = 0; e < 16; ++e)
+                Rn[(i - kn2) * kTiN + 16 * c + e] = 16 * c == k0 ? wj[e] : __uint_as_float(v[c][e]);
             }
           }
         }
@@ -310,57 +372,44 @@ __global__ void __launch_bounds__(kTiThreads, 1) inv_tc_kernel(const float* __re
     ok = __syncthreads_and(ok) != 0;
     tc_fence_after();
     if (!ok) break;
-    // 4. the next pivot block's inverse
-    if (warp == 5 && has_next) {
-      float A[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) A[e] = Rk[pr * kTiN + kn + pc + e];
-      warp_sweep<kTiNB>(A, lane);
-#pragma unroll
-      for (int e = 0; e < 8; ++e) Qs[pr * kTiNB + pc + e] = -A[e];
-    }
-    __syncthreads();
+    float* const t = RkA;
+    RkA = RkB;
+    RkB = t;
   }
 
-  // outputs from -S, row i per row thread
+  // ---- outputs from -S, row i per row thread (all 128 columns read at once)
   if (ok && row_thread) {
+    uint32_t v[kTiN / 16][16];
+#pragma unroll
+    for (int c = 0; c < kTiN / 16; ++c) tmem_ld16(trow + (uint32_t)(16 * c), v[c]);
+    tmem_wait_ld();
     if (MODE == 0 && op != nullptr) {
       float mx = 0.f;
-#pragma unroll 1
-      for (int c = 0; c < kTiN / 16; ++c) {
-        uint32_t v[16];
-        tmem_ld16(trow + (uint32_t)(16 * c), v);
-        tmem_wait_ld();
+#pragma unroll
+      for (int c = 0; c < kTiN / 16; ++c)
 #pragma unroll
         for (int e = 0; e < 16; ++e)
-          if (i < w && 16 * c + e < w) mx = fmaxf(mx, fabsf(__uint_as_float(v[e])));
-      }
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+          if (i < w && 16 * c + e < w) mx = fmaxf(mx, fabsf(__uint_as_float(v[c][e])));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
       if (lane == 0) red[warp] = mx;
       bar_rows();
       mx = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
       const int sg = fp16_scale_exp(mx);
       const float sc = ldexpf(1.f, sg);
-      // row i: the 16-byte chunk j of K atom ka holds Ginv[i][64 ka + 8 j .. + 7]
-#pragma unroll 1
-      for (int c = 0; c < kTiN / 16; ++c) {
-        uint32_t v[16];
-        tmem_ld16(trow + (uint32_t)(16 * c), v);
-        tmem_wait_ld();
+      // row i: the 16-byte chunk of columns k .. k + 7 (k = 0, 8, ..., 120) at k_major_offset(128, i, k)
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {   // the two 8-column chunks of these 16 columns
+      for (int c = 0; c < kTiN / 16; ++c) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
           const int k = 16 * c + 8 * h;
           uint32_t hi[4], lo[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
             __half h0, l0, h1, l1;
             const int j0 = k + 2 * e, j1 = j0 + 1;
-            split_f16((i < w && j0 < w) ? -__uint_as_float(v[8 * h + 2 * e]) * sc : 0.f, h0, l0);
-            split_f16((i < w && j1 < w) ? -__uint_as_float(v[8 * h + 2 * e + 1]) * sc : 0.f, h1, l1);
+            split_f16((i < w && j0 < w) ? -__uint_as_float(v[c][8 * h + 2 * e]) * sc : 0.f, h0, l0);
+            split_f16((i < w && j1 < w) ? -__uint_as_float(v[c][8 * h + 2 * e + 1]) * sc : 0.f, h1, l1);
             hi[e] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
             lo[e] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
           }
@@ -371,30 +420,22 @@ __global__ void __launch_bounds__(kTiThreads, 1) inv_tc_kernel(const float* __re
       }
       if (i == 0) *reinterpret_cast<int*>(op + 4 * 16384u) = sg;
     } else if (MODE == 0) {
-#pragma unroll 1
-      for (int c = 0; c < kTiN / 16; ++c) {
-        uint32_t v[16];
-        tmem_ld16(trow + (uint32_t)(16 * c), v);
-        tmem_wait_ld();
+#pragma unroll
+      for (int c = 0; c < kTiN / 16; ++c)
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int j = 16 * c + e;
-          if (i < w && j < w) out[(long long)i * w + j] = -__uint_as_float(v[e]);
+          if (i < w && j < w) out[(long long)i * w + j] = -__uint_as_float(v[c][e]);
         }
-      }
     } else {
       F2 acc;
-#pragma unroll 1
-      for (int c = 0; c < kTiN / 16; ++c) {
-        uint32_t v[16];
-        tmem_ld16(trow + (uint32_t)(16 * c), v);
-        tmem_wait_ld();
+#pragma unroll
+      for (int c = 0; c < kTiN / 16; ++c)
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int j = 16 * c + e;
-          if (j < w) acc = f2_add(acc, -__uint_as_float(v[e]) * r[j]);
+          if (j < w) acc = f2_add(acc, -__uint_as_float(v[c][e]) * r[j]);
         }
-      }
       if (i < w) out[i] = acc.hi + acc.lo;
     }
   }
@@ -422,10 +463,11 @@ cudaError_t launch_tc(const float* Gpart, int splits, int w, const float* GVraw,
 
 }  // namespace
 
-// Off unless EXTERND_TCINV=1: on GB300 the register-tiled sweep is faster (about 31 us against 40-52 us at
-// w = 128). Per step the tensor-core version spends ~600 cycles on the MMA but ~3,800 on W = Q Rk, the operand
-// splits and the pivot sweep, and ~2,400 on rewriting the pivot rows (tensor-memory loads of the K quadrant);
-// its Gram staging and operand-image epilogue add ~12 us.
+// Off unless EXTERND_TCINV=1: on GB300 the register-tiled sweep is faster (28-31 us against ~42 us alone and
+// ~55 us in the graph at w = 128). A clock64 timeline of one launch: the MMA is hidden (its wait takes ~200
+// cycles), but each step still spends ~1,400 cycles on W and the operand splits, ~2,500 on the next pivot rows
+// and ~2,500 on rewriting the pivot rows beside the next sweep, all on four latency-bound warps, and the
+// prologue (Gram staging and mirror, tensor-memory fill, first sweep) ~23,000 cycles.
 bool inverse_tc_enabled(int w) {
   static const bool enabled = [] {
     const char* e = std::getenv("EXTERND_TCINV");
