@@ -131,3 +131,43 @@ def test_host_side_argument_errors(lib):
     se.restype = ctypes.c_char_p
     for code in (0, -1, -2, -3, -4, -5, 7):
         assert se(code)
+
+
+C_CALLER = r"""
+#include <stdio.h>
+#include <stdint.h>
+#include "externd.h"
+
+int main(void) {
+    int64_t k = 0;
+    double energy = 0.0;
+    if (externd_rank(2560, 9728, 3.0, &k) != EXTERND_OK || k != 7680) return 1;
+    /* the decomposition with the twelve parameters of the boundary: an empty matrix is rejected on the host */
+    if (externd_decompose((const float*)0, 0, 9728, 3.0, 1.0, 128, 4, (const float*)0, (int8_t*)0, (float*)0,
+                          (int8_t*)0, &energy) != EXTERND_EINVAL) return 2;
+    if (externd_energy((const float*)0, 0, 9728, (const int8_t*)0, (const float*)0, (const int8_t*)0, 7680,
+                       (const float*)0, &energy) != EXTERND_EINVAL) return 3;
+    if (externd_strerror(EXTERND_EINVAL) == 0) return 4;
+    printf("ok %lld\n", (long long)k);
+    return 0;
+}
+"""
+
+
+def test_c_caller_compiles_links_and_runs(lib, tmp_path):
+    """A plain C99 program written to the boundary compiles against the header, links and runs its host-side
+    checks (no GPU needed)."""
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    from paper_2607_13511_gb300 import build
+    libdir = os.path.dirname(build.LIB)
+    src = tmp_path / "caller.c"
+    src.write_text(C_CALLER)
+    exe = tmp_path / "caller"
+    res = subprocess.run([cc, "-std=c99", "-Wall", "-Werror", "-I", os.path.join(ROOT, "include"), str(src), "-o",
+                          str(exe), "-L", libdir, "-lexternd", f"-Wl,-rpath,{libdir}"], capture_output=True, text=True)
+    assert res.returncode == 0, res.stderr
+    run = subprocess.run([str(exe)], capture_output=True, text=True, timeout=120)
+    assert run.returncode == 0 and run.stdout.strip() == "ok 7680", (run.returncode, run.stdout, run.stderr)
