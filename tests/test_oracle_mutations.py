@@ -68,6 +68,29 @@ MUTATIONS = {
     "block width cap at min / 4": [("return max(1, min(int(block), min(m, n) // 8))",
                                     "return max(1, min(int(block), min(m, n) // 4))")],
     "inner rank truncated": [("return int(math.floor(mu * min(m, n) + 0.5))", "return int(math.floor(mu * min(m, n)))")],
+    "eq3 v-step without the gram inverse (naive batching)": [("    return vstep_solve(vstep_product(R, U), U)",
+                                                              "    return vstep_product(R, U)")],
+    "eq3 u-step without the gram inverse": [
+        ("    return np.linalg.solve(G + ridge(G) * np.eye(G.shape[0]), np.asarray(PU, dtype=np.float64).T).T",
+         "    return np.asarray(PU, dtype=np.float64)")],
+    "sec25 u-step gram unweighted": [("    G = gram_v(Cb, h)\n    return np.linalg.solve",
+                                      "    G = gram_v(Cb, None)\n    return np.linalg.solve")],
+    "initial columns by unweighted energy": [
+        ("energy = np.asarray(h, dtype=np.float64) * np.sum(np.asarray(R, dtype=np.float64) ** 2, axis=0)",
+         "energy = np.sum(np.asarray(R, dtype=np.float64) ** 2, axis=0)")],
+    "eq2 threshold from the largest magnitude": [("theta = tau * (math.fsum(mag.tolist()) / length)",
+                                                  "theta = tau * float(mag.max())")],
+    "deflation without the scales": [
+        ("return np.asarray(R, dtype=np.float64) - (U * np.asarray(d, dtype=np.float64)) @ np.asarray(Cb, dtype=np.float64)",
+         "return np.asarray(R, dtype=np.float64) - U @ np.asarray(Cb, dtype=np.float64)")],
+    "weighted energy over the unweighted norm of A": [
+        ("return 1.0 - weighted_norm2(A - Ahat, h) / weighted_norm2(A, h)",
+         "return 1.0 - weighted_norm2(A - Ahat, h) / weighted_norm2(A, None)")],
+    "sequential u-step on the unweighted residual": [("u = ternarize(R @ (h * v), tau)", "u = ternarize(R @ v, tau)")],
+    "eq4 r without U": [("r = np.sum(np.asarray(U, dtype=np.float64) * np.asarray(PU, dtype=np.float64), axis=0)",
+                         "r = np.sum(np.asarray(PU, dtype=np.float64), axis=0)")],
+    "eq3 ridge over the trace, not its mean": [("return EPS_REL * float(np.trace(G)) / G.shape[0]",
+                                                 "return EPS_REL * float(np.trace(G))")],
 }
 
 
