@@ -148,9 +148,9 @@ __global__ void __launch_bounds__(kTiThreads, 1) inv_tc_kernel(const float* __re
     }
   }
   // ---- stage the Gram (the integer upper triangle, or the float partials) and, for Eq. 4, G_V
-  const bool vec = (w & 3) == 0;   // rows start on 16-byte boundaries in global memory
   auto stage = [&](uint32_t* dst, const uint32_t* src) {
-    if (vec) {
+    // 16-byte copies where every row starts on a 16-byte boundary in global memory, else 4-byte ones
+    if ((w & 3) == 0 && (reinterpret_cast<uintptr_t>(src) & 15) == 0) {
       const int q4 = w >> 2;
       for (int a = warp; a < w; a += kTiThreads / 32)
         for (int c = lane; c < q4; c += 32) cp_async16(smem_addr(dst + a * kTiP + 4 * c), src + (long long)a * w + 4 * c);
